@@ -1,0 +1,281 @@
+"""Pins of the fp64 oracle to things the paper and the mathematics fix.
+
+Each test checks the oracle against something other than itself: a number
+the paper prints (tests/golden/paper_ratios.json), a closed form, a library
+routine on a special case, or a second enumeration written independently.
+"""
+import json
+import math
+import os
+from fractions import Fraction
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import brute, msp, mssa, schedule, stream
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "paper_ratios.json")
+
+
+def _golden():
+    with open(GOLDEN) as f:
+        return json.load(f)
+
+
+# ---------------------------------------------------------------- Eq. 3 --
+
+def test_eq3_rho_tok_matches_paper():
+    g = _golden()["rho_tok"]
+    scales = g["scales"]
+    # closed form of Eq. 3
+    assert float(schedule.rho_tok(scales)) == pytest.approx(g["value"], abs=1e-12)
+    # the same ratio from the enumerated token counts on the 480p grid
+    cnt = schedule.token_counts(scales, 30, 52)
+    assert cnt == [1560, 1560, 390, 390, 390]
+    assert Fraction(sum(cnt), 5 * 30 * 52) == Fraction(55, 100)
+    assert 1 - sum(cnt) / (5 * 1560) == pytest.approx(g["token_reduction"], abs=1e-12)
+
+
+@pytest.mark.parametrize("scales,gh,gw,expect", [
+    ((1, 1, 2), 8, 8, [64, 64, 16]),
+    ((1, 1, 2, 2, 4, 4), 48, 80, [3840, 3840, 960, 960, 240, 240]),
+    ((1, 1, 1, 1, 1), 30, 52, [1560] * 5),
+])
+def test_eq3_counts_and_bijective_token_index(scales, gh, gw, expect):
+    cnt = schedule.token_counts(scales, gh, gw)
+    assert cnt == expect
+    seen = set()
+    for l, s in enumerate(scales):
+        for i in range(gh // s):
+            for j in range(gw // s):
+                seen.add(schedule.token_of(scales, gh, gw, l, i, j))
+    assert seen == set(range(sum(expect)))
+
+
+def test_schedule_validation():
+    with pytest.raises(ValueError):
+        schedule.validate((1, 2, 1), 8, 8)        # not monotone
+    with pytest.raises(ValueError):
+        schedule.validate((1, 3), 6, 6)           # not a power of two
+    with pytest.raises(ValueError):
+        schedule.validate((1, 1, 2, 2, 4), 30, 52)  # 30 not divisible by 4
+    schedule.validate((1, 1, 2, 2, 2), 30, 52)
+
+
+# ---------------------------------------------------------------- Eq. 5 --
+
+def test_eq5_pair_reduction_matches_paper():
+    g = _golden()["r_mssa"]
+    scales, gh, gw = g["scales"], 30, 52
+    G = gh * gw
+    # one sink frame at full resolution = G sink tokens; one history frame
+    pairs = schedule.attention_pairs(scales, gh, gw, G * g["sink_frames"], g["history_frames"])
+    dense = schedule.msp_only_pairs(scales, gh, gw, G * g["sink_frames"], g["history_frames"])
+    r_enum = 1 - Fraction(pairs, dense)
+    r_eq5 = schedule.r_mssa_eq5(scales, g["sink_frames"], g["history_frames"])
+    # enumeration of Eq. 4 contexts and the closed form of Eq. 5 agree exactly
+    assert r_enum == r_eq5
+    # and round to the paper's printed 12.9%
+    assert round(float(r_enum), g["printed_digits"]) == pytest.approx(g["value"], abs=1e-12)
+
+
+def test_eq5_other_layouts_enum_vs_closed_form():
+    for scales, gh, gw, nh in [((1, 1, 2, 2, 4, 4), 48, 80, 2), ((1, 2), 4, 4, 3),
+                               ((2, 2, 4), 8, 8, 1), ((1, 1, 1), 4, 6, 2)]:
+        G = gh * gw
+        pairs = schedule.attention_pairs(scales, gh, gw, G, nh)
+        dense = schedule.msp_only_pairs(scales, gh, gw, G, nh)
+        assert 1 - Fraction(pairs, dense) == schedule.r_mssa_eq5(scales, 1, nh)
+    # an all-fine schedule removes nothing
+    assert schedule.r_mssa_eq5((1, 1, 1, 1, 1), 1, 1) == 0
+
+
+def test_cfg1_flops():
+    # 480p layer: 3120 x 8970 + 1170 x 4290 pairs per head, 12 heads, D = 128
+    pairs = schedule.attention_pairs((1, 1, 2, 2, 2), 30, 52, 1560, 2)
+    assert pairs == 3120 * 8970 + 1170 * 4290
+    fl = schedule.attention_flops((1, 1, 2, 2, 2), 30, 52, 1560, 2, 12, 128)
+    assert fl == 4 * 128 * 12 * pairs
+    assert fl / 1e9 == pytest.approx(202.79, abs=0.01)
+
+
+# ------------------------------------------------------------- resample --
+
+@pytest.mark.parametrize("mode", [mssa.AVG, mssa.STRIDED])
+@pytest.mark.parametrize("sigma", [1, 2, 4])
+def test_resample_constant_field_is_identity(mode, sigma):
+    x = np.full((2, 8 * 12, 3, 5), 0.375)
+    y = mssa.resample(x, 8, 12, sigma, mode)
+    assert y.shape == (2, (8 // sigma) * (12 // sigma), 3, 5)
+    assert np.all(y == 0.375)
+
+
+@pytest.mark.parametrize("sigma", [2, 4])
+def test_resample_linear_ramp(sigma):
+    gh, gw = 8, 16
+    a, b, c = 0.7, -1.3, 2.0
+    i, j = np.meshgrid(np.arange(gh), np.arange(gw), indexing="ij")
+    x = (a * i + b * j + c).reshape(1, gh * gw, 1, 1)
+    oi, oj = np.meshgrid(np.arange(gh // sigma), np.arange(gw // sigma), indexing="ij")
+    centre = a * (sigma * oi + (sigma - 1) / 2) + b * (sigma * oj + (sigma - 1) / 2) + c
+    corner = a * (sigma * oi) + b * (sigma * oj) + c
+    avg = mssa.resample(x, gh, gw, sigma, mssa.AVG).reshape(gh // sigma, gw // sigma)
+    st = mssa.resample(x, gh, gw, sigma, mssa.STRIDED).reshape(gh // sigma, gw // sigma)
+    np.testing.assert_allclose(avg, centre, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(st, corner, rtol=0, atol=0)
+
+
+def test_resample_mean_is_block_mean_by_library_reshape():
+    rng = np.random.default_rng(3)
+    x = rng.standard_normal((2, 8 * 12, 2, 4))
+    y = mssa.resample(x, 8, 12, 4, mssa.AVG)
+    ref = x.reshape(2, 2, 4, 3, 4, 2, 4).mean(axis=(2, 4)).reshape(2, 6, 2, 4)
+    np.testing.assert_allclose(y, ref, rtol=0, atol=1e-13)
+
+
+# ------------------------------------------------------------ attention --
+
+def _rand_inputs(rng, scales, gh, gw, ns, nh, H, D, B=1):
+    N = sum(schedule.token_counts(scales, gh, gw))
+    G = gh * gw
+    return dict(
+        q=rng.standard_normal((B, N, H, D)), k_win=rng.standard_normal((B, N, H, D)),
+        v_win=rng.standard_normal((B, N, H, D)), k_sink=rng.standard_normal((B, ns, H, D)),
+        v_sink=rng.standard_normal((B, ns, H, D)), k_hist=rng.standard_normal((B, nh, G, H, D)),
+        v_hist=rng.standard_normal((B, nh, G, H, D)))
+
+
+def test_all_fine_reduces_to_plain_attention_sdpa():
+    rng = np.random.default_rng(0)
+    scales, gh, gw = (1, 1, 1), 4, 6
+    x = _rand_inputs(rng, scales, gh, gw, ns=5, nh=2, H=3, D=16, B=2)
+    out = mssa.mssa_forward(x["q"], x["k_win"], x["v_win"], x["k_sink"], x["v_sink"],
+                            x["k_hist"], x["v_hist"], scales, gh, gw)
+    B, N, H, D = x["q"].shape
+    kh = x["k_hist"].reshape(B, -1, H, D)
+    vh = x["v_hist"].reshape(B, -1, H, D)
+    K = np.concatenate([x["k_sink"], kh, x["k_win"]], axis=1)
+    V = np.concatenate([x["v_sink"], vh, x["v_win"]], axis=1)
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a.transpose(0, 2, 1, 3)))
+    ref = torch.nn.functional.scaled_dot_product_attention(t(x["q"]), t(K), t(V))
+    np.testing.assert_allclose(out, ref.numpy().transpose(0, 2, 1, 3), rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("mode", [mssa.AVG, mssa.STRIDED])
+@pytest.mark.parametrize("scales,gh,gw,ns,nh", [
+    ((1, 2), 4, 4, 3, 1),
+    ((1, 2, 4), 4, 8, 2, 2),
+    ((1, 1, 2), 8, 8, 64, 1),     # the tiny workload's grid and schedule
+    ((2, 2, 4), 4, 8, 1, 1),      # no fine state at all
+])
+def test_brute_force_eq4(mode, scales, gh, gw, ns, nh):
+    rng = np.random.default_rng(11)
+    x = _rand_inputs(rng, scales, gh, gw, ns, nh, H=2, D=6)
+    out = mssa.mssa_forward(x["q"], x["k_win"], x["v_win"], x["k_sink"], x["v_sink"],
+                            x["k_hist"], x["v_hist"], scales, gh, gw, mode=mode)
+    ref = brute.mssa_brute(x["q"].tolist(), x["k_win"].tolist(), x["v_win"].tolist(),
+                           x["k_sink"].tolist(), x["v_sink"].tolist(), x["k_hist"].tolist(),
+                           x["v_hist"].tolist(), scales, gh, gw, mode=mode)
+    np.testing.assert_allclose(out, np.array(ref), rtol=0, atol=1e-12)
+
+
+def test_equal_keys_give_weighted_value_mean():
+    """All keys equal -> uniform softmax -> o = mean of the context values.
+    For AVG pooling a frame pooled by s contributes (1/s^2) * (sum of its fine
+    values) over (G/s^2) rows; the closed form below never builds a context."""
+    rng = np.random.default_rng(5)
+    scales, gh, gw, ns, nh = (1, 2, 4), 8, 8, 7, 2
+    x = _rand_inputs(rng, scales, gh, gw, ns, nh, H=2, D=3)
+    for key in ("k_win", "k_sink", "k_hist"):
+        x[key] = np.ones_like(x[key]) * 0.25
+    out = mssa.mssa_forward(x["q"], x["k_win"], x["v_win"], x["k_sink"], x["v_sink"],
+                            x["k_hist"], x["v_hist"], scales, gh, gw)
+    G = gh * gw
+    cnt = [G // (s * s) for s in scales]
+    offs = np.cumsum([0] + cnt)
+    for l, g in enumerate(scales):
+        num = x["v_sink"][0].sum(axis=0)
+        den = ns
+        for f in range(nh):
+            num = num + x["v_hist"][0, f].sum(axis=0) / (g * g)
+            den += G // (g * g)
+        for m, s in enumerate(scales):
+            st = max(1, g // s)
+            num = num + x["v_win"][0, offs[m]:offs[m + 1]].sum(axis=0) / (st * st)
+            den += cnt[m] // (st * st)
+        expect = num / den
+        got = out[0, offs[l]:offs[l + 1]]
+        np.testing.assert_allclose(got, np.broadcast_to(expect, got.shape), rtol=0, atol=1e-12)
+
+
+def test_permutation_invariance_and_convexity():
+    rng = np.random.default_rng(7)
+    scales, gh, gw, ns, nh = (1, 1, 2), 8, 8, 9, 2
+    x = _rand_inputs(rng, scales, gh, gw, ns, nh, H=2, D=8)
+    args = lambda d: (d["q"], d["k_win"], d["v_win"], d["k_sink"], d["v_sink"], d["k_hist"],
+                      d["v_hist"], scales, gh, gw)
+    out = mssa.mssa_forward(*args(x))
+    perm = rng.permutation(ns)
+    y = dict(x)
+    y["k_sink"] = x["k_sink"][:, perm]
+    y["v_sink"] = x["v_sink"][:, perm]
+    y["k_hist"] = x["k_hist"][:, ::-1]
+    y["v_hist"] = x["v_hist"][:, ::-1]
+    np.testing.assert_allclose(mssa.mssa_forward(*args(y)), out, rtol=0, atol=1e-12)
+    allv = np.concatenate([x["v_sink"], x["v_hist"].reshape(1, -1, 2, 8), x["v_win"]], axis=1)
+    lo, hi = allv.min(axis=1, keepdims=True), allv.max(axis=1, keepdims=True)
+    assert np.all(out >= lo - 1e-12) and np.all(out <= hi + 1e-12)
+
+
+def test_softmax_scale_default_is_inverse_sqrt_d():
+    rng = np.random.default_rng(9)
+    q = rng.standard_normal((1, 3, 1, 16))
+    k = rng.standard_normal((1, 5, 1, 16))
+    v = rng.standard_normal((1, 5, 1, 16))
+    o = mssa.attention(q, k, v, 0.25)
+    s = q[0, :, 0] @ k[0, :, 0].T / math.sqrt(16)
+    p = np.exp(s) / np.exp(s).sum(axis=1, keepdims=True)
+    np.testing.assert_allclose(o[0, :, 0], p @ v[0, :, 0], rtol=0, atol=1e-13)
+
+
+# ------------------------------------------------------------------ MSP --
+
+@pytest.mark.parametrize("P", [1, 2, 4, 8])
+def test_patchify_roundtrip_and_library_reshape(P):
+    rng = np.random.default_rng(P)
+    B, C, Hl, Wl = 2, 3, 16, 24
+    x = rng.standard_normal((B, C, Hl, Wl))
+    t = msp.patchify(x, P)
+    gh, gw = Hl // P, Wl // P
+    ref = x.reshape(B, C, gh, P, gw, P).transpose(0, 2, 4, 1, 3, 5).reshape(B, gh * gw, C * P * P)
+    assert np.array_equal(t, ref)
+    assert np.array_equal(msp.unpatchify(t, P, C, Hl, Wl), x)
+
+
+def test_patch_embedding_equals_strided_conv():
+    """Tier embedding of (c, dy, dx)-ordered patches == Conv2d with kernel = stride = P."""
+    rng = np.random.default_rng(1)
+    B, C, Hl, Wl, P, E = 1, 4, 8, 12, 2, 5
+    x = rng.standard_normal((B, C, Hl, Wl))
+    W = rng.standard_normal((C * P * P, E))
+    emb = msp.patchify(x, P) @ W
+    conv = torch.nn.functional.conv2d(torch.from_numpy(x),
+                                      torch.from_numpy(W.T.reshape(E, C, P, P).copy()), stride=P)
+    ref = conv.numpy().reshape(B, E, -1).transpose(0, 2, 1)
+    np.testing.assert_allclose(emb, ref, rtol=0, atol=1e-12)
+
+
+# ------------------------------------------------------------ streaming --
+
+def test_history_ring_keeps_newest_frames():
+    B, G, H, D, cap = 1, 4, 1, 2, 4
+    h0 = np.stack([np.full((B, G, H, D), f) for f in range(2)], axis=1)
+    hist = stream.History(h0, h0 + 100, cap)
+    for f in range(2, 9):
+        hist.append(np.full((B, G, H, D), f), np.full((B, G, H, D), f + 100))
+        k, v = hist.frames()
+        assert k.shape[1] == min(cap, f + 1)
+        live = sorted(int(k[0, s, 0, 0, 0]) for s in range(k.shape[1]))
+        assert live == list(range(max(0, f + 1 - cap), f + 1))
+        assert np.all(v == k + 100)
