@@ -1,0 +1,232 @@
+/*
+ * msf.h - C ABI of the Ms. Forcing multi-scale window pass on one GB300.
+ *
+ * The library computes, for one rolling denoising window (Sec. 3.1, Eq. 2):
+ *   - Multi-Scale Patchification (MSP, Sec. 4.1, Eq. 3): latent states are
+ *     cut into patches of size p_l = s_l * p, coarser for noisier positions;
+ *   - the per-scale key/value pyramid that Eq. 4's Subsample() needs;
+ *   - Multi-Scale Self-Attention (MSSA, Sec. 4.1, Eq. 4): queries of scale g
+ *     attend to the full-resolution sink, then to every history frame and
+ *     every window state, each subsampled by max(1, g / s_b);
+ *   - the history-cache update after a pass (Algorithm 1, KV update with the
+ *     emitted head state).
+ *
+ * Conventions shared by every call:
+ *   - Every call returns msf_status; MSF_OK is 0. Argument and state errors
+ *     are reported synchronously, before anything is launched.
+ *   - The library never allocates device memory. The caller owns every
+ *     device buffer, including the workspace whose size msf_plan_query
+ *     reports. The library owns only the opaque host-side plan.
+ *   - Device pointers must be 16-byte aligned. Tensors are contiguous,
+ *     row-major, with the last index fastest.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream). Kernels run asynchronously on it; outputs are valid once the
+ *     stream has reached the call.
+ *   - Element type is the plan's dtype (bf16 or fp32) for every tensor.
+ *   - Notation: B streams, T window states, fine token grid Gh x Gw
+ *     (G = Gh*Gw tokens per fine frame), H heads, D head_dim, Ns sink tokens,
+ *     N = sum_l G / s_l^2 window tokens (Eq. 3), E = embedding width.
+ */
+#ifndef MSF_H
+#define MSF_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum msf_status {
+    MSF_OK = 0,
+    MSF_ERR_INVALID_ARG = 1,  /* null/misaligned pointer, bad size, bad index */
+    MSF_ERR_UNSUPPORTED = 2,  /* a schedule or shape outside what is built */
+    MSF_ERR_CUDA = 3,         /* a CUDA runtime call failed; see msf_last_cuda_error */
+    MSF_ERR_TIMEOUT = 4,      /* a device-side wait hit its bound (kernel returned early) */
+    MSF_ERR_STATE = 5,        /* plan not bound, or history operation not allowed */
+    MSF_ERR_WORKSPACE = 6     /* workspace smaller than msf_plan_query reports */
+} msf_status;
+
+typedef enum msf_dtype { MSF_DTYPE_BF16 = 0, MSF_DTYPE_F32 = 1 } msf_dtype;
+
+/* Eq. 4's Subsample(C_b, stride): AVG takes the mean of each stride x stride
+ * block (the coarse-token proxy of the MSP probe, Sec. 3.2); STRIDED keeps the
+ * block's top-left token (the stride-2 key/value subsampling of the MSSA
+ * probe, Sec. 3.2). */
+typedef enum msf_resample_mode { MSF_RESAMPLE_AVG = 0, MSF_RESAMPLE_STRIDED = 1 } msf_resample_mode;
+
+/* msf_kv_resample flags. */
+#define MSF_RESAMPLE_FULL 0         /* pool history frames and window states */
+#define MSF_RESAMPLE_WINDOW_ONLY 1  /* window states only; history pyramid is kept
+                                       up to date by msf_history_append */
+
+#define MSF_MAX_STATES 16
+#define MSF_MAX_GROUPS 8
+
+/* Static schedule and shapes (Sec. 4.1: p_1 <= ... <= p_T, p_l in {p,2p,4p,...}). */
+typedef struct msf_plan_desc {
+    int32_t T;                        /* window states, 1..MSF_MAX_STATES */
+    int32_t scales[MSF_MAX_STATES];   /* s_l = p_l / p: powers of two, non-decreasing */
+    int32_t grid_h, grid_w;           /* fine token grid; divisible by max s_l */
+    int32_t heads;                    /* H >= 1 */
+    int32_t head_dim;                 /* D: 64 or 128 */
+    int32_t sink_tokens;              /* Ns >= 0, never resampled */
+    int32_t history_frames;           /* live history frames at bind time */
+    int32_t history_capacity;         /* ring capacity (>= history_frames) */
+    int32_t batch;                    /* B independent streams */
+    int32_t dtype;                    /* msf_dtype */
+    int32_t resample;                 /* msf_resample_mode */
+    float softmax_scale;              /* 0 -> 1/sqrt(D) */
+    int32_t latent_channels;          /* C of the latent (patchify); 0 if unused */
+    int32_t patch;                    /* native patch p in latent pixels; 0 if unused */
+    int32_t embed_dim;                /* E of the tier projections; 0 = raw tokens only */
+} msf_plan_desc;
+
+typedef struct msf_group_info {
+    int32_t scale;        /* g: scale shared by this group's query states */
+    int32_t q_begin;      /* first query token (window order) */
+    int32_t q_end;        /* one past the last */
+    int32_t n_kv;         /* context length Nkv_g with the current history count */
+    int32_t n_pyramid;    /* tokens of the resampled part (history@g + finer states) */
+    int32_t pyr_offset;   /* token offset of that part in the workspace pyramid, -1 if g==1 */
+} msf_group_info;
+
+typedef struct msf_plan_info {
+    int32_t T;
+    int32_t n_tokens;                 /* N = N_MSP (Eq. 3) */
+    int32_t n_tokens_fine;            /* T * G (all-fine window, N_RF of Eq. 3) */
+    int32_t fine_tokens;              /* G */
+    int32_t state_offset[MSF_MAX_STATES];
+    int32_t state_tokens[MSF_MAX_STATES];
+    int32_t state_grid_h[MSF_MAX_STATES];
+    int32_t state_grid_w[MSF_MAX_STATES];
+    int32_t n_groups;
+    msf_group_info groups[MSF_MAX_GROUPS];
+    int32_t history_count;            /* live frames in the history ring */
+    int32_t history_next_slot;        /* slot the next msf_history_append writes */
+    int32_t pyramid_tokens;           /* tokens per stream in the workspace pyramid */
+    int32_t _pad;
+    uint64_t workspace_bytes;         /* device workspace msf_plan_bind needs */
+    uint64_t attention_flops;         /* 4*D*H*B*sum_g Nq_g*Nkv_g (current history) */
+    uint64_t dense_flops;             /* same window with every s_l = 1 (no MSP, no MSSA) */
+    uint64_t resample_bytes;          /* bytes read+written by a full msf_kv_resample */
+    uint64_t pyramid_k_offset;        /* byte offset of the K pyramid [B, pyramid_tokens, H, D]
+                                         inside the workspace */
+    uint64_t pyramid_v_offset;        /* byte offset of the V pyramid */
+} msf_plan_info;
+
+typedef struct msf_plan* msf_plan_t;
+
+/* Human-readable name of a status code. Never NULL. */
+const char* msf_status_string(msf_status s);
+
+/* The last cudaError_t value seen by a call that returned MSF_ERR_CUDA
+ * (thread-local; 0 if none). */
+int msf_last_cuda_error(void);
+
+/* Validate `desc` and build the static schedule tables (Eq. 3 token counts,
+ * Eq. 4 query groups and context layout). Host only; no CUDA call.
+ * Errors: INVALID_ARG (null pointers, non-positive sizes), UNSUPPORTED
+ * (non-monotone or non-power-of-two scales, grid not divisible by max s_l,
+ * head_dim not 64/128, too many groups). On success *out owns a plan that
+ * msf_plan_destroy frees. */
+msf_status msf_plan_create(const msf_plan_desc* desc, msf_plan_t* out);
+
+/* Free a plan. NULL-safe. Device buffers stay the caller's. */
+void msf_plan_destroy(msf_plan_t plan);
+
+/* Fill `info` (host memory) with the plan's tables and sizes. Host only. */
+msf_status msf_plan_query(msf_plan_t plan, msf_plan_info* info);
+
+/* Enumerate the context rows of query group `group` in the order the kernels
+ * and the oracle use (Eq. 4: sink, history frames in slot order, window
+ * states 1..T). Each row is 5 int32: kind (0 sink, 1 history, 2 window),
+ * frame (history slot or window position, 0-based), stride (the Subsample
+ * stride applied to that frame), row, col (on the pooled grid; for the sink
+ * row = sink token, col = 0). Writes at most `cap_rows` rows to `out` (host
+ * memory, may be NULL when cap_rows is 0) and sets *n_rows to the total.
+ * Host only. */
+msf_status msf_plan_index_map(msf_plan_t plan, int32_t group, int32_t* out, size_t cap_rows,
+                              size_t* n_rows);
+
+/* Attach device buffers that persist across passes:
+ *   workspace  >= info.workspace_bytes bytes (status word + per-scale pyramid)
+ *   k_sink, v_sink [B, Ns, H, D]           (read only, never resampled)
+ *   k_hist, v_hist [B, capacity, G, H, D]  history ring, fine scale; the first
+ *                                          history_frames slots hold live frames
+ * Resets the history count to desc.history_frames and zeroes the device status
+ * word (a cudaMemsetAsync on the legacy stream, completed before returning).
+ * Builds the TMA descriptors for the bound buffers. Errors: INVALID_ARG,
+ * WORKSPACE, CUDA. */
+msf_status msf_plan_bind(msf_plan_t plan, void* workspace, size_t workspace_bytes,
+                         const void* k_sink, const void* v_sink, void* k_hist, void* v_hist);
+
+/* MSP patchify (Sec. 4.1). latent [B, T, C, Hl, Wl] with Hl = patch*Gh,
+ * Wl = patch*Gw. Token (i, j) of state l has feature c*P^2 + dy*P + dx =
+ * latent[b, l, c, P*i + dy, P*j + dx], P = patch * s_l.
+ *   w_tier == NULL: tokens is the raw layout [B, T, C*Hl*Wl]; state l's block
+ *                   is [G/s_l^2, C*P^2] (a permutation of its latent).
+ *   w_tier != NULL: array of T device pointers, w_tier[l] = the tier's
+ *                   patch-embedding weight [E, C*P^2] (the Conv2d weight
+ *                   [E, C, P, P] flattened); tokens is [B, N, E] and
+ *                   row off_l + i*gw_l + j holds sum_f patch[f] * w[e, f]
+ *                   (fp32 accumulation, one rounding to the dtype).
+ * Errors: INVALID_ARG, UNSUPPORTED (no latent_channels/patch, or E == 0 with
+ * weights), CUDA. */
+msf_status msf_patchify(msf_plan_t plan, const void* latent, const void* const* w_tier,
+                        void* tokens, void* stream);
+
+/* MSP unpatchify of window position `position` (0-based): the inverse of
+ * msf_patchify for that state.
+ *   w_out == NULL: tokens is the raw layout [B, T, C*Hl*Wl] of msf_patchify.
+ *   w_out != NULL: tokens is [B, N, E] (for example the attention output viewed
+ *                  as [B, N, H*D]); rows of the state are de-embedded by
+ *                  w_out [C*P^2, E] (the nn.Linear weight E -> C*P^2) with fp32
+ *                  accumulation, then rearranged.
+ * latent_out [B, C, Hl, Wl]. Errors: INVALID_ARG, UNSUPPORTED, CUDA. */
+msf_status msf_unpatchify(msf_plan_t plan, int32_t position, const void* tokens,
+                          const void* w_out, void* latent_out, void* stream);
+
+/* Build the per-scale key/value pyramid in the workspace: for every query
+ * group g > 1, the bound history frames (fine, pooled by g) and the window
+ * states with s_l < g (pooled by g/s_l), from k_win, v_win [B, N, H, D].
+ * Pooling is the plan's Subsample mode; AVG sums in fp32 and rounds once.
+ * flags: MSF_RESAMPLE_FULL or MSF_RESAMPLE_WINDOW_ONLY. Errors: INVALID_ARG,
+ * STATE (not bound), CUDA. */
+msf_status msf_kv_resample(msf_plan_t plan, const void* k_win, const void* v_win, int32_t flags,
+                           void* stream);
+
+/* MSSA (Eq. 4): out[b, t, h, :] = sum_j softmax_j(scale * q[b,t,h,:] . K_g[j]) V_g[j]
+ * over the context of t's group g (sink, history, window; no mask).
+ * q, k_win, v_win, out [B, N, H, D]; out may not alias q/k/v. Reads the
+ * pyramid the last msf_kv_resample on the same stream produced. bf16 plans
+ * run the tcgen05 tensor-core kernel (bf16 operands, fp32 softmax and
+ * accumulation); fp32 plans run an fp32 CUDA-core kernel. Errors:
+ * INVALID_ARG, STATE, CUDA. */
+msf_status msf_mssa_forward(msf_plan_t plan, const void* q, const void* k_win, const void* v_win,
+                            void* out, void* stream);
+
+/* Same computation always on the fp32 CUDA-core kernel (a cross-check of the
+ * tensor-core kernel for bf16 plans). */
+msf_status msf_mssa_forward_simt(msf_plan_t plan, const void* q, const void* k_win,
+                                 const void* v_win, void* out, void* stream);
+
+/* History-cache update after a pass (Algorithm 1): copy the head state's fine
+ * K/V (window position 0, tokens [0, G)) into the ring slot
+ * info.history_next_slot (the next free slot, else the oldest frame), and
+ * pool it into that slot of every coarser pyramid level. Advances the
+ * host-side count/slot state. Errors: STATE (not bound, capacity 0, or
+ * s_1 != 1), INVALID_ARG, CUDA. */
+msf_status msf_history_append(msf_plan_t plan, const void* k_win, const void* v_win,
+                              void* stream);
+
+/* Synchronise `stream`, read and clear the device status word. Returns
+ * MSF_ERR_TIMEOUT if a kernel gave up on a bounded wait since the last
+ * check, MSF_OK otherwise. */
+msf_status msf_plan_device_status(msf_plan_t plan, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MSF_H */

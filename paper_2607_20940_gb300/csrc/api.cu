@@ -1,0 +1,387 @@
+// C ABI entry points that touch the device: binding, MSP, KV pyramid,
+// attention, history update, device status.
+#include <cuda_runtime.h>
+#include <string.h>
+
+#include "attn_tc.h"
+#include "internal.h"
+#include "kernels.h"
+
+using msf::Plan;
+
+namespace {
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+msf_status cuda_status(cudaError_t e) {
+    if (e == cudaSuccess) return MSF_OK;
+    msf::set_cuda_error((int)e);
+    return MSF_ERR_CUDA;
+}
+
+size_t row_bytes(const Plan& p) { return (size_t)p.H * p.D * p.elem; }
+
+// Jobs that pool the history frames (full mode) and the window states finer
+// than each group's scale into that group's pyramid part.
+void add_window_jobs(const Plan& p, const void* k_win, const void* v_win, bool with_history,
+                     msf::PoolBatch& jb) {
+    const size_t row = row_bytes(p);
+    const long long win_bs = (long long)p.N * row;
+    const long long hist_bs = (long long)p.d.history_capacity * p.G * row;
+    const long long pyr_bs = (long long)p.pyr_tokens * row;
+    for (int gi = 0; gi < p.n_groups; ++gi) {
+        const msf::Group& g = p.groups[gi];
+        if (g.scale == 1) continue;
+        if (with_history) {
+            for (int f = 0; f < p.hist_count; ++f) {
+                msf::PoolJob& j = jb.j[jb.n++];
+                size_t so = (size_t)f * p.G * row;
+                size_t dof = (size_t)(g.pyr_offset + f * g.pooled) * row;
+                j.src_k = (const char*)p.k_hist + so;
+                j.src_v = (const char*)p.v_hist + so;
+                j.dst_k = msf::pyr_k(p) + dof;
+                j.dst_v = msf::pyr_v(p) + dof;
+                j.src_bstride = hist_bs;
+                j.dst_bstride = pyr_bs;
+                j.src_gw = p.d.grid_w;
+                j.out_gw = p.d.grid_w / g.scale;
+                j.out_n = g.pooled;
+                j.sigma = g.scale;
+            }
+        }
+        for (int l = 0; l < g.n_finer; ++l) {
+            msf::PoolJob& j = jb.j[jb.n++];
+            size_t so = (size_t)p.st_off[l] * row;
+            size_t dof = (size_t)(g.pyr_offset + (p.hist_count + l) * g.pooled) * row;
+            j.src_k = (const char*)k_win + so;
+            j.src_v = (const char*)v_win + so;
+            j.dst_k = msf::pyr_k(p) + dof;
+            j.dst_v = msf::pyr_v(p) + dof;
+            j.src_bstride = win_bs;
+            j.dst_bstride = pyr_bs;
+            j.src_gw = p.st_gw[l];
+            j.out_gw = p.d.grid_w / g.scale;
+            j.out_n = g.pooled;
+            j.sigma = g.scale / p.d.scales[l];
+        }
+    }
+}
+
+int count_window_jobs(const Plan& p, bool with_history) {
+    int n = 0;
+    for (int gi = 0; gi < p.n_groups; ++gi) {
+        const msf::Group& g = p.groups[gi];
+        if (g.scale == 1) continue;
+        n += g.n_finer + (with_history ? p.hist_count : 0);
+    }
+    return n;
+}
+
+// The context segments of every query group (Eq. 4 order: sink, history,
+// window), pointing at the bound buffers, the pyramid and k_win/v_win.
+void build_attn_args(const Plan& p, const void* q, const void* k_win, const void* v_win,
+                     void* out, msf::AttnArgs& a) {
+    memset(&a, 0, sizeof(a));
+    const size_t row = row_bytes(p);
+    a.q = (const char*)q;
+    a.out = (char*)out;
+    a.q_bstride = (long long)p.N * row;
+    a.H = p.H;
+    a.D = p.D;
+    a.B = p.B;
+    a.scale_log2 = p.scale * 1.4426950408889634f;
+    a.n_groups = p.n_groups;
+    a.status = msf::status_word(p);
+    for (int gi = 0; gi < p.n_groups; ++gi) {
+        const msf::Group& g = p.groups[gi];
+        msf::AttnGroup& ag = a.g[gi];
+        ag.q_begin = g.q_begin;
+        ag.q_end = g.q_end;
+        int ns = 0;
+        if (p.d.sink_tokens > 0) {
+            msf::Segment& s = ag.seg[ns++];
+            s.k = (const char*)p.k_sink;
+            s.v = (const char*)p.v_sink;
+            s.bstride = (long long)p.d.sink_tokens * row;
+            s.row0 = 0;
+            s.len = p.d.sink_tokens;
+            s.rows_total = p.d.sink_tokens;
+            s.map_id = msf::kMapSink;
+        }
+        if (g.scale == 1) {
+            if (p.hist_count > 0) {
+                msf::Segment& s = ag.seg[ns++];
+                s.k = (const char*)p.k_hist;
+                s.v = (const char*)p.v_hist;
+                s.bstride = (long long)p.d.history_capacity * p.G * row;
+                s.row0 = 0;
+                s.len = p.hist_count * p.G;
+                s.rows_total = p.d.history_capacity * p.G;
+                s.map_id = msf::kMapHist;
+            }
+        } else {
+            int n = msf::group_npyr(p, gi);
+            if (n > 0) {
+                msf::Segment& s = ag.seg[ns++];
+                s.k = msf::pyr_k(p);
+                s.v = msf::pyr_v(p);
+                s.bstride = (long long)p.pyr_tokens * row;
+                s.row0 = g.pyr_offset;
+                s.len = n;
+                s.rows_total = p.pyr_tokens;
+                s.map_id = msf::kMapPyr;
+            }
+        }
+        {
+            msf::Segment& s = ag.seg[ns++];
+            s.k = (const char*)k_win;
+            s.v = (const char*)v_win;
+            s.bstride = (long long)p.N * row;
+            s.row0 = g.q_begin;
+            s.len = p.N - g.q_begin;
+            s.rows_total = p.N;
+            s.map_id = msf::kMapWin;
+        }
+        ag.n_seg = ns;
+    }
+}
+
+}  // namespace
+
+extern "C" void msf_plan_destroy_caches(msf_plan_t plan) { msf::tc_cache_free(plan); }
+
+extern "C" msf_status msf_plan_bind(msf_plan_t plan, void* workspace, size_t workspace_bytes,
+                                    const void* k_sink, const void* v_sink, void* k_hist,
+                                    void* v_hist) {
+    if (!plan || !workspace) return MSF_ERR_INVALID_ARG;
+    Plan& p = *plan;
+    if (workspace_bytes < p.ws_bytes) return MSF_ERR_WORKSPACE;
+    if (!aligned16(workspace)) return MSF_ERR_INVALID_ARG;
+    if (p.d.sink_tokens > 0 && (!k_sink || !v_sink || !aligned16(k_sink) || !aligned16(v_sink)))
+        return MSF_ERR_INVALID_ARG;
+    if (p.d.history_capacity > 0 &&
+        (!k_hist || !v_hist || !aligned16(k_hist) || !aligned16(v_hist)))
+        return MSF_ERR_INVALID_ARG;
+    p.ws = workspace;
+    p.ws_size = workspace_bytes;
+    p.k_sink = k_sink;
+    p.v_sink = v_sink;
+    p.k_hist = k_hist;
+    p.v_hist = v_hist;
+    p.hist_count = p.d.history_frames;
+    p.hist_oldest = 0;
+    p.bound = true;
+    msf::tc_cache_invalidate(plan);
+    cudaError_t e = cudaMemset(msf::status_word(p), 0, msf::kStatusBytes);
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    return cuda_status(e);
+}
+
+extern "C" msf_status msf_kv_resample(msf_plan_t plan, const void* k_win, const void* v_win,
+                                      int32_t flags, void* stream) {
+    if (!plan || !k_win || !v_win) return MSF_ERR_INVALID_ARG;
+    const Plan& p = *plan;
+    if (!p.bound) return MSF_ERR_STATE;
+    if (!aligned16(k_win) || !aligned16(v_win)) return MSF_ERR_INVALID_ARG;
+    if (flags != MSF_RESAMPLE_FULL && flags != MSF_RESAMPLE_WINDOW_ONLY) return MSF_ERR_INVALID_ARG;
+    const bool with_hist = flags == MSF_RESAMPLE_FULL;
+    if (count_window_jobs(p, with_hist) > msf::kMaxPoolJobs) return MSF_ERR_UNSUPPORTED;
+    msf::PoolBatch jb;
+    memset(&jb, 0, sizeof(jb));
+    jb.row_vecs = (int)(row_bytes(p) / 16);
+    jb.mode = p.d.resample;
+    add_window_jobs(p, k_win, v_win, with_hist, jb);
+    return cuda_status(msf::launch_pool(jb, p.B, p.elem == 2, (cudaStream_t)stream));
+}
+
+extern "C" msf_status msf_history_append(msf_plan_t plan, const void* k_win, const void* v_win,
+                                         void* stream) {
+    if (!plan || !k_win || !v_win) return MSF_ERR_INVALID_ARG;
+    Plan& p = *plan;
+    if (!p.bound || p.d.history_capacity == 0 || p.d.scales[0] != 1) return MSF_ERR_STATE;
+    if (!aligned16(k_win) || !aligned16(v_win)) return MSF_ERR_INVALID_ARG;
+    const int slot = p.hist_count < p.d.history_capacity ? p.hist_count : p.hist_oldest;
+    const size_t row = row_bytes(p);
+    msf::PoolBatch jb;
+    memset(&jb, 0, sizeof(jb));
+    jb.row_vecs = (int)(row / 16);
+    jb.mode = p.d.resample;
+    {
+        // the head state (position 1, fine) into its ring slot
+        msf::PoolJob& j = jb.j[jb.n++];
+        j.src_k = (const char*)k_win;
+        j.src_v = (const char*)v_win;
+        j.dst_k = (char*)p.k_hist + (size_t)slot * p.G * row;
+        j.dst_v = (char*)p.v_hist + (size_t)slot * p.G * row;
+        j.src_bstride = (long long)p.N * row;
+        j.dst_bstride = (long long)p.d.history_capacity * p.G * row;
+        j.src_gw = p.d.grid_w;
+        j.out_gw = p.d.grid_w;
+        j.out_n = p.G;
+        j.sigma = 1;
+    }
+    for (int gi = 0; gi < p.n_groups; ++gi) {
+        const msf::Group& g = p.groups[gi];
+        if (g.scale == 1) continue;
+        // and, pooled, into the same slot of every coarser level
+        msf::PoolJob& j = jb.j[jb.n++];
+        size_t dof = (size_t)(g.pyr_offset + slot * g.pooled) * row;
+        j.src_k = (const char*)k_win;
+        j.src_v = (const char*)v_win;
+        j.dst_k = msf::pyr_k(p) + dof;
+        j.dst_v = msf::pyr_v(p) + dof;
+        j.src_bstride = (long long)p.N * row;
+        j.dst_bstride = (long long)p.pyr_tokens * row;
+        j.src_gw = p.d.grid_w;
+        j.out_gw = p.d.grid_w / g.scale;
+        j.out_n = g.pooled;
+        j.sigma = g.scale;
+    }
+    msf_status st = cuda_status(msf::launch_pool(jb, p.B, p.elem == 2, (cudaStream_t)stream));
+    if (st != MSF_OK) return st;
+    if (p.hist_count < p.d.history_capacity) {
+        ++p.hist_count;
+    } else {
+        p.hist_oldest = (p.hist_oldest + 1) % p.d.history_capacity;
+    }
+    return MSF_OK;
+}
+
+static msf_status check_attn_args(const Plan& p, const void* q, const void* k_win,
+                                  const void* v_win, void* out) {
+    if (!q || !k_win || !v_win || !out) return MSF_ERR_INVALID_ARG;
+    if (!p.bound) return MSF_ERR_STATE;
+    if (!aligned16(q) || !aligned16(k_win) || !aligned16(v_win) || !aligned16(out))
+        return MSF_ERR_INVALID_ARG;
+    if (out == q || out == k_win || out == v_win) return MSF_ERR_INVALID_ARG;
+    return MSF_OK;
+}
+
+extern "C" msf_status msf_mssa_forward_simt(msf_plan_t plan, const void* q, const void* k_win,
+                                            const void* v_win, void* out, void* stream) {
+    if (!plan) return MSF_ERR_INVALID_ARG;
+    const Plan& p = *plan;
+    msf_status st = check_attn_args(p, q, k_win, v_win, out);
+    if (st != MSF_OK) return st;
+    msf::AttnArgs a;
+    build_attn_args(p, q, k_win, v_win, out, a);
+    return cuda_status(msf::launch_attn_simt(a, p.elem == 2, (cudaStream_t)stream));
+}
+
+extern "C" msf_status msf_mssa_forward(msf_plan_t plan, const void* q, const void* k_win,
+                                       const void* v_win, void* out, void* stream) {
+    if (!plan) return MSF_ERR_INVALID_ARG;
+    Plan& p = *plan;
+    msf_status st = check_attn_args(p, q, k_win, v_win, out);
+    if (st != MSF_OK) return st;
+    msf::AttnArgs a;
+    build_attn_args(p, q, k_win, v_win, out, a);
+    if (p.elem == 2) return msf::launch_attn_tc(plan, a, (cudaStream_t)stream);
+    return cuda_status(msf::launch_attn_simt(a, false, (cudaStream_t)stream));
+}
+
+static msf::MspShape msp_shape(const Plan& p) {
+    msf::MspShape sh;
+    memset(&sh, 0, sizeof(sh));
+    sh.T = p.T;
+    sh.C = p.d.latent_channels;
+    sh.patch = p.d.patch;
+    sh.Hl = p.d.grid_h * p.d.patch;
+    sh.Wl = p.d.grid_w * p.d.patch;
+    for (int l = 0; l < p.T; ++l) sh.scales[l] = p.d.scales[l];
+    return sh;
+}
+
+extern "C" msf_status msf_patchify(msf_plan_t plan, const void* latent, const void* const* w_tier,
+                                   void* tokens, void* stream) {
+    if (!plan || !latent || !tokens) return MSF_ERR_INVALID_ARG;
+    const Plan& p = *plan;
+    if (p.d.latent_channels <= 0 || p.d.patch <= 0) return MSF_ERR_UNSUPPORTED;
+    if (!aligned16(latent) || !aligned16(tokens)) return MSF_ERR_INVALID_ARG;
+    const msf::MspShape sh = msp_shape(p);
+    cudaStream_t s = (cudaStream_t)stream;
+    const bool bf16 = p.elem == 2;
+    if (!w_tier) return cuda_status(msf::launch_patchify_raw(latent, tokens, sh, p.B, bf16, s));
+    if (p.d.embed_dim <= 0) return MSF_ERR_UNSUPPORTED;
+    if (!p.bound) return MSF_ERR_STATE;  // the raw tokens go through the workspace
+    for (int l = 0; l < p.T; ++l)
+        if (!w_tier[l] || !aligned16(w_tier[l])) return MSF_ERR_INVALID_ARG;
+    char* raw = msf::msp_scratch(p);
+    cudaError_t e = msf::launch_patchify_raw(latent, raw, sh, p.B, bf16, s);
+    if (e != cudaSuccess) return cuda_status(e);
+    const long long per = (long long)sh.C * sh.Hl * sh.Wl;
+    const int E = p.d.embed_dim;
+    for (int l = 0; l < p.T; ++l) {
+        const int P = p.d.patch * p.d.scales[l];
+        const int F = sh.C * P * P;
+        msf::GemmArgs g;
+        g.A = raw + (size_t)l * per * p.elem;
+        g.B = w_tier[l];
+        g.C = (char*)tokens + (size_t)p.st_off[l] * E * p.elem;
+        g.M = p.st_n[l];
+        g.N = E;
+        g.K = F;
+        g.lda = F;
+        g.ldb = F;
+        g.ldc = E;
+        g.a_bstride = (long long)p.T * per;
+        g.c_bstride = (long long)p.N * E;
+        e = msf::launch_gemm_nt_simt(g, p.B, bf16, s);
+        if (e != cudaSuccess) return cuda_status(e);
+    }
+    return MSF_OK;
+}
+
+extern "C" msf_status msf_unpatchify(msf_plan_t plan, int32_t position, const void* tokens,
+                                     const void* w_out, void* latent_out, void* stream) {
+    if (!plan || !tokens || !latent_out) return MSF_ERR_INVALID_ARG;
+    const Plan& p = *plan;
+    if (p.d.latent_channels <= 0 || p.d.patch <= 0) return MSF_ERR_UNSUPPORTED;
+    if (position < 0 || position >= p.T) return MSF_ERR_INVALID_ARG;
+    if (!aligned16(tokens) || !aligned16(latent_out)) return MSF_ERR_INVALID_ARG;
+    const msf::MspShape sh = msp_shape(p);
+    cudaStream_t s = (cudaStream_t)stream;
+    const bool bf16 = p.elem == 2;
+    const long long per = (long long)sh.C * sh.Hl * sh.Wl;
+    if (!w_out)
+        return cuda_status(msf::launch_unpatchify_raw(tokens, latent_out, sh, position,
+                                                      (long long)p.T * per, (int)(position * per),
+                                                      p.B, bf16, s));
+    if (p.d.embed_dim <= 0) return MSF_ERR_UNSUPPORTED;
+    if (!p.bound) return MSF_ERR_STATE;
+    if (!aligned16(w_out)) return MSF_ERR_INVALID_ARG;
+    const int P = p.d.patch * p.d.scales[position];
+    const int F = sh.C * P * P;
+    const int E = p.d.embed_dim;
+    char* raw = msf::msp_scratch(p);
+    msf::GemmArgs g;
+    g.A = (const char*)tokens + (size_t)p.st_off[position] * E * p.elem;
+    g.B = w_out;
+    g.C = raw;
+    g.M = p.st_n[position];
+    g.N = F;
+    g.K = E;
+    g.lda = E;
+    g.ldb = E;
+    g.ldc = F;
+    g.a_bstride = (long long)p.N * E;
+    g.c_bstride = per;
+    cudaError_t e = msf::launch_gemm_nt_simt(g, p.B, bf16, s);
+    if (e != cudaSuccess) return cuda_status(e);
+    return cuda_status(msf::launch_unpatchify_raw(raw, latent_out, sh, position, per, 0, p.B, bf16, s));
+}
+
+extern "C" msf_status msf_plan_device_status(msf_plan_t plan, void* stream) {
+    if (!plan) return MSF_ERR_INVALID_ARG;
+    const Plan& p = *plan;
+    if (!p.bound) return MSF_ERR_STATE;
+    cudaStream_t s = (cudaStream_t)stream;
+    unsigned int word = 0;
+    cudaError_t e = cudaStreamSynchronize(s);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(&word, msf::status_word(p), sizeof(word), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(msf::status_word(p), 0, sizeof(word), s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_status(e);
+    return word ? MSF_ERR_TIMEOUT : MSF_OK;
+}

@@ -1,0 +1,22 @@
+// Tensor-core MSSA attention (tcgen05 + TMA) launcher interface.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include "internal.h"
+#include "kernels.h"
+
+namespace msf {
+
+// Tensor-map slots of the context segments.
+enum : int { kMapSink = 0, kMapHist = 1, kMapWin = 2, kMapPyr0 = 3 };
+// Segments of groups with a pyramid part use map kMapPyr0 + group index;
+// build_attn_args marks them kMapPyr and the launcher resolves the slot.
+constexpr int kMapPyr = -1;
+constexpr int kNumMaps = kMapPyr0 + MSF_MAX_GROUPS;
+
+msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st);
+void tc_cache_free(msf_plan_t plan);
+void tc_cache_invalidate(msf_plan_t plan);
+
+}  // namespace msf

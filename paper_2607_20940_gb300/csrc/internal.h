@@ -1,0 +1,98 @@
+// Internal plan state shared by the host plan code and the kernel launchers.
+#pragma once
+
+#include <stddef.h>
+#include <stdint.h>
+
+#include "../../include/msf.h"
+
+namespace msf {
+
+struct Group {
+    int scale;       // g
+    int q_begin, q_end;
+    int n_finer;     // window states with s_l < g (pooled into the pyramid)
+    int pooled;      // G / g^2 tokens per pooled frame at this scale
+    int pyr_offset;  // token offset of the group's pyramid part (per stream), -1 for g == 1
+    int pyr_cap;     // tokens reserved: (history_capacity + n_finer) * pooled
+};
+
+}  // namespace msf
+
+// The opaque plan of the C ABI.
+struct msf_plan {
+    msf_plan_desc d;
+    int T, G, N, H, D, B;
+    int elem;  // bytes per element
+    int st_off[MSF_MAX_STATES], st_n[MSF_MAX_STATES];
+    int st_gh[MSF_MAX_STATES], st_gw[MSF_MAX_STATES];
+    int n_groups;
+    msf::Group groups[MSF_MAX_GROUPS];
+    int pyr_tokens;   // per stream
+    size_t ws_bytes;
+    float scale;      // softmax scale
+
+    // history ring state (host side)
+    int hist_count;
+    int hist_oldest;
+
+    // bound buffers
+    bool bound;
+    void* ws;
+    size_t ws_size;
+    const void* k_sink;
+    const void* v_sink;
+    void* k_hist;
+    void* v_hist;
+
+    // opaque per-kernel caches (tensor maps etc.)
+    void* tc_cache;
+};
+
+namespace msf {
+using Plan = ::msf_plan;
+
+// Workspace layout: [status area | pyramid K | pyramid V | MSP scratch]
+constexpr size_t kStatusBytes = 256;
+inline size_t round256(size_t x) { return (x + 255) / 256 * 256; }
+inline size_t pyramid_bytes(const Plan& p) {
+    return round256((size_t)p.B * p.pyr_tokens * p.H * p.D * p.elem);
+}
+// Raw MSP tokens of every state: [B, T, C*Hl*Wl].
+inline size_t msp_scratch_bytes(const Plan& p) {
+    if (p.d.latent_channels <= 0 || p.d.patch <= 0) return 0;
+    size_t per = (size_t)p.d.latent_channels * p.d.patch * p.d.grid_h * p.d.patch * p.d.grid_w;
+    return round256((size_t)p.B * p.T * per * p.elem);
+}
+inline size_t workspace_bytes(const Plan& p) {
+    return kStatusBytes + 2 * pyramid_bytes(p) + msp_scratch_bytes(p);
+}
+inline unsigned int* status_word(const Plan& p) { return (unsigned int*)p.ws; }
+inline char* pyr_k(const Plan& p) { return (char*)p.ws + kStatusBytes; }
+inline char* pyr_v(const Plan& p) { return (char*)p.ws + kStatusBytes + pyramid_bytes(p); }
+inline char* msp_scratch(const Plan& p) {
+    return (char*)p.ws + kStatusBytes + 2 * pyramid_bytes(p);
+}
+
+// Number of context tokens of group gi with the current history count.
+inline int group_nkv(const Plan& p, int gi) {
+    const Group& g = p.groups[gi];
+    int n = p.d.sink_tokens + p.hist_count * g.pooled;
+    for (int l = 0; l < p.T; ++l) {
+        int s = p.d.scales[l];
+        n += (s < g.scale) ? g.pooled : p.st_n[l];
+    }
+    return n;
+}
+// Tokens of the pyramid part of group gi (history@g + finer window states).
+inline int group_npyr(const Plan& p, int gi) {
+    const Group& g = p.groups[gi];
+    return (p.hist_count + g.n_finer) * g.pooled;
+}
+
+void set_cuda_error(int e);
+
+// Device status codes written into the status word.
+constexpr unsigned int kDevTimeout = 1u;
+
+}  // namespace msf

@@ -1,0 +1,85 @@
+// Launch interfaces of the CUDA kernels (host side of each .cu file).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "internal.h"
+
+namespace msf {
+
+// ------------------------------------------------------------------ pooling
+struct PoolJob {
+    const char* src_k;      // source block, stream 0
+    const char* src_v;
+    char* dst_k;            // destination block, stream 0
+    char* dst_v;
+    long long src_bstride;  // bytes between streams
+    long long dst_bstride;
+    int src_gw;             // source grid width (tokens)
+    int out_gw;             // pooled grid width
+    int out_n;              // pooled tokens
+    int sigma;              // stride (1 = copy)
+};
+constexpr int kMaxPoolJobs = 40;
+struct PoolBatch {
+    PoolJob j[kMaxPoolJobs];
+    int n;
+    int row_vecs;  // 16-byte vectors per token row (H*D*elem/16)
+    int mode;      // msf_resample_mode
+};
+cudaError_t launch_pool(const PoolBatch& jobs, int batch, bool bf16, cudaStream_t st);
+
+// -------------------------------------------------------------------- MSP
+struct MspShape {
+    int T, C, Hl, Wl, patch;
+    int scales[MSF_MAX_STATES];
+};
+cudaError_t launch_patchify_raw(const void* latent, void* raw, const MspShape& sh, int batch,
+                                bool bf16, cudaStream_t st);
+cudaError_t launch_unpatchify_raw(const void* raw, void* latent, const MspShape& sh, int position,
+                                  long long raw_bstride, int raw_offset, int batch, bool bf16,
+                                  cudaStream_t st);
+
+struct GemmArgs {
+    const void* A;  // [M, K] (+ a_bstride per batch), element strides
+    const void* B;  // [N, K]
+    void* C;        // [M, N]
+    int M, N, K;
+    long long lda, ldb, ldc;
+    long long a_bstride, c_bstride;
+};
+cudaError_t launch_gemm_nt_simt(const GemmArgs& g, int batch, bool bf16, cudaStream_t st);
+
+// --------------------------------------------------------------- attention
+// One context segment of a query group: rows [row0, row0 + len) of a
+// [B, rows_total, H, D] tensor pair.
+struct Segment {
+    const char* k;
+    const char* v;
+    long long bstride;  // bytes between streams
+    int row0;
+    int len;
+    int rows_total;     // rows of the underlying tensor (TMA extent)
+    int map_id;         // which tensor map (tensor-core kernel)
+};
+constexpr int kMaxSeg = 3;
+struct AttnGroup {
+    int q_begin, q_end;
+    int n_seg;
+    Segment seg[kMaxSeg];
+};
+struct AttnArgs {
+    const char* q;
+    char* out;
+    long long q_bstride;  // bytes between streams of q/out/k_win
+    int H, D, B;
+    float scale_log2;     // softmax scale * log2(e)
+    int n_groups;
+    AttnGroup g[MSF_MAX_GROUPS];
+    unsigned int* status;
+};
+cudaError_t launch_attn_simt(const AttnArgs& a, bool bf16, cudaStream_t st);
+
+}  // namespace msf

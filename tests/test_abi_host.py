@@ -1,0 +1,133 @@
+"""Host-side checks of the C ABI (no GPU): the library loads, exports every
+function include/msf.h declares, and its static plan tables (Eq. 3 counts,
+Eq. 4 context layout, FLOP counts) equal the oracle's own enumeration."""
+import ctypes
+import os
+import random
+import re
+
+import numpy as np
+import pytest
+
+from oracle import schedule
+from paper_2607_20940_gb300 import synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _msf():
+    from paper_2607_20940_gb300 import msf
+    return msf
+
+
+def _declared():
+    names = set()
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            src = open(os.path.join(ROOT, "include", fn)).read()
+            src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+            names |= set(re.findall(r"\b(msf_[a-z0-9_]+)\s*\(", src))
+    return names
+
+
+def test_library_exports_every_declared_symbol():
+    msf = _msf()
+    lib = ctypes.CDLL(msf.LIB_PATH)
+    declared = _declared()
+    assert declared, "no declarations found"
+    for name in sorted(declared):
+        assert hasattr(lib, name), f"{name} declared in include/ but not exported"
+    assert declared == set(msf.EXPORTS)
+
+
+def _plan(scales, gh, gw, ns, nh, cap=None, H=2, D=64, B=1):
+    msf = _msf()
+    return msf.Plan(msf.make_desc(scales, gh, gw, H, D, ns, nh, history_capacity=cap, batch=B))
+
+
+CASES = [
+    (synth.TINY.scales, 8, 8, 64, 1),
+    (synth.LAYER_480P.scales, 30, 52, 1560, 2),
+    (synth.THREE_SCALE.scales, 48, 80, 3840, 2),
+    ((1, 1, 1, 1, 1), 30, 52, 1560, 2),
+    ((2, 2, 4), 8, 8, 5, 3),
+    ((1,), 4, 4, 0, 0),
+]
+
+
+@pytest.mark.parametrize("scales,gh,gw,ns,nh", CASES)
+def test_plan_tables_match_oracle(scales, gh, gw, ns, nh):
+    p = _plan(scales, gh, gw, ns, nh)
+    info = p.info
+    cnt = schedule.token_counts(scales, gh, gw)
+    offs = schedule.token_offsets(scales, gh, gw)
+    assert info.n_tokens == sum(cnt)
+    assert info.n_tokens_fine == len(scales) * gh * gw
+    assert list(info.state_tokens[:len(scales)]) == cnt
+    assert list(info.state_offset[:len(scales)]) == offs
+    groups = schedule.query_groups(scales, gh, gw)
+    assert info.n_groups == len(groups)
+    for gi, g in enumerate(groups):
+        gi_ = info.groups[gi]
+        assert (gi_.scale, gi_.q_begin, gi_.q_end) == (g.scale, g.q_begin, g.q_end)
+        rows = schedule.context_rows(scales, gh, gw, ns, nh, g.scale)
+        assert gi_.n_kv == len(rows)
+        got = p.index_map(gi)
+        want = np.array(rows, dtype=np.int32).reshape(-1, 5)
+        assert got.shape == want.shape
+        assert np.array_equal(got, want)
+    assert info.attention_flops == schedule.attention_flops(scales, gh, gw, ns, nh, 2, 64)
+
+
+def test_plan_tables_random_schedules():
+    rng = random.Random(1234)
+    for _ in range(40):
+        T = rng.randint(1, 6)
+        levels = sorted(rng.choice([1, 1, 2, 2, 4, 8]) for _ in range(T))
+        smax = max(levels)
+        gh, gw = smax * rng.randint(1, 4), smax * rng.randint(1, 5)
+        ns, nh = rng.randint(0, 9), rng.randint(0, 3)
+        p = _plan(levels, gh, gw, ns, nh, cap=nh + rng.randint(0, 2), B=rng.randint(1, 3))
+        for gi, g in enumerate(schedule.query_groups(levels, gh, gw)):
+            want = np.array(schedule.context_rows(levels, gh, gw, ns, nh, g.scale),
+                            dtype=np.int32).reshape(-1, 5)
+            assert np.array_equal(p.index_map(gi), want)
+
+
+def test_480p_numbers():
+    info = _plan(synth.LAYER_480P.scales, 30, 52, 1560, 2, H=12, D=128).info
+    assert info.n_tokens == 4290 and info.n_tokens_fine == 7800
+    assert info.attention_flops == 202787020800
+    assert info.dense_flops == 4 * 128 * 12 * 7800 * (1560 + 2 * 1560 + 7800)
+    assert info.resample_bytes == 2 * 4 * (1560 + 390) * 12 * 128 * 2
+
+
+@pytest.mark.parametrize("bad", [
+    dict(scales=(1, 2, 1)), dict(scales=(1, 3)), dict(scales=(1, 4), gh=30),
+    dict(D=96), dict(H=0), dict(nh=3, cap=2),
+])
+def test_plan_validation(bad):
+    msf = _msf()
+    args = dict(scales=(1, 2), gh=8, gw=8, ns=4, nh=1, cap=None, H=2, D=64)
+    args.update(bad)
+    with pytest.raises(msf.MsfError) as ei:
+        _plan(args["scales"], args["gh"], args["gw"], args["ns"], args["nh"], cap=args["cap"],
+              H=args["H"], D=args["D"])
+    assert ei.value.status in (msf.MSF_ERR_INVALID_ARG, msf.MSF_ERR_UNSUPPORTED)
+
+
+def test_calls_before_bind_and_bad_pointers_fail_without_cuda():
+    msf = _msf()
+    p = _plan((1, 2), 8, 8, 4, 1)
+    lib = msf._lib
+    # unbound plan: STATE, reported before any CUDA call
+    assert lib.msf_mssa_forward(p.handle, 4096, 8192, 12288, 16384, None) == msf.MSF_ERR_STATE
+    assert lib.msf_kv_resample(p.handle, 4096, 8192, 0, None) == msf.MSF_ERR_STATE
+    assert lib.msf_history_append(p.handle, 4096, 8192, None) == msf.MSF_ERR_STATE
+    # null / misaligned
+    assert lib.msf_mssa_forward(p.handle, None, 8192, 12288, 16384, None) == msf.MSF_ERR_INVALID_ARG
+    assert lib.msf_plan_bind(p.handle, 4096, 16, 4096, 4096, 4096, 4096) == msf.MSF_ERR_WORKSPACE
+    assert lib.msf_plan_bind(p.handle, 4097, 1 << 30, 4096, 4096, 4096, 4096) == msf.MSF_ERR_INVALID_ARG
+    assert lib.msf_plan_index_map(p.handle, 7, None, 0, ctypes.byref(ctypes.c_size_t())) == \
+        msf.MSF_ERR_INVALID_ARG
+    assert msf.msf_status_string(msf.MSF_ERR_TIMEOUT) == "device wait timed out"
