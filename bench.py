@@ -1,0 +1,414 @@
+"""Benchmark of the Ms. Forcing MSSA window pass on GB300.
+
+A step is one rolling-window pass of the whole hot path at the 480p layer
+shapes (T=5, 30x52 fine grid, scales (1,1,2,2,2), 12 heads of 128, sink 1560
+tokens, history ring of 2 frames):
+  MSP patchify + tier embedding of the 5 latent states (16x60x104 -> 4290x1536)
+  -> window part of the K/V pyramid -> MSSA attention (Eq. 4)
+  -> de-embed + unpatchify of the head state -> history append (head K/V).
+`value` is the MSSA FLOPs the schedule requires (4*D*H*sum_g Nq_g*Nkv_g =
+202.79 GFLOP) divided by the device time of the whole step, in TFLOP/s.
+Inputs are resident in HBM; the L2 is flushed (a 256 MiB write) between
+timed steps, outside the timed events.
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+Under torchrun every rank runs its own stream of windows (weak scaling);
+rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "MSSA TFLOP/s and µs per window-pass layer (bf16, 1 GB300); % of tensor peak"
+UNIT = "TFLOP/s"
+FLUSH_BYTES = 256 << 20
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return d, "measured"
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = os.path.join("/tmp", f"msf_clocks_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    mx = float(parts[2])
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower() == "active":
+                        reasons.add(n)
+        try:
+            os.remove(self.path)
+        except OSError:
+            pass
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def max_over_ranks(value: float, device) -> float:
+    """The largest per-rank time (the job ends when the slowest rank ends)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return value
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def _oracle_step(w, x, m, heads=None):
+    """The oracle's version of one step (patchify+embed, MSSA, de-embed+unpatchify
+    of the head state, history append as a copy)."""
+    import numpy as np
+
+    from oracle import msp as omsp
+    from oracle import mssa as omssa
+    from paper_2607_20940_gb300 import synth
+    f = synth.to_f64
+    tiers = {s: f(m["w_tier"][s]) for s in set(w.scales)}
+    omsp.patchify_window(f(m["latent"]), w.scales, w.patch, tiers)
+    out = omssa.mssa_forward(f(x["q"]), f(x["k_win"]), f(x["v_win"]), f(x["k_sink"]),
+                             f(x["v_sink"]), f(x["k_hist"]), f(x["v_hist"]), w.scales, w.grid_h,
+                             w.grid_w, heads=heads)
+    G = w.grid_h * w.grid_w
+    if heads is None:
+        head_tok = out[:, :G].reshape(w.batch, G, -1)
+        omsp.unpatchify_state(head_tok, w.patch, w.latent_channels, w.grid_h * w.patch,
+                              w.grid_w * w.patch, f(m["w_out"]))
+    np.copy(f(x["k_win"])[:, :G])
+    return out
+
+
+def run_reference(args, w):
+    """The oracle (fp64 numpy) on the host cores, same workload and metric.
+    Each step computes 3 of the 12 heads of the layer (a bounded sample);
+    FLOPs are counted for the heads computed."""
+    import torch
+
+    from oracle import schedule
+    from paper_2607_20940_gb300 import synth
+    x = synth.attention_inputs(w, torch.bfloat16)
+    m = synth.msp_inputs(w, torch.bfloat16)
+    heads = [0, 5, 11]
+    fl = schedule.attention_flops(w.scales, w.grid_h, w.grid_w, w.sink_tokens, w.history_frames,
+                                  len(heads), w.head_dim, w.batch)
+    for _ in range(args.warmup):
+        _oracle_step(w, x, m, heads)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        _oracle_step(w, x, m, heads)
+        times.append(time.perf_counter() - t0)
+    tot = sum(times)
+    value = fl * args.steps / tot / 1e12
+    cores = os.cpu_count()
+    sample = f"3 of 12 heads of the 480p layer per step (oracle fp64, numpy), {fl/1e9:.2f} GFLOP"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": {"workload": w.name, "kind": "oracle sample"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+
+
+def _traffic_from_profile(kernel_src: str):
+    """dram bytes per launch of the attention kernel from the committed ncu
+    summary, if it was taken on the current kernel source."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "mssa_tc_480p_traffic.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        h = hashlib.sha256(open(kernel_src, "rb").read()).hexdigest()[:16]
+        if d.get("kernel_sha") == h:
+            return float(d["dram_bytes_per_launch"])
+    except Exception:
+        pass
+    return None
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+
+    world, rank, local = _dist()
+    from paper_2607_20940_gb300 import synth
+    w = synth.LAYER_480P
+
+    if args.impl == "reference":
+        if rank == 0:
+            run_reference(args, w)
+        return
+
+    import torch
+    import torch.distributed as dist
+
+    from paper_2607_20940_gb300 import msf
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream()
+
+    # ------------------------------------------------------------ set-up
+    x = synth.attention_inputs(w, torch.bfloat16, seed=w.seed + 1000 * rank)
+    mi = synth.msp_inputs(w, torch.bfloat16, seed=w.seed + 1000 * rank)
+    plan = msf.Plan(msf.make_desc(w.scales, w.grid_h, w.grid_w, w.heads, w.head_dim,
+                                  w.sink_tokens, w.history_frames, w.history_capacity,
+                                  batch=w.batch, latent_channels=w.latent_channels, patch=w.patch,
+                                  embed_dim=w.embed_dim))
+    info = plan.info
+    d = {k: v.to(dev) for k, v in x.items()}
+    ws = plan.workspace(dev)
+    plan.bind(ws, d["k_sink"], d["v_sink"], d["k_hist"], d["v_hist"])
+    lat = mi["latent"].to(dev)
+    w_tier = [mi["w_tier"][s].t().contiguous().to(dev) for s in w.scales]
+    w_out = mi["w_out"].t().contiguous().to(dev)
+    N, E = info.n_tokens, w.embed_dim
+    tok = torch.empty((w.batch, N, E), dtype=torch.bfloat16, device=dev)
+    out = torch.empty_like(d["q"])
+    lat_out = torch.empty((w.batch, w.latent_channels, w.grid_h * w.patch, w.grid_w * w.patch),
+                          dtype=torch.bfloat16, device=dev)
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    flops = info.attention_flops
+
+    ev_a = []  # attention start/end events of timed steps
+
+    def step(q, k, v, latent, timed_attn=False):
+        plan.patchify(latent, w_tier, tok)
+        plan.kv_resample(k, v, msf.MSF_RESAMPLE_WINDOW_ONLY)
+        if timed_attn:
+            a0 = torch.cuda.Event(enable_timing=True)
+            a1 = torch.cuda.Event(enable_timing=True)
+            a0.record(stream)
+        plan.mssa_forward(q, k, v, out)
+        if timed_attn:
+            a1.record(stream)
+            ev_a.append((a0, a1))
+        plan.unpatchify(0, out.view(w.batch, N, E), w_out, lat_out)
+        plan.history_append(k, v)
+
+    plan.kv_resample(d["k_win"], d["v_win"], msf.MSF_RESAMPLE_FULL)
+    for _ in range(args.warmup):
+        step(d["q"], d["k_win"], d["v_win"], lat)
+    torch.cuda.synchronize()
+    if plan.device_status() != msf.MSF_OK:
+        raise RuntimeError("device status error during warm-up")
+
+    # ------------------------------------------------------- timed steps
+    clocks = ClockSampler(local)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    launches0 = msf.msf_kernel_launches()
+    ev = []
+    for _ in range(args.steps):
+        flush.fill_(1)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        step(d["q"], d["k_win"], d["v_win"], lat, timed_attn=True)
+        e1.record(stream)
+        ev.append((e0, e1))
+    torch.cuda.synchronize()
+    launches = msf.msf_kernel_launches() - launches0
+    clk = clocks.stop()
+    if world > 1:
+        dist.barrier()
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    attn_ms = [a.elapsed_time(b) for a, b in ev_a]
+    tot_ms = max_over_ranks(sum(step_ms), dev)
+    status = plan.device_status()
+
+    # ------------------------------------------- end to end (host buffers)
+    pin = {k: x[k].pin_memory() for k in ("q", "k_win", "v_win")}
+    pin_lat = mi["latent"].pin_memory()
+    host_out = torch.empty(lat_out.shape, dtype=lat_out.dtype).pin_memory()
+    dq, dk, dv, dl = (torch.empty_like(d["q"]), torch.empty_like(d["k_win"]),
+                      torch.empty_like(d["v_win"]), torch.empty_like(lat))
+    h2d = sum(t.numel() * t.element_size() for t in list(pin.values()) + [pin_lat])
+    d2h = host_out.numel() * host_out.element_size()
+    ev2 = []
+    for i in range(args.warmup + args.steps):
+        flush.fill_(1)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        dq.copy_(pin["q"], non_blocking=True)
+        dk.copy_(pin["k_win"], non_blocking=True)
+        dv.copy_(pin["v_win"], non_blocking=True)
+        dl.copy_(pin_lat, non_blocking=True)
+        step(dq, dk, dv, dl)
+        host_out.copy_(lat_out, non_blocking=True)
+        e1.record(stream)
+        if i >= args.warmup:
+            ev2.append((e0, e1))
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(sum(a.elapsed_time(b) for a, b in ev2), dev)
+
+    # ------------------------------------------------- all-fine baseline
+    wf = w.with_scales((1, 1, 1, 1, 1))
+    plan_f = msf.Plan(msf.make_desc(wf.scales, wf.grid_h, wf.grid_w, wf.heads, wf.head_dim,
+                                    wf.sink_tokens, wf.history_frames, wf.history_capacity,
+                                    batch=wf.batch))
+    xf = synth.attention_inputs(wf, torch.bfloat16, seed=wf.seed + 1000 * rank)
+    df = {k: v.to(dev) for k, v in xf.items()}
+    wsf = plan_f.workspace(dev)
+    plan_f.bind(wsf, df["k_sink"], df["v_sink"], df["k_hist"], df["v_hist"])
+    outf = torch.empty_like(df["q"])
+    plan_f.kv_resample(df["k_win"], df["v_win"])
+    fine_ms = []
+    for i in range(args.warmup + max(5, args.steps // 2)):
+        flush.fill_(1)
+        a0 = torch.cuda.Event(enable_timing=True)
+        a1 = torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        plan_f.mssa_forward(df["q"], df["k_win"], df["v_win"], outf)
+        a1.record(stream)
+        if i >= args.warmup:
+            fine_ms.append((a0, a1))
+    torch.cuda.synchronize()
+    fine_attn_ms = statistics.mean(a.elapsed_time(b) for a, b in fine_ms)
+    fine_flops = plan_f.info.attention_flops
+
+    if rank != 0:
+        if world > 1:
+            dist.barrier()
+            dist.destroy_process_group()
+        return
+
+    # ------------------------------------------------------- CPU baseline
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        t0 = time.perf_counter()
+        _oracle_step(w, x, mi)
+        dt = time.perf_counter() - t0
+        cpu = {"value": flops / dt / 1e12, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+               "sample": f"one full 480p step (all 12 heads) in fp64 numpy, {dt:.1f} s"}
+
+    peaks, peak_src = _peaks()
+    attn_avg_ms = statistics.mean(attn_ms)
+    achieved = flops / (attn_avg_ms * 1e-3) / 1e12
+    peak = float(peaks["bf16_tflops"])
+    traffic = _traffic_from_profile(os.path.join(ROOT, "paper_2607_20940_gb300", "csrc", "attn_tc.cu"))
+    ms_per_step = tot_ms / args.steps
+    line = {
+        "metric": METRIC,
+        "value": world * flops * args.steps / (tot_ms * 1e-3) / 1e12,
+        "unit": UNIT,
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": ms_per_step,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic",
+        "config": {
+            "workload": w.name, "T": w.T, "scales": list(w.scales), "grid": [w.grid_h, w.grid_w],
+            "heads": w.heads, "head_dim": w.head_dim, "sink_tokens": w.sink_tokens,
+            "history_frames": w.history_frames, "batch_per_gpu": w.batch,
+            "latent": [w.latent_channels, w.grid_h * w.patch, w.grid_w * w.patch],
+            "embed_dim": w.embed_dim, "attention_gflop": flops / 1e9,
+            "us_per_layer": ms_per_step * 1e3, "l2": "flushed between steps (256 MiB write)",
+            "parallelism": f"replica x{world}",
+        },
+        "roofline": {
+            "bound": "tensor", "kernel": "mssa_tc_kernel<128>", "achieved": achieved, "peak": peak,
+            "unit": "TFLOP/s", "frac": achieved / peak, "traffic": traffic,
+            "peak_source": f"{peak_src} bf16_tflops (burst)",
+            "frac_of_sustained": achieved / float(peaks.get("bf16_tflops_sustained", peak)),
+            "attention_us": attn_avg_ms * 1e3,
+        },
+        "all_fine": {"attention_us": fine_attn_ms * 1e3, "gflop": fine_flops / 1e9,
+                     "tflops": fine_flops / (fine_attn_ms * 1e-3) / 1e12,
+                     "speedup_vs_all_fine": fine_attn_ms / attn_avg_ms},
+        "cpu_baseline": cpu,
+        "e2e": {"value": world * flops * args.steps / (e2e_ms * 1e-3) / 1e12, "unit": UNIT,
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "ms_per_step": e2e_ms / args.steps},
+        "gpu_launches": launches,
+        "clocks": clk,
+        "device_status": msf.msf_status_string(status),
+    }
+    print(json.dumps(line))
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

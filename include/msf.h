@@ -220,6 +220,10 @@ msf_status msf_mssa_forward_simt(msf_plan_t plan, const void* q, const void* k_w
 msf_status msf_history_append(msf_plan_t plan, const void* k_win, const void* v_win,
                               void* stream);
 
+/* Number of kernels this library has launched in this process (all plans,
+ * all devices), for accounting in benchmarks. Host only. */
+uint64_t msf_kernel_launches(void);
+
 /* Synchronise `stream`, read and clear the device status word. Returns
  * MSF_ERR_TIMEOUT if a kernel gave up on a bounded wait since the last
  * check, MSF_OK otherwise. */

@@ -4,6 +4,7 @@
 #include <string.h>
 
 #include "attn_tc.h"
+#include "gemm_tc.h"
 #include "internal.h"
 #include "kernels.h"
 
@@ -173,6 +174,8 @@ extern "C" msf_status msf_plan_bind(msf_plan_t plan, void* workspace, size_t wor
     p.bound = true;
     msf::tc_cache_invalidate(plan);
     cudaError_t e = cudaMemset(msf::status_word(p), 0, msf::kStatusBytes);
+    if (e == cudaSuccess && msf::attn_counter_bytes(p) > 0)
+        e = cudaMemset(msf::attn_counters(p), 0, msf::attn_counter_bytes(p));
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
     return cuda_status(e);
 }
@@ -311,6 +314,56 @@ extern "C" msf_status msf_patchify(msf_plan_t plan, const void* latent, const vo
     if (e != cudaSuccess) return cuda_status(e);
     const long long per = (long long)sh.C * sh.Hl * sh.Wl;
     const int E = p.d.embed_dim;
+    if (bf16) {
+        // One tensor-core GEMM per run of consecutive states that share a tier
+        // (same scale, same weight): their raw blocks and output rows are
+        // contiguous.
+        bool all_tc = true;
+        for (int l0 = 0; l0 < p.T && all_tc;) {
+            int l1 = l0 + 1;
+            while (l1 < p.T && p.d.scales[l1] == p.d.scales[l0] && w_tier[l1] == w_tier[l0]) ++l1;
+            const int P = p.d.patch * p.d.scales[l0];
+            msf::GemmTcArgs g;
+            g.K = sh.C * P * P;
+            g.A = raw + (size_t)l0 * per * p.elem;
+            g.B = w_tier[l0];
+            g.C = (char*)tokens + (size_t)p.st_off[l0] * E * p.elem;
+            g.M = p.st_off[l1 - 1] + p.st_n[l1 - 1] - p.st_off[l0];
+            g.N = E;
+            g.lda = g.K;
+            g.ldb = g.K;
+            g.ldc = E;
+            g.a_bstride = (long long)p.T * per;
+            g.c_bstride = (long long)p.N * E;
+            g.status = msf::status_word(p);
+            all_tc = msf::gemm_tc_supported(g);
+            l0 = l1;
+        }
+        if (all_tc) {
+            for (int l0 = 0; l0 < p.T;) {
+                int l1 = l0 + 1;
+                while (l1 < p.T && p.d.scales[l1] == p.d.scales[l0] && w_tier[l1] == w_tier[l0]) ++l1;
+                const int P = p.d.patch * p.d.scales[l0];
+                msf::GemmTcArgs g;
+                g.K = sh.C * P * P;
+                g.A = raw + (size_t)l0 * per * p.elem;
+                g.B = w_tier[l0];
+                g.C = (char*)tokens + (size_t)p.st_off[l0] * E * p.elem;
+                g.M = p.st_off[l1 - 1] + p.st_n[l1 - 1] - p.st_off[l0];
+                g.N = E;
+                g.lda = g.K;
+                g.ldb = g.K;
+                g.ldc = E;
+                g.a_bstride = (long long)p.T * per;
+                g.c_bstride = (long long)p.N * E;
+                g.status = msf::status_word(p);
+                e = msf::launch_gemm_tc(g, p.B, s);
+                if (e != cudaSuccess) return cuda_status(e);
+                l0 = l1;
+            }
+            return MSF_OK;
+        }
+    }
     for (int l = 0; l < p.T; ++l) {
         const int P = p.d.patch * p.d.scales[l];
         const int F = sh.C * P * P;
@@ -354,6 +407,27 @@ extern "C" msf_status msf_unpatchify(msf_plan_t plan, int32_t position, const vo
     const int F = sh.C * P * P;
     const int E = p.d.embed_dim;
     char* raw = msf::msp_scratch(p);
+    if (bf16) {
+        msf::GemmTcArgs t;
+        t.A = (const char*)tokens + (size_t)p.st_off[position] * E * p.elem;
+        t.B = w_out;
+        t.C = raw;
+        t.M = p.st_n[position];
+        t.N = F;
+        t.K = E;
+        t.lda = E;
+        t.ldb = E;
+        t.ldc = F;
+        t.a_bstride = (long long)p.N * E;
+        t.c_bstride = per;
+        t.status = msf::status_word(p);
+        if (msf::gemm_tc_supported(t)) {
+            cudaError_t e = msf::launch_gemm_tc(t, p.B, s);
+            if (e != cudaSuccess) return cuda_status(e);
+            return cuda_status(
+                msf::launch_unpatchify_raw(raw, latent_out, sh, position, per, 0, p.B, bf16, s));
+        }
+    }
     msf::GemmArgs g;
     g.A = (const char*)tokens + (size_t)p.st_off[position] * E * p.elem;
     g.B = w_out;

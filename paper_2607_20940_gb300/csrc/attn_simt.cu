@@ -107,14 +107,14 @@ cudaError_t launch_attn_simt(const AttnArgs& a, bool bf16, cudaStream_t st) {
     dim3 grid((unsigned)tiles, (unsigned)a.H, (unsigned)a.B);
     if (a.D == 128) {
         if (bf16)
-            attn_simt_kernel<__nv_bfloat16, 128><<<grid, 128, 0, st>>>(a);
+            { note_launch(); attn_simt_kernel<__nv_bfloat16, 128><<<grid, 128, 0, st>>>(a); }
         else
-            attn_simt_kernel<float, 128><<<grid, 128, 0, st>>>(a);
+            { note_launch(); attn_simt_kernel<float, 128><<<grid, 128, 0, st>>>(a); }
     } else {
         if (bf16)
-            attn_simt_kernel<__nv_bfloat16, 64><<<grid, 128, 0, st>>>(a);
+            { note_launch(); attn_simt_kernel<__nv_bfloat16, 64><<<grid, 128, 0, st>>>(a); }
         else
-            attn_simt_kernel<float, 64><<<grid, 128, 0, st>>>(a);
+            { note_launch(); attn_simt_kernel<float, 64><<<grid, 128, 0, st>>>(a); }
     }
     return cudaGetLastError();
 }

@@ -1,10 +1,19 @@
 // MSSA attention on the sm_103a tensor cores (Eq. 4 context, bf16 operands,
 // fp32 online softmax and accumulation).
 //
-// One CTA owns a 256-row query block (two 128-row tiles Q0, Q1) of one
-// (stream, head, query group) and walks that group's context segments
-// (sink, history or pyramid part, window suffix) in 128-row K/V tiles:
-//   warp 0      TMA producer: Q0/Q1 once, then K_j and V_j into a 2-stage ring
+// Work: an item is one 256-row query block (two 128-row tiles Q0, Q1) of one
+// (stream, head, query group); it walks that group's context segments (sink,
+// history or pyramid part, window suffix) in 128-row K/V tiles. All items'
+// tiles form one sequence (longest contexts first) that a persistent grid
+// splits into equal contiguous ranges, one per CTA (stream-K). A piece is the
+// part of one item inside one CTA's range. A piece that is a whole item
+// writes its normalised output; a piece of a split item writes its
+// unnormalised output with the running max and sum to a partial slot, and the
+// piece that finishes last merges all of them (per-item counter in the
+// workspace, reset by the merger).
+//
+// Roles inside a CTA (384 threads):
+//   warp 0      TMA producer: Q0/Q1 per piece, then K_j, V_j into a 2-stage ring
 //   warp 1      MMA issuer (one thread): S_t = Q_t K_j^T into TMEM (SS form),
 //               O_t += P_t V_j with P_t read from TMEM (TS form, V MN-major)
 //   warp 2      TMEM allocation (all 512 columns)
@@ -17,7 +26,7 @@
 // signals S_t(j+1) also covers PV_t(j): a softmax warp that sees S ready may
 // rescale O_t in place. Every segment has its own tensor map whose extent is
 // the segment's end, so rows past it load as zeros; their scores are masked.
-// Waits are bounded; a wait that gives up raises the CTA's abort flag, sets
+// Every wait is bounded; a wait that gives up raises the CTA's abort flag and
 // the device status word, and every role winds down without hanging.
 #include <cuda.h>
 #include <cuda_bf16.h>
@@ -37,30 +46,44 @@ constexpr int kBlockM = 128;   // query rows per tile
 constexpr int kBlockN = 128;   // context rows per K/V tile
 constexpr int kStages = 2;     // K/V ring depth
 constexpr int kThreads = 384;  // 12 warps
+// Registers: 168 per thread at launch (12 warps x 168 = 64512 of 65536). The
+// producer/MMA warpgroup drops to 120 and the two softmax warpgroups rise to
+// 192: 4 x 120 + 8 x 192 = 12 x 168, so the increase is always satisfiable.
+// The launcher refuses to run if the compiled kernel does not use exactly
+// kLaunchRegs per thread.
+constexpr int kLaunchRegs = 168;
+constexpr int kCtrlRegs = 120;
+constexpr int kSoftmaxRegs = 192;
+static_assert(4 * kCtrlRegs + 8 * kSoftmaxRegs == 12 * kLaunchRegs, "register split");
 constexpr long long kWaitLimit = 2000000000LL;  // ~1 s of SM clock
 
 struct TcSeg {
     int map;
     int row0;
     int len;
-    int ntiles;
+    int tile0;  // first tile of this segment in the item's tile sequence
 };
 struct TcGroup {
     int q_begin, q_end;
-    int n_qb;      // 256-row query blocks
-    int n_items;   // B * H * n_qb
+    int n_qb;        // 256-row query blocks
+    int n_items;     // B * H * n_qb
     int n_seg;
-    int n_tiles;   // sum of segment tiles
+    int n_tiles;     // tiles per item
+    long long tile_base;  // first tile of this group in the global sequence
+    int item_base;        // first item index of this group (merge counters)
     TcSeg seg[kMaxSeg];
 };
 struct TcParams {
     int H, B;
     float scale_log2;
     int n_groups;
+    long long total_tiles;
     TcGroup g[MSF_MAX_GROUPS];  // longest context first
     __nv_bfloat16* out;
     long long out_bstride;  // elements
     unsigned int* status;
+    unsigned int* counters;  // per item
+    float* partials;         // 2 slots per CTA
     long long wait_limit;
 };
 struct TcMaps {
@@ -74,12 +97,68 @@ struct Cfg {
     static constexpr int kChunks = D / 64;                    // 128-byte swizzle chunks per row
     static constexpr int kTileBytes = kBlockM * D * 2;        // one Q / K / V tile
     static constexpr int kSmem = (2 + 2 * kStages) * kTileBytes + 1024;
+    static constexpr int kSlotFloats = 2 * kBlockM * (D + 2);
 };
 
 __device__ __forceinline__ float ex2(float x) {
     float y;
     asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
     return y;
+}
+
+// One piece of work: tiles [u0, u1) of one item.
+struct Piece {
+    int gi, item, b, h, q_row0, u0, u1;
+    bool whole;
+    long long item_start;  // global index of the item's first tile
+};
+
+__device__ __forceinline__ long long cta_begin(long long c, long long T, long long n) {
+    return c * T / n;
+}
+// The CTA whose range [cta_begin(c), cta_begin(c+1)) holds tile t.
+__device__ __forceinline__ long long cta_of(long long t, long long T, long long n) {
+    return ((t + 1) * n - 1) / T;
+}
+
+__device__ __forceinline__ Piece locate(const TcParams& p, long long t, long long r1) {
+    Piece pc;
+    int gi = 0;
+    while (gi < p.n_groups - 1 && t >= p.g[gi + 1].tile_base) ++gi;
+    const TcGroup& G = p.g[gi];
+    const long long rel = t - G.tile_base;
+    const int item = (int)(rel / G.n_tiles);
+    const int u0 = (int)(rel - (long long)item * G.n_tiles);
+    long long u1 = u0 + (r1 - t);
+    if (u1 > G.n_tiles) u1 = G.n_tiles;
+    pc.gi = gi;
+    pc.item = item;
+    const int qb = item % G.n_qb;
+    pc.h = (item / G.n_qb) % p.H;
+    pc.b = item / (G.n_qb * p.H);
+    pc.q_row0 = G.q_begin + qb * 2 * kBlockM;
+    pc.u0 = u0;
+    pc.u1 = (int)u1;
+    pc.whole = (u0 == 0 && u1 == G.n_tiles);
+    pc.item_start = G.tile_base + (long long)item * G.n_tiles;
+    return pc;
+}
+
+// Segment, context row and valid row count of tile u of an item of group G.
+__device__ __forceinline__ void tile_info(const TcGroup& G, int u, int& seg, int& row, int& valid) {
+    int s = 0;
+    while (s < G.n_seg - 1 && u >= G.seg[s + 1].tile0) ++s;
+    const int kt = u - G.seg[s].tile0;
+    seg = s;
+    row = G.seg[s].row0 + kt * kBlockN;
+    valid = min(kBlockN, G.seg[s].len - kt * kBlockN);
+}
+
+// Partial slot of the piece of an item that CTA c holds: a CTA's first piece
+// uses slot 2c, a later (last) piece slot 2c+1.
+__device__ __forceinline__ int slot_of(long long c, long long c1, long long item_start, long long T,
+                                       long long n) {
+    return 2 * (int)c + ((c == c1 && cta_begin(c, T, n) < item_start) ? 1 : 0);
 }
 
 template <int D>
@@ -92,31 +171,27 @@ __global__ void __launch_bounds__(kThreads, 1)
     unsigned char* sK = smem + 2 * C::kTileBytes;              // [kStages][tile]
     unsigned char* sV = sK + kStages * C::kTileBytes;          // [kStages][tile]
 
-    __shared__ uint64_t q_full, o_full;
+    __shared__ uint64_t q_full, q_empty, o_full, drain_bar;
     __shared__ uint64_t k_full[kStages], k_empty[kStages], v_full[kStages], v_empty[kStages];
     __shared__ uint64_t s_full[2], p_full[2];
+    __shared__ uint64_t epi_written, epi_decided;
     __shared__ uint32_t tmem_base_sh;
     __shared__ int abort_flag;
+    __shared__ int merge_flag;
 
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-
-    // ---- work item: group (longest first), then q block fastest, head, stream
-    int item = blockIdx.x, gi = 0;
-    while (gi < p.n_groups - 1 && item >= p.g[gi].n_items) {
-        item -= p.g[gi].n_items;
-        ++gi;
-    }
-    const TcGroup& G = p.g[gi];
-    const int qb = item % G.n_qb;
-    const int h = (item / G.n_qb) % p.H;
-    const int b = item / (G.n_qb * p.H);
-    const int q_row0 = G.q_begin + qb * 2 * kBlockM;
-    const int n_tiles = G.n_tiles;
+    const long long T = p.total_tiles;
+    const long long ncta = gridDim.x;
+    const long long r0 = cta_begin(blockIdx.x, T, ncta);
+    const long long r1 = cta_begin(blockIdx.x + 1, T, ncta);
 
     if (threadIdx.x == 0) {
         abort_flag = 0;
+        merge_flag = 0;
         ptx::mbar_init(&q_full, 1);
+        ptx::mbar_init(&q_empty, 1);
         ptx::mbar_init(&o_full, 1);
+        ptx::mbar_init(&drain_bar, 1);
         for (int s = 0; s < kStages; ++s) {
             ptx::mbar_init(&k_full[s], 1);
             ptx::mbar_init(&k_empty[s], 1);
@@ -127,6 +202,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             ptx::mbar_init(&s_full[t], 1);
             ptx::mbar_init(&p_full[t], 128);
         }
+        ptx::mbar_init(&epi_written, 256);
+        ptx::mbar_init(&epi_decided, 1);
         ptx::fence_mbar_init();
     }
     if (warp == 2) {
@@ -138,27 +215,39 @@ __global__ void __launch_bounds__(kThreads, 1)
     ptx::tc_fence_after();
     const uint32_t tbase = tmem_base_sh;
     volatile int* abort_p = &abort_flag;
+    volatile int never = 0;
 
-    if (warp == 0) {
+    if (warp < 4) {
+        ptx::setmaxnreg_dec<kCtrlRegs>();
+        if (warp == 0) {
         // =========================== TMA producer ===========================
         if (lane == 0) {
             ptx::prefetch_tmap(&maps.q);
             bool ok = true;
-            ptx::mbar_arrive_expect_tx(&q_full, 2 * C::kTileBytes);
-            for (int t = 0; t < 2; ++t)
-                for (int c = 0; c < C::kChunks; ++c)
-                    ptx::tma_load_4d(sQ + t * C::kTileBytes + c * (kBlockM * 128), &maps.q, &q_full,
-                                     c * 64, h, q_row0 + t * kBlockM, b);
-            int issued = 0;
-            for (int si = 0; si < G.n_seg && ok; ++si) {
-                const TcSeg& sg = G.seg[si];
-                const CUtensorMap* mk = &maps.k[sg.map];
-                const CUtensorMap* mv = &maps.v[sg.map];
-                for (int kt = 0; kt < sg.ntiles; ++kt) {
-                    const int j = issued;
-                    const int st = j % kStages;
-                    const uint32_t ph = (uint32_t)((j / kStages) & 1);
-                    const int row = sg.row0 + kt * kBlockN;
+            long long js = 0;  // global K/V step
+            int piece = 0;
+            bool q_in_flight = false;
+            for (long long t = r0; t < r1 && ok; ++piece) {
+                const Piece pc = locate(p, t, r1);
+                const TcGroup& G = p.g[pc.gi];
+                if (!ptx::mbar_wait_bounded(&q_empty, (uint32_t)((piece & 1) ^ 1), abort_p,
+                                            p.wait_limit)) {
+                    ok = false;
+                    break;
+                }
+                ptx::mbar_arrive_expect_tx(&q_full, 2 * C::kTileBytes);
+                for (int qt = 0; qt < 2; ++qt)
+                    for (int c = 0; c < C::kChunks; ++c)
+                        ptx::tma_load_4d(sQ + qt * C::kTileBytes + c * (kBlockM * 128), &maps.q,
+                                         &q_full, c * 64, pc.h, pc.q_row0 + qt * kBlockM, pc.b);
+                q_in_flight = true;
+                for (int u = pc.u0; u < pc.u1; ++u, ++js) {
+                    int seg, row, valid;
+                    tile_info(G, u, seg, row, valid);
+                    const CUtensorMap* mk = &maps.k[G.seg[seg].map];
+                    const CUtensorMap* mv = &maps.v[G.seg[seg].map];
+                    const int st = (int)(js % kStages);
+                    const uint32_t ph = (uint32_t)((js / kStages) & 1);
                     if (!ptx::mbar_wait_bounded(&k_empty[st], ph ^ 1u, abort_p, p.wait_limit)) {
                         ok = false;
                         break;
@@ -166,10 +255,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ptx::mbar_arrive_expect_tx(&k_full[st], C::kTileBytes);
                     for (int c = 0; c < C::kChunks; ++c)
                         ptx::tma_load_4d(sK + st * C::kTileBytes + c * (kBlockN * 128), mk,
-                                         &k_full[st], c * 64, h, row, b);
+                                         &k_full[st], c * 64, pc.h, row, pc.b);
                     if (!ptx::mbar_wait_bounded(&v_empty[st], ph ^ 1u, abort_p, p.wait_limit)) {
-                        // K of this step is in flight: let it land before leaving
-                        volatile int never = 0;
                         ptx::mbar_wait_bounded(&k_full[st], ph, &never, kWaitLimit);
                         ok = false;
                         break;
@@ -177,16 +264,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ptx::mbar_arrive_expect_tx(&v_full[st], C::kTileBytes);
                     for (int c = 0; c < C::kChunks; ++c)
                         ptx::tma_load_4d(sV + st * C::kTileBytes + c * (kBlockN * 128), mv,
-                                         &v_full[st], c * 64, h, row, b);
-                    ++issued;
+                                         &v_full[st], c * 64, pc.h, row, pc.b);
                 }
+                t += pc.u1 - pc.u0;
             }
             if (!ok) {
                 // Drain: every copy issued must land before the CTA exits.
-                volatile int never = 0;
-                ptx::mbar_wait_bounded(&q_full, 0, &never, kWaitLimit);
-                for (int j = (issued > kStages ? issued - kStages : 0); j < issued; ++j) {
-                    const int st = j % kStages;
+                if (q_in_flight)
+                    ptx::mbar_wait_bounded(&q_full, (uint32_t)((piece - 1) & 1), &never, kWaitLimit);
+                for (long long j = (js > kStages ? js - kStages : 0); j < js; ++j) {
+                    const int st = (int)(j % kStages);
                     const uint32_t ph = (uint32_t)((j / kStages) & 1);
                     ptx::mbar_wait_bounded(&k_full[st], ph, &never, kWaitLimit);
                     ptx::mbar_wait_bounded(&v_full[st], ph, &never, kWaitLimit);
@@ -194,7 +281,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 atomicOr(p.status, kDevTimeout);
             }
         }
-    } else if (warp == 1) {
+        } else if (warp == 1) {
         // ============================ MMA issuer ============================
         if (lane == 0) {
             constexpr uint32_t idS = ptx::idesc_bf16(kBlockM, kBlockN, false, false);
@@ -222,51 +309,66 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 (acc || kk > 0) ? 1u : 0u);
                 }
             };
-            bool ok = ptx::mbar_wait_bounded(&q_full, 0, abort_p, p.wait_limit);
-            ok = ok && ptx::mbar_wait_bounded(&k_full[0], 0, abort_p, p.wait_limit);
-            if (ok) {
-                ptx::tc_fence_after();
-                issue_s(0, 0);
-                issue_s(1, 0);
-                ptx::mma_commit(&k_empty[0]);
-            }
-            for (int j = 0; j < n_tiles && ok; ++j) {
-                const int st = j % kStages;
-                const uint32_t ph = (uint32_t)((j / kStages) & 1);
-                const int st1 = (j + 1) % kStages;
-                const uint32_t ph1 = (uint32_t)(((j + 1) / kStages) & 1);
-                const bool more = j + 1 < n_tiles;
-                ok = ptx::mbar_wait_bounded(&v_full[st], ph, abort_p, p.wait_limit) &&
-                     ptx::mbar_wait_bounded(&p_full[0], (uint32_t)(j & 1), abort_p, p.wait_limit);
+            bool ok = true;
+            long long js = 0;
+            int piece = 0;
+            for (long long t = r0; t < r1 && ok; ++piece) {
+                const Piece pc = locate(p, t, r1);
+                const int n = pc.u1 - pc.u0;
+                const int st0 = (int)(js % kStages);
+                ok = ptx::mbar_wait_bounded(&q_full, (uint32_t)(piece & 1), abort_p, p.wait_limit) &&
+                     ptx::mbar_wait_bounded(&k_full[st0], (uint32_t)((js / kStages) & 1), abort_p,
+                                            p.wait_limit);
                 if (!ok) break;
                 ptx::tc_fence_after();
-                issue_pv(0, st, j > 0);
-                if (more) {
-                    ok = ptx::mbar_wait_bounded(&k_full[st1], ph1, abort_p, p.wait_limit);
+                issue_s(0, st0);
+                issue_s(1, st0);
+                ptx::mma_commit(&k_empty[st0]);
+                if (n == 1) ptx::mma_commit(&q_empty);
+                for (int jl = 0; jl < n; ++jl) {
+                    const long long j = js + jl;
+                    const int st = (int)(j % kStages);
+                    const uint32_t ph = (uint32_t)((j / kStages) & 1);
+                    const int st1 = (int)((j + 1) % kStages);
+                    const uint32_t ph1 = (uint32_t)(((j + 1) / kStages) & 1);
+                    const bool more = jl + 1 < n;
+                    ok = ptx::mbar_wait_bounded(&v_full[st], ph, abort_p, p.wait_limit) &&
+                         ptx::mbar_wait_bounded(&p_full[0], (uint32_t)(j & 1), abort_p, p.wait_limit);
                     if (!ok) break;
                     ptx::tc_fence_after();
-                    issue_s(0, st1);
+                    issue_pv(0, st, jl > 0);
+                    if (more) {
+                        ok = ptx::mbar_wait_bounded(&k_full[st1], ph1, abort_p, p.wait_limit);
+                        if (!ok) break;
+                        ptx::tc_fence_after();
+                        issue_s(0, st1);
+                    }
+                    ok = ptx::mbar_wait_bounded(&p_full[1], (uint32_t)(j & 1), abort_p, p.wait_limit);
+                    if (!ok) break;
+                    ptx::tc_fence_after();
+                    issue_pv(1, st, jl > 0);
+                    ptx::mma_commit(&v_empty[st]);
+                    if (more) {
+                        issue_s(1, st1);
+                        ptx::mma_commit(&k_empty[st1]);
+                        if (jl + 2 == n) ptx::mma_commit(&q_empty);  // last use of Q issued
+                    }
                 }
-                ok = ptx::mbar_wait_bounded(&p_full[1], (uint32_t)(j & 1), abort_p, p.wait_limit);
                 if (!ok) break;
-                ptx::tc_fence_after();
-                issue_pv(1, st, j > 0);
-                ptx::mma_commit(&v_empty[st]);
-                if (more) {
-                    issue_s(1, st1);
-                    ptx::mma_commit(&k_empty[st1]);
-                }
+                ptx::mma_commit(&o_full);
+                js += n;
+                t += n;
             }
-            // o_full covers every MMA issued, on the normal and the abort path,
-            // so TMEM is never released under a running MMA.
-            ptx::mma_commit(&o_full);
             if (!ok) {
-                volatile int never = 0;
-                ptx::mbar_wait_bounded(&o_full, 0, &never, kWaitLimit);
+                // drain_bar covers every MMA issued: TMEM is never released under one.
+                ptx::mma_commit(&drain_bar);
+                ptx::mbar_wait_bounded(&drain_bar, 0, &never, kWaitLimit);
                 atomicOr(p.status, kDevTimeout);
             }
         }
-    } else if (warp >= 4) {
+        }
+    } else {
+        ptx::setmaxnreg_inc<kSoftmaxRegs>();
         // ============================== softmax =============================
         const int t = (warp - 4) / 4;
         const int wq = warp % 4;
@@ -275,14 +377,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t tS = tbase + t * 128 + lane_off;
         const uint32_t tO = tbase + 256 + t * 128 + lane_off;
         const float sl2 = p.scale_log2;
-        float m_used = -INFINITY, l = 0.f;
         bool ok = true;
-        int j = 0;
-        for (int si = 0; si < G.n_seg && ok; ++si) {
-            const TcSeg& sg = G.seg[si];
-            for (int kt = 0; kt < sg.ntiles; ++kt, ++j) {
-                const int valid = min(kBlockN, sg.len - kt * kBlockN);
-                ok = ptx::mbar_wait_bounded(&s_full[t], (uint32_t)(j & 1), abort_p, p.wait_limit);
+        long long js = 0;
+        int piece = 0, nsplit = 0;
+        for (long long tt = r0; tt < r1 && ok; ++piece) {
+            const Piece pc = locate(p, tt, r1);
+            const TcGroup& G = p.g[pc.gi];
+            float m_used = -INFINITY, l = 0.f;
+            for (int u = pc.u0; u < pc.u1; ++u, ++js) {
+                int seg, row, valid;
+                tile_info(G, u, seg, row, valid);
+                ok = ptx::mbar_wait_bounded(&s_full[t], (uint32_t)(js & 1), abort_p, p.wait_limit);
                 ok = __all_sync(0xffffffffu, ok);
                 if (!ok) break;
                 ptx::tc_fence_after();
@@ -290,20 +395,25 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                 for (int q4 = 0; q4 < 4; ++q4) ptx::tmem_ld32(tS + 32 * q4, s[q4]);
                 ptx::tmem_wait_ld();
-                float mx = -INFINITY;
+                float mx[8];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) mx[e] = -INFINITY;
                 if (valid == kBlockN) {
 #pragma unroll
-                    for (int c = 0; c < 128; ++c) mx = fmaxf(mx, __uint_as_float(s[c >> 5][c & 31]));
+                    for (int c = 0; c < 128; ++c)
+                        mx[c & 7] = fmaxf(mx[c & 7], __uint_as_float(s[c >> 5][c & 31]));
                 } else {
 #pragma unroll
                     for (int c = 0; c < 128; ++c)
-                        if (c < valid) mx = fmaxf(mx, __uint_as_float(s[c >> 5][c & 31]));
+                        if (c < valid) mx[c & 7] = fmaxf(mx[c & 7], __uint_as_float(s[c >> 5][c & 31]));
                 }
-                const float m_new = fmaxf(m_used, mx * sl2);
-                if (j == 0) {
+                const float m_tile = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                                           fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+                const float m_new = fmaxf(m_used, m_tile * sl2);
+                if (u == pc.u0) {
                     m_used = m_new;
                 } else if (__any_sync(0xffffffffu, m_new > m_used + 8.0f)) {
-                    // O_t holds every PV up to step j-1 (the S_t(j) commit covers it).
+                    // O_t holds every PV up to the previous step (the S_t commit covers it).
                     const float f = ex2(m_used - m_new);
                     l *= f;
                     m_used = m_new;
@@ -319,66 +429,167 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ptx::tmem_wait_st();
                 }
                 const float nm = -m_used;
-                float sum = 0.f;
+                float sm[4] = {0.f, 0.f, 0.f, 0.f};
                 if (valid == kBlockN) {
 #pragma unroll
-                    for (int c = 0; c < 64; ++c) {
-                        const float p0 = ex2(fmaf(__uint_as_float(s[(2 * c) >> 5][(2 * c) & 31]), sl2, nm));
-                        const float p1 = ex2(fmaf(__uint_as_float(s[(2 * c + 1) >> 5][(2 * c + 1) & 31]), sl2, nm));
-                        sum += p0 + p1;
-                        s[c >> 5][c & 31] = ptx::pack_bf16(p0, p1);
+                    for (int q4 = 0; q4 < 4; ++q4) {
+                        uint32_t pk[16];
+#pragma unroll
+                        for (int c = 0; c < 16; ++c) {
+                            const float p0 = ex2(fmaf(__uint_as_float(s[q4][2 * c]), sl2, nm));
+                            const float p1 = ex2(fmaf(__uint_as_float(s[q4][2 * c + 1]), sl2, nm));
+                            sm[c & 3] += p0 + p1;
+                            pk[c] = ptx::pack_bf16(p0, p1);
+                        }
+                        ptx::tmem_st16(tS + 16 * q4, pk);
                     }
                 } else {
 #pragma unroll
-                    for (int c = 0; c < 64; ++c) {
-                        const float p0 =
-                            (2 * c < valid) ? ex2(fmaf(__uint_as_float(s[(2 * c) >> 5][(2 * c) & 31]), sl2, nm)) : 0.f;
-                        const float p1 = (2 * c + 1 < valid)
-                                             ? ex2(fmaf(__uint_as_float(s[(2 * c + 1) >> 5][(2 * c + 1) & 31]), sl2, nm))
-                                             : 0.f;
-                        sum += p0 + p1;
-                        s[c >> 5][c & 31] = ptx::pack_bf16(p0, p1);
+                    for (int q4 = 0; q4 < 4; ++q4) {
+                        uint32_t pk[16];
+#pragma unroll
+                        for (int c = 0; c < 16; ++c) {
+                            const int c0 = q4 * 32 + 2 * c;
+                            const float p0 =
+                                c0 < valid ? ex2(fmaf(__uint_as_float(s[q4][2 * c]), sl2, nm)) : 0.f;
+                            const float p1 =
+                                c0 + 1 < valid ? ex2(fmaf(__uint_as_float(s[q4][2 * c + 1]), sl2, nm)) : 0.f;
+                            sm[c & 3] += p0 + p1;
+                            pk[c] = ptx::pack_bf16(p0, p1);
+                        }
+                        ptx::tmem_st16(tS + 16 * q4, pk);
                     }
                 }
-                l += sum;
-                ptx::tmem_st32(tS + 0, s[0]);
-                ptx::tmem_st32(tS + 32, s[1]);
+                l += (sm[0] + sm[1]) + (sm[2] + sm[3]);
                 ptx::tmem_wait_st();
                 ptx::tc_fence_before();
                 ptx::mbar_arrive(&p_full[t]);
             }
-        }
-        if (ok) {
-            ok = ptx::mbar_wait_bounded(&o_full, 0, abort_p, p.wait_limit);
+            if (!ok) break;
+            ok = ptx::mbar_wait_bounded(&o_full, (uint32_t)(piece & 1), abort_p, p.wait_limit);
             ok = __all_sync(0xffffffffu, ok);
-        }
-        if (ok) {
+            if (!ok) break;
             ptx::tc_fence_after();
-            const int qrow = q_row0 + t * kBlockM + r;
+            const int qrow = pc.q_row0 + t * kBlockM + r;
             const bool store = qrow < G.q_end;
-            const float inv = 1.0f / l;
-            __nv_bfloat16* dst = p.out + (size_t)b * p.out_bstride +
-                                 ((size_t)qrow * p.H + h) * D;
+            __nv_bfloat16* dst =
+                p.out + (size_t)pc.b * p.out_bstride + ((size_t)qrow * p.H + pc.h) * D;
+            if (pc.whole) {
+                const float inv = 1.0f / l;
 #pragma unroll
-            for (int c = 0; c < D / 32; ++c) {
-                uint32_t o[32];
-                ptx::tmem_ld32(tO + c * 32, o);
-                ptx::tmem_wait_ld();
-                uint32_t pk[16];
+                for (int c = 0; c < D / 32; ++c) {
+                    uint32_t o[32];
+                    ptx::tmem_ld32(tO + c * 32, o);
+                    ptx::tmem_wait_ld();
+                    uint32_t pk[16];
 #pragma unroll
-                for (int e = 0; e < 16; ++e)
-                    pk[e] = ptx::pack_bf16(__uint_as_float(o[2 * e]) * inv,
-                                           __uint_as_float(o[2 * e + 1]) * inv);
-                if (store) {
-                    uint4* d4 = reinterpret_cast<uint4*>(dst + c * 32);
+                    for (int e = 0; e < 16; ++e)
+                        pk[e] = ptx::pack_bf16(__uint_as_float(o[2 * e]) * inv,
+                                               __uint_as_float(o[2 * e + 1]) * inv);
+                    if (store) {
+                        uint4* d4 = reinterpret_cast<uint4*>(dst + c * 32);
 #pragma unroll
-                    for (int e = 0; e < 4; ++e)
-                        d4[e] = make_uint4(pk[4 * e], pk[4 * e + 1], pk[4 * e + 2], pk[4 * e + 3]);
+                        for (int e = 0; e < 4; ++e)
+                            d4[e] = make_uint4(pk[4 * e], pk[4 * e + 1], pk[4 * e + 2], pk[4 * e + 3]);
+                    }
+                }
+            } else {
+                // ---- split item: write this piece's partial result
+                const long long c1 = cta_of(pc.item_start, T, ncta);
+                const long long c2 = cta_of(pc.item_start + G.n_tiles - 1, T, ncta);
+                const int slot = slot_of(blockIdx.x, c1, pc.item_start, T, ncta);
+                float* ps = p.partials + (size_t)slot * C::kSlotFloats;
+                float* prow = ps + (size_t)(t * kBlockM + r) * D;
+#pragma unroll
+                for (int c = 0; c < D / 32; ++c) {
+                    uint32_t o[32];
+                    ptx::tmem_ld32(tO + c * 32, o);
+                    ptx::tmem_wait_ld();
+                    float4* d4 = reinterpret_cast<float4*>(prow + c * 32);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+                        d4[e] = make_float4(__uint_as_float(o[4 * e]), __uint_as_float(o[4 * e + 1]),
+                                            __uint_as_float(o[4 * e + 2]), __uint_as_float(o[4 * e + 3]));
+                }
+                float* pml = ps + (size_t)2 * kBlockM * D + (size_t)(t * kBlockM + r) * 2;
+                pml[0] = m_used;
+                pml[1] = l;
+                __threadfence();
+                ptx::mbar_arrive(&epi_written);
+                const uint32_t par = (uint32_t)(nsplit & 1);
+                ++nsplit;
+                if (warp == 4 && lane == 0) {
+                    // All 256 rows are written (and fenced): count this piece in.
+                    bool okw = ptx::mbar_wait_bounded(&epi_written, par, abort_p, p.wait_limit);
+                    int last = 0;
+                    if (okw) {
+                        unsigned int* cnt = p.counters + G.item_base + pc.item;
+                        const unsigned int old = atomicAdd(cnt, 1u);
+                        last = (old == (unsigned int)(c2 - c1));
+                        if (last) {
+                            atomicExch(cnt, 0u);
+                            __threadfence();
+                        }
+                    }
+                    merge_flag = last;
+                    ptx::mbar_arrive(&epi_decided);
+                }
+                ok = ptx::mbar_wait_bounded(&epi_decided, par, abort_p, p.wait_limit);
+                ok = __all_sync(0xffffffffu, ok);
+                if (!ok) break;
+                if (*(volatile int*)&merge_flag) {
+                    // ---- last piece: merge every piece of this item
+                    float M = -INFINITY;
+                    for (long long c = c1; c <= c2; ++c) {
+                        const float* q = p.partials +
+                                         (size_t)slot_of(c, c1, pc.item_start, T, ncta) * C::kSlotFloats +
+                                         (size_t)2 * kBlockM * D + (size_t)(t * kBlockM + r) * 2;
+                        M = fmaxf(M, __ldcg(q));
+                    }
+                    float L = 0.f;
+                    for (long long c = c1; c <= c2; ++c) {
+                        const float* q = p.partials +
+                                         (size_t)slot_of(c, c1, pc.item_start, T, ncta) * C::kSlotFloats +
+                                         (size_t)2 * kBlockM * D + (size_t)(t * kBlockM + r) * 2;
+                        L += ex2(__ldcg(q) - M) * __ldcg(q + 1);
+                    }
+                    const float inv = 1.0f / L;
+#pragma unroll 1
+                    for (int ch = 0; ch < D / 32; ++ch) {
+                        float acc[32];
+#pragma unroll
+                        for (int e = 0; e < 32; ++e) acc[e] = 0.f;
+                        for (long long c = c1; c <= c2; ++c) {
+                            const float* base =
+                                p.partials + (size_t)slot_of(c, c1, pc.item_start, T, ncta) * C::kSlotFloats;
+                            const float w =
+                                ex2(__ldcg(base + (size_t)2 * kBlockM * D + (size_t)(t * kBlockM + r) * 2) - M);
+                            const float4* src = reinterpret_cast<const float4*>(
+                                base + (size_t)(t * kBlockM + r) * D + ch * 32);
+#pragma unroll
+                            for (int e = 0; e < 8; ++e) {
+                                const float4 v = __ldcg(src + e);
+                                acc[4 * e] = fmaf(w, v.x, acc[4 * e]);
+                                acc[4 * e + 1] = fmaf(w, v.y, acc[4 * e + 1]);
+                                acc[4 * e + 2] = fmaf(w, v.z, acc[4 * e + 2]);
+                                acc[4 * e + 3] = fmaf(w, v.w, acc[4 * e + 3]);
+                            }
+                        }
+                        if (store) {
+                            uint4* d4 = reinterpret_cast<uint4*>(dst + ch * 32);
+#pragma unroll
+                            for (int e = 0; e < 4; ++e)
+                                d4[e] = make_uint4(ptx::pack_bf16(acc[8 * e] * inv, acc[8 * e + 1] * inv),
+                                                   ptx::pack_bf16(acc[8 * e + 2] * inv, acc[8 * e + 3] * inv),
+                                                   ptx::pack_bf16(acc[8 * e + 4] * inv, acc[8 * e + 5] * inv),
+                                                   ptx::pack_bf16(acc[8 * e + 6] * inv, acc[8 * e + 7] * inv));
+                        }
+                    }
                 }
             }
-        } else if (lane == 0) {
-            atomicOr(p.status, kDevTimeout);
+            tt += pc.u1 - pc.u0;
         }
+        if (!ok && lane == 0) atomicOr(p.status, kDevTimeout);
     }
 
     ptx::tc_fence_before();
@@ -433,6 +644,7 @@ struct TcCache {
     int key_rows[2 * kNumMaps + 1];
     bool valid[2 * kNumMaps + 1];
     bool attr_set[2];
+    int num_sms;
 };
 
 }  // namespace
@@ -448,6 +660,7 @@ void tc_cache_invalidate(msf_plan_t plan) {
     if (plan && plan->tc_cache) {
         TcCache* c = (TcCache*)plan->tc_cache;
         for (int i = 0; i < 2 * kNumMaps + 1; ++i) c->valid[i] = false;
+        c->num_sms = 0;
     }
 }
 
@@ -459,6 +672,17 @@ msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st) {
     }
     TcCache& cache = *(TcCache*)P.tc_cache;
     const long long row = (long long)P.H * P.D * 2;
+    cudaError_t e;
+    if (cache.num_sms == 0) {
+        int dev = 0, sms = 0;
+        e = cudaGetDevice(&dev);
+        if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        if (e != cudaSuccess) {
+            set_cuda_error((int)e);
+            return MSF_ERR_CUDA;
+        }
+        cache.num_sms = sms;
+    }
 
     auto ensure = [&](int slot, CUtensorMap* m, const void* base, int rows, long long bs) -> bool {
         if (cache.valid[slot] && cache.key_ptr[slot] == base && cache.key_rows[slot] == rows)
@@ -478,13 +702,15 @@ msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st) {
     tp.out = (__nv_bfloat16*)a.out;
     tp.out_bstride = (long long)P.N * P.H * P.D;
     tp.status = a.status;
+    tp.counters = attn_counters(P);
+    tp.partials = attn_partials(P);
     tp.wait_limit = kWaitLimit;
 
     if (!ensure(2 * kNumMaps, &cache.maps.q, a.q, P.N, a.q_bstride)) {
         set_cuda_error((int)cudaErrorInvalidValue);
         return MSF_ERR_CUDA;
     }
-    // Order groups by context length, longest first (their CTAs start first).
+    // Order groups by context length, longest first.
     int order[MSF_MAX_GROUPS];
     for (int i = 0; i < a.n_groups; ++i) order[i] = i;
     for (int i = 0; i < a.n_groups; ++i)
@@ -498,7 +724,8 @@ msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st) {
                 order[k] = tmp;
             }
         }
-    long long total_items = 0;
+    long long total_tiles = 0;
+    int item_base = 0;
     for (int oi = 0; oi < a.n_groups; ++oi) {
         const int gi = order[oi];
         const AttnGroup& ag = a.g[gi];
@@ -535,18 +762,33 @@ msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st) {
             ts.map = slot;
             ts.row0 = row0;
             ts.len = sg.len;
-            ts.ntiles = (sg.len + kBlockN - 1) / kBlockN;
-            tg.n_tiles += ts.ntiles;
+            ts.tile0 = tg.n_tiles;
+            tg.n_tiles += (sg.len + kBlockN - 1) / kBlockN;
         }
-        total_items += tg.n_items;
+        tg.tile_base = total_tiles;
+        tg.item_base = item_base;
+        total_tiles += (long long)tg.n_items * tg.n_tiles;
+        item_base += tg.n_items;
     }
     tp.n_groups = a.n_groups;
-    if (total_items == 0) return MSF_OK;
-    if (total_items > 0x7fffffffLL) return MSF_ERR_UNSUPPORTED;
+    tp.total_tiles = total_tiles;
+    if (total_tiles == 0) return MSF_OK;
+    if (item_base > P.attn_items) return MSF_ERR_STATE;
+    long long ncta = cache.num_sms;
+    if (ncta > P.attn_max_ctas) ncta = P.attn_max_ctas;
+    if (ncta > total_tiles) ncta = total_tiles;
+    if (ncta < 1) ncta = 1;
 
-    cudaError_t e;
     if (P.D == 128) {
         if (!cache.attr_set[1]) {
+            // The warpgroup register split assumes exactly kLaunchRegs per thread.
+            cudaFuncAttributes fa;
+            e = cudaFuncGetAttributes(&fa, mssa_tc_kernel<128>);
+            if (e != cudaSuccess) {
+                set_cuda_error((int)e);
+                return MSF_ERR_CUDA;
+            }
+            if (fa.numRegs != kLaunchRegs) return MSF_ERR_UNSUPPORTED;
             e = cudaFuncSetAttribute(mssa_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      Cfg<128>::kSmem);
             if (e != cudaSuccess) {
@@ -555,9 +797,17 @@ msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st) {
             }
             cache.attr_set[1] = true;
         }
-        mssa_tc_kernel<128><<<(unsigned)total_items, kThreads, Cfg<128>::kSmem, st>>>(cache.maps, tp);
+        note_launch();
+        mssa_tc_kernel<128><<<(unsigned)ncta, kThreads, Cfg<128>::kSmem, st>>>(cache.maps, tp);
     } else {
         if (!cache.attr_set[0]) {
+            cudaFuncAttributes fa;
+            e = cudaFuncGetAttributes(&fa, mssa_tc_kernel<64>);
+            if (e != cudaSuccess) {
+                set_cuda_error((int)e);
+                return MSF_ERR_CUDA;
+            }
+            if (fa.numRegs != kLaunchRegs) return MSF_ERR_UNSUPPORTED;
             e = cudaFuncSetAttribute(mssa_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      Cfg<64>::kSmem);
             if (e != cudaSuccess) {
@@ -566,7 +816,8 @@ msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st) {
             }
             cache.attr_set[0] = true;
         }
-        mssa_tc_kernel<64><<<(unsigned)total_items, kThreads, Cfg<64>::kSmem, st>>>(cache.maps, tp);
+        note_launch();
+        mssa_tc_kernel<64><<<(unsigned)ncta, kThreads, Cfg<64>::kSmem, st>>>(cache.maps, tp);
     }
     e = cudaGetLastError();
     if (e != cudaSuccess) {

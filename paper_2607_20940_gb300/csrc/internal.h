@@ -29,6 +29,9 @@ struct msf_plan {
     int n_groups;
     msf::Group groups[MSF_MAX_GROUPS];
     int pyr_tokens;   // per stream
+    // tensor-core attention scheduling state in the workspace
+    int attn_items;     // 256-row query blocks over all groups, streams and heads
+    int attn_max_ctas;  // persistent CTAs the partial-result slots are sized for
     size_t ws_bytes;
     float scale;      // softmax scale
 
@@ -64,14 +67,33 @@ inline size_t msp_scratch_bytes(const Plan& p) {
     size_t per = (size_t)p.d.latent_channels * p.d.patch * p.d.grid_h * p.d.patch * p.d.grid_w;
     return round256((size_t)p.B * p.T * per * p.elem);
 }
+// Tensor-core attention (bf16 plans): one merge counter per query block, and
+// two partial-result slots per persistent CTA, each [256 rows][D] fp32 output
+// followed by [256 rows][2] fp32 (running max, running sum).
+constexpr int kAttnMaxCtas = 160;
+constexpr int kAttnBlockRows = 256;
+inline size_t attn_counter_bytes(const Plan& p) {
+    return p.elem == 2 ? round256((size_t)p.attn_items * 4) : 0;
+}
+inline size_t attn_slot_floats(const Plan& p) { return (size_t)kAttnBlockRows * (p.D + 2); }
+inline size_t attn_partial_bytes(const Plan& p) {
+    return p.elem == 2 ? round256((size_t)2 * p.attn_max_ctas * attn_slot_floats(p) * 4) : 0;
+}
 inline size_t workspace_bytes(const Plan& p) {
-    return kStatusBytes + 2 * pyramid_bytes(p) + msp_scratch_bytes(p);
+    return kStatusBytes + 2 * pyramid_bytes(p) + msp_scratch_bytes(p) + attn_counter_bytes(p) +
+           attn_partial_bytes(p);
 }
 inline unsigned int* status_word(const Plan& p) { return (unsigned int*)p.ws; }
 inline char* pyr_k(const Plan& p) { return (char*)p.ws + kStatusBytes; }
 inline char* pyr_v(const Plan& p) { return (char*)p.ws + kStatusBytes + pyramid_bytes(p); }
 inline char* msp_scratch(const Plan& p) {
     return (char*)p.ws + kStatusBytes + 2 * pyramid_bytes(p);
+}
+inline unsigned int* attn_counters(const Plan& p) {
+    return (unsigned int*)(msp_scratch(p) + msp_scratch_bytes(p));
+}
+inline float* attn_partials(const Plan& p) {
+    return (float*)((char*)attn_counters(p) + attn_counter_bytes(p));
 }
 
 // Number of context tokens of group gi with the current history count.
@@ -91,6 +113,8 @@ inline int group_npyr(const Plan& p, int gi) {
 }
 
 void set_cuda_error(int e);
+// Count one kernel launch (see msf_kernel_launches).
+void note_launch();
 
 // Device status codes written into the status word.
 constexpr unsigned int kDevTimeout = 1u;

@@ -100,9 +100,9 @@ cudaError_t launch_pool(const PoolBatch& jobs, int batch, bool bf16, cudaStream_
     long long work = (long long)max_n * jobs.row_vecs;
     dim3 grid((unsigned)((work + 255) / 256), (unsigned)jobs.n, (unsigned)batch);
     if (bf16)
-        pool_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(jobs);
+        { note_launch(); pool_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(jobs); }
     else
-        pool_kernel<float><<<grid, 256, 0, st>>>(jobs);
+        { note_launch(); pool_kernel<float><<<grid, 256, 0, st>>>(jobs); }
     return cudaGetLastError();
 }
 
@@ -150,6 +150,7 @@ cudaError_t launch_patchify_raw(const void* latent, void* raw, const MspShape& s
                                 bool bf16, cudaStream_t st) {
     const int per = sh.C * sh.Hl * sh.Wl;
     dim3 grid((unsigned)((per + 255) / 256), (unsigned)sh.T, (unsigned)batch);
+    note_launch();
     if (bf16)
         patchify_raw_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(
             (const __nv_bfloat16*)latent, (__nv_bfloat16*)raw, sh);
@@ -163,6 +164,7 @@ cudaError_t launch_unpatchify_raw(const void* raw, void* latent, const MspShape&
                                   cudaStream_t st) {
     const int per = sh.C * sh.Hl * sh.Wl;
     dim3 grid((unsigned)((per + 255) / 256), 1, (unsigned)batch);
+    note_launch();
     if (bf16)
         unpatchify_raw_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(
             (const __nv_bfloat16*)raw, (__nv_bfloat16*)latent, sh, position, raw_bstride,
@@ -238,9 +240,9 @@ __global__ void __launch_bounds__(256) gemm_nt_simt_kernel(GemmArgs g) {
 cudaError_t launch_gemm_nt_simt(const GemmArgs& g, int batch, bool bf16, cudaStream_t st) {
     dim3 grid((unsigned)((g.N + 63) / 64), (unsigned)((g.M + 63) / 64), (unsigned)batch);
     if (bf16)
-        gemm_nt_simt_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(g);
+        { note_launch(); gemm_nt_simt_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(g); }
     else
-        gemm_nt_simt_kernel<float><<<grid, 256, 0, st>>>(g);
+        { note_launch(); gemm_nt_simt_kernel<float><<<grid, 256, 0, st>>>(g); }
     return cudaGetLastError();
 }
 

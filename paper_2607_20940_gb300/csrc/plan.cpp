@@ -4,14 +4,19 @@
 #include <stdlib.h>
 #include <string.h>
 
+#include <atomic>
 #include <new>
 
 #include "internal.h"
 
 namespace msf {
 static thread_local int g_last_cuda_error = 0;
+static std::atomic<uint64_t> g_launches{0};
 void set_cuda_error(int e) { g_last_cuda_error = e; }
+void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 }  // namespace msf
+
+extern "C" uint64_t msf_kernel_launches(void) { return msf::g_launches.load(); }
 
 using msf::Plan;
 
@@ -118,6 +123,28 @@ extern "C" msf_status msf_plan_create(const msf_plan_desc* desc, msf_plan_t* out
         }
     }
     p->pyr_tokens = pyr;
+    // Attention work: 256-row query blocks and 128-row context tiles, counted
+    // at full history (the most tiles the schedule can ever hold).
+    {
+        long long items = 0, tiles = 0;
+        for (int gi = 0; gi < ng; ++gi) {
+            const msf::Group& g = p->groups[gi];
+            long long it = (long long)p->B * p->H * ((g.q_end - g.q_begin + 255) / 256);
+            long long nt = (d.sink_tokens + 127) / 128 + (p->N - g.q_begin + 127) / 128;
+            if (g.scale == 1)
+                nt += ((long long)d.history_capacity * p->G + 127) / 128;
+            else
+                nt += ((long long)(d.history_capacity + g.n_finer) * g.pooled + 127) / 128;
+            items += it;
+            tiles += it * nt;
+        }
+        if (items > (1 << 30)) {
+            delete p;
+            return MSF_ERR_UNSUPPORTED;
+        }
+        p->attn_items = (int)items;
+        p->attn_max_ctas = (int)(tiles < msf::kAttnMaxCtas ? tiles : msf::kAttnMaxCtas);
+    }
     p->ws_bytes = msf::workspace_bytes(*p);
     p->hist_count = d.history_frames;
     p->hist_oldest = 0;

@@ -34,7 +34,7 @@ EXPORTS = (
     "msf_status_string", "msf_last_cuda_error", "msf_plan_create", "msf_plan_destroy",
     "msf_plan_query", "msf_plan_index_map", "msf_plan_bind", "msf_patchify", "msf_unpatchify",
     "msf_kv_resample", "msf_mssa_forward", "msf_mssa_forward_simt", "msf_history_append",
-    "msf_plan_device_status",
+    "msf_plan_device_status", "msf_kernel_launches",
 )
 
 
@@ -93,6 +93,7 @@ def _load():
         "msf_mssa_forward_simt": (ctypes.c_int, [P, VP, VP, VP, VP, VP]),
         "msf_history_append": (ctypes.c_int, [P, VP, VP, VP]),
         "msf_plan_device_status": (ctypes.c_int, [P, VP]),
+        "msf_kernel_launches": (ctypes.c_uint64, []),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -205,6 +206,10 @@ def msf_history_append(plan: int, k_win, v_win, stream=None) -> None:
 
 def msf_plan_device_status(plan: int, stream=None) -> int:
     return _lib.msf_plan_device_status(plan, _stream(stream))
+
+
+def msf_kernel_launches() -> int:
+    return int(_lib.msf_kernel_launches())
 
 
 # ------------------------------------------------------------ convenience
