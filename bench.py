@@ -232,7 +232,8 @@ def main():
     ws = plan.workspace(dev)
     plan.bind(ws, d["k_sink"], d["v_sink"], d["k_hist"], d["v_hist"])
     lat = mi["latent"].to(dev)
-    w_tier = [mi["w_tier"][s].t().contiguous().to(dev) for s in w.scales]
+    tiers = {s: mi["w_tier"][s].t().contiguous().to(dev) for s in set(w.scales)}
+    w_tier = [tiers[s] for s in w.scales]  # positions of one tier share its weight
     w_out = mi["w_out"].t().contiguous().to(dev)
     N, E = info.n_tokens, w.embed_dim
     tok = torch.empty((w.batch, N, E), dtype=torch.bfloat16, device=dev)

@@ -421,9 +421,14 @@ extern "C" msf_status msf_unpatchify(msf_plan_t plan, int32_t position, const vo
         t.a_bstride = (long long)p.N * E;
         t.c_bstride = per;
         t.status = msf::status_word(p);
+        t.C32 = msf::msp_split(p);
+        t.max_splits = msf::kMaxDeembedSplits;
         if (msf::gemm_tc_supported(t)) {
             cudaError_t e = msf::launch_gemm_tc(t, p.B, s);
             if (e != cudaSuccess) return cuda_status(e);
+            if (t.splits_used > 1)
+                return cuda_status(msf::launch_unpatchify_splitk(msf::msp_split(p), t.splits_used,
+                                                                 latent_out, sh, position, p.B, s));
             return cuda_status(
                 msf::launch_unpatchify_raw(raw, latent_out, sh, position, per, 0, p.B, bf16, s));
         }

@@ -4,12 +4,16 @@
 // to bf16. Used for the patch embedding of each tier (K = C*P^2, N = E) and
 // the de-embedding of an emitted state (K = E, N = C*P^2).
 //
-// One CTA computes a 128 x BN tile of one stream's problem:
+// One CTA computes a 128 x BN tile of one stream's problem (optionally one
+// K split of it):
 //   warp 0  TMA producer: 64-wide K chunks of A (128 rows) and B (BN rows),
-//           128-byte swizzled, into a kStages ring
+//           128-byte swizzled, into a STAGES ring
 //   warp 1  MMA issuer: 4 x tcgen05.mma (K = 16) per chunk, accumulator in TMEM
 //   warp 2  TMEM allocation
-//   warps 4-7 epilogue: tcgen05.ld of the accumulator rows, bf16 pack, stores
+//   warps 4-7 epilogue: tcgen05.ld of the accumulator rows, then either a
+//           bf16 pack and store, or fp32 partial sums of a K split
+// The shared-memory ring and TMEM columns are small enough for 2-4 CTAs per
+// SM, so short problems overlap one CTA's loads with another's epilogue.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -25,9 +29,9 @@ namespace {
 constexpr int kThreads = 256;
 constexpr long long kWaitLimit = 2000000000LL;
 
-template <int BN>
+template <int BN, int STAGES>
 struct GCfg {
-    static constexpr int kStages = BN >= 256 ? 4 : 6;
+    static constexpr int kStages = STAGES;
     static constexpr int kABytes = 128 * 128;    // 128 rows x 64 bf16
     static constexpr int kBBytes = BN * 128;     // BN rows x 64 bf16
     static constexpr int kStageBytes = kABytes + kBBytes;
@@ -37,9 +41,11 @@ struct GCfg {
 
 struct GemmTcParams {
     int M, N, K;
-    __nv_bfloat16* C;
+    int batch, splits;    // grid.z = batch * splits
+    __nv_bfloat16* C;     // splits == 1: bf16 output
     long long ldc;        // elements
     long long c_bstride;  // elements
+    float* C32;           // splits > 1: fp32 partial sums [split][batch][M][N]
     unsigned int* status;
 };
 struct GemmTcMaps {
@@ -47,18 +53,21 @@ struct GemmTcMaps {
     CUtensorMap b;  // {K, N}
 };
 
-template <int BN>
+template <int BN, int STAGES>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ GemmTcMaps maps, const __grid_constant__ GemmTcParams p) {
-    using C = GCfg<BN>;
+    using C = GCfg<BN, STAGES>;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     __shared__ uint64_t full[C::kStages], empty[C::kStages], acc_full;
     __shared__ uint32_t tmem_base_sh;
     __shared__ int abort_flag;
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-    const int m0 = blockIdx.x * 128, n0 = blockIdx.y * BN, b = blockIdx.z;
-    const int nk = (p.K + 63) / 64;
+    const int m0 = blockIdx.x * 128, n0 = blockIdx.y * BN;
+    const int b = blockIdx.z % p.batch, split = blockIdx.z / p.batch;
+    const int nk_all = (p.K + 63) / 64;
+    const int kc0 = (int)((long long)split * nk_all / p.splits);
+    const int nk = (int)((long long)(split + 1) * nk_all / p.splits) - kc0;
 
     if (threadIdx.x == 0) {
         abort_flag = 0;
@@ -93,8 +102,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             unsigned char* sa = smem + st * C::kStageBytes;
             ptx::mbar_arrive_expect_tx(&full[st], C::kStageBytes);
-            ptx::tma_load_3d(sa, &maps.a, &full[st], kc * 64, m0, b);
-            ptx::tma_load_2d(sa + C::kABytes, &maps.b, &full[st], kc * 64, n0);
+            ptx::tma_load_3d(sa, &maps.a, &full[st], (kc0 + kc) * 64, m0, b);
+            ptx::tma_load_2d(sa + C::kABytes, &maps.b, &full[st], (kc0 + kc) * 64, n0);
             ++issued;
         }
         if (!ok) {
@@ -140,26 +149,46 @@ __global__ void __launch_bounds__(kThreads, 1)
             ptx::tc_fence_after();
             const int m = m0 + r;
             const bool store = m < p.M;
-            __nv_bfloat16* crow = p.C + (size_t)b * p.c_bstride + (size_t)m * p.ldc + n0;
             const uint32_t taddr = tbase + ((uint32_t)(wq * 32) << 16);
+            if (p.splits == 1) {
+                __nv_bfloat16* crow = p.C + (size_t)b * p.c_bstride + (size_t)m * p.ldc + n0;
 #pragma unroll 1
-            for (int c = 0; c < BN / 32; ++c) {
-                uint32_t v[32];
-                ptx::tmem_ld32(taddr + c * 32, v);
-                ptx::tmem_wait_ld();
-                uint32_t pk[16];
+                for (int c = 0; c < BN / 32; ++c) {
+                    uint32_t v[32];
+                    ptx::tmem_ld32(taddr + c * 32, v);
+                    ptx::tmem_wait_ld();
+                    uint32_t pk[16];
 #pragma unroll
-                for (int e = 0; e < 16; ++e)
-                    pk[e] = ptx::pack_bf16(__uint_as_float(v[2 * e]), __uint_as_float(v[2 * e + 1]));
-                const int ncol = n0 + c * 32;
-                if (store && ncol + 32 <= p.N) {
-                    uint4* d4 = reinterpret_cast<uint4*>(crow + c * 32);
+                    for (int e = 0; e < 16; ++e)
+                        pk[e] = ptx::pack_bf16(__uint_as_float(v[2 * e]), __uint_as_float(v[2 * e + 1]));
+                    const int ncol = n0 + c * 32;
+                    if (store && ncol + 32 <= p.N) {
+                        uint4* d4 = reinterpret_cast<uint4*>(crow + c * 32);
 #pragma unroll
-                    for (int e = 0; e < 4; ++e)
-                        d4[e] = make_uint4(pk[4 * e], pk[4 * e + 1], pk[4 * e + 2], pk[4 * e + 3]);
-                } else if (store) {
-                    const __nv_bfloat16* hb = reinterpret_cast<const __nv_bfloat16*>(pk);
-                    for (int e = 0; e < 32 && ncol + e < p.N; ++e) crow[c * 32 + e] = hb[e];
+                        for (int e = 0; e < 4; ++e)
+                            d4[e] = make_uint4(pk[4 * e], pk[4 * e + 1], pk[4 * e + 2], pk[4 * e + 3]);
+                    } else if (store) {
+                        const __nv_bfloat16* hb = reinterpret_cast<const __nv_bfloat16*>(pk);
+                        for (int e = 0; e < 32 && ncol + e < p.N; ++e) crow[c * 32 + e] = hb[e];
+                    }
+                }
+            } else {
+                float* crow = p.C32 + (((size_t)split * p.batch + b) * p.M + m) * p.N + n0;
+#pragma unroll 1
+                for (int c = 0; c < BN / 32; ++c) {
+                    uint32_t v[32];
+                    ptx::tmem_ld32(taddr + c * 32, v);
+                    ptx::tmem_wait_ld();
+                    const int ncol = n0 + c * 32;
+                    if (store && ncol + 32 <= p.N) {
+                        float4* d4 = reinterpret_cast<float4*>(crow + c * 32);
+#pragma unroll
+                        for (int e = 0; e < 8; ++e)
+                            d4[e] = make_float4(__uint_as_float(v[4 * e]), __uint_as_float(v[4 * e + 1]),
+                                                __uint_as_float(v[4 * e + 2]), __uint_as_float(v[4 * e + 3]));
+                    } else if (store) {
+                        for (int e = 0; e < 32 && ncol + e < p.N; ++e) crow[c * 32 + e] = __uint_as_float(v[e]);
+                    }
                 }
             }
         } else if (lane == 0) {
@@ -192,8 +221,8 @@ EncodeTiledFn encoder() {
     return fn;
 }
 
-template <int BN>
-cudaError_t launch_bn(const GemmTcArgs& g, int batch, cudaStream_t st) {
+template <int BN, int STAGES>
+cudaError_t launch_bn(const GemmTcArgs& g, int batch, int splits, cudaStream_t st) {
     EncodeTiledFn enc = encoder();
     if (!enc) return cudaErrorNotSupported;
     GemmTcMaps maps;
@@ -222,20 +251,25 @@ cudaError_t launch_bn(const GemmTcArgs& g, int batch, cudaStream_t st) {
     p.M = g.M;
     p.N = g.N;
     p.K = g.K;
+    p.batch = batch;
+    p.splits = splits;
     p.C = (__nv_bfloat16*)g.C;
     p.ldc = g.ldc;
     p.c_bstride = g.c_bstride;
+    p.C32 = g.C32;
     p.status = g.status;
     static bool attr = false;
     if (!attr) {
-        cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, GCfg<BN>::kSmem);
+        cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             GCfg<BN, STAGES>::kSmem);
         if (e != cudaSuccess) return e;
         attr = true;
     }
-    dim3 grid((unsigned)((g.M + 127) / 128), (unsigned)((g.N + BN - 1) / BN), (unsigned)batch);
+    dim3 grid((unsigned)((g.M + 127) / 128), (unsigned)((g.N + BN - 1) / BN),
+              (unsigned)(batch * splits));
     note_launch();
-    gemm_tc_kernel<BN><<<grid, kThreads, GCfg<BN>::kSmem, st>>>(maps, p);
+    gemm_tc_kernel<BN, STAGES><<<grid, kThreads, GCfg<BN, STAGES>::kSmem, st>>>(maps, p);
     return cudaGetLastError();
 }
 
@@ -251,9 +285,23 @@ bool gemm_tc_supported(const GemmTcArgs& g) {
 }
 
 cudaError_t launch_gemm_tc(const GemmTcArgs& g, int batch, cudaStream_t st) {
-    if (g.N <= 64) return launch_bn<64>(g, batch, st);
-    if (g.N <= 128) return launch_bn<128>(g, batch, st);
-    return launch_bn<256>(g, batch, st);
+    // Few, long tiles (the de-embedding: K = E, N = C*P^2): split K across
+    // CTAs into fp32 partial sums when the caller provides room for them.
+    if (g.C32 && g.max_splits > 1) {
+        const int tiles = ((g.M + 127) / 128) * ((g.N + 127) / 128) * batch;
+        const int nk = g.K / 64;
+        int splits = 1;
+        while (splits * 2 <= g.max_splits && tiles * splits * 2 <= 160 && nk / (splits * 2) >= 2)
+            splits *= 2;
+        g.splits_used = splits;
+        if (splits > 1) {
+            if (g.N <= 64) return launch_bn<64, 4>(g, batch, splits, st);
+            return launch_bn<128, 4>(g, batch, splits, st);
+        }
+    }
+    g.splits_used = 1;
+    if (g.N <= 64) return launch_bn<64, 4>(g, batch, 1, st);
+    return launch_bn<128, 2>(g, batch, 1, st);
 }
 
 }  // namespace msf

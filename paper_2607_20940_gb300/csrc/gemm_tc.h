@@ -16,6 +16,12 @@ struct GemmTcArgs {
     long long lda, ldb, ldc;       // elements
     long long a_bstride, c_bstride;  // elements
     unsigned int* status;
+    // Optional split-K: room for max_splits fp32 partial outputs
+    // [split][batch][M][N] (contiguous). The launcher reports the split count
+    // it used in splits_used; 1 means C was written directly.
+    float* C32 = nullptr;
+    int max_splits = 1;
+    mutable int splits_used = 1;
 };
 
 bool gemm_tc_supported(const GemmTcArgs& g);

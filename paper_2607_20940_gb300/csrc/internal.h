@@ -79,9 +79,16 @@ inline size_t attn_slot_floats(const Plan& p) { return (size_t)kAttnBlockRows * 
 inline size_t attn_partial_bytes(const Plan& p) {
     return p.elem == 2 ? round256((size_t)2 * p.attn_max_ctas * attn_slot_floats(p) * 4) : 0;
 }
+// fp32 partial sums of a split-K de-embedding: [splits][B][C*Hl*Wl].
+constexpr int kMaxDeembedSplits = 8;
+inline size_t msp_split_bytes(const Plan& p) {
+    if (p.d.latent_channels <= 0 || p.d.patch <= 0 || p.elem != 2) return 0;
+    size_t per = (size_t)p.d.latent_channels * p.d.patch * p.d.grid_h * p.d.patch * p.d.grid_w;
+    return round256((size_t)kMaxDeembedSplits * p.B * per * 4);
+}
 inline size_t workspace_bytes(const Plan& p) {
     return kStatusBytes + 2 * pyramid_bytes(p) + msp_scratch_bytes(p) + attn_counter_bytes(p) +
-           attn_partial_bytes(p);
+           attn_partial_bytes(p) + msp_split_bytes(p);
 }
 inline unsigned int* status_word(const Plan& p) { return (unsigned int*)p.ws; }
 inline char* pyr_k(const Plan& p) { return (char*)p.ws + kStatusBytes; }
@@ -94,6 +101,9 @@ inline unsigned int* attn_counters(const Plan& p) {
 }
 inline float* attn_partials(const Plan& p) {
     return (float*)((char*)attn_counters(p) + attn_counter_bytes(p));
+}
+inline float* msp_split(const Plan& p) {
+    return (float*)((char*)attn_partials(p) + attn_partial_bytes(p));
 }
 
 // Number of context tokens of group gi with the current history count.

@@ -42,6 +42,11 @@ cudaError_t launch_unpatchify_raw(const void* raw, void* latent, const MspShape&
                                   long long raw_bstride, int raw_offset, int batch, bool bf16,
                                   cudaStream_t st);
 
+// Sum `splits` fp32 partial token blocks [split][B][N_l * C*P^2] (fixed
+// order), round once to bf16 and rearrange into the latent [B, C, Hl, Wl].
+cudaError_t launch_unpatchify_splitk(const float* part, int splits, void* latent, const MspShape& sh,
+                                     int position, int batch, cudaStream_t st);
+
 struct GemmArgs {
     const void* A;  // [M, K] (+ a_bstride per batch), element strides
     const void* B;  // [N, K]

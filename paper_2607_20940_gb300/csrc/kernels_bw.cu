@@ -175,6 +175,36 @@ cudaError_t launch_unpatchify_raw(const void* raw, void* latent, const MspShape&
     return cudaGetLastError();
 }
 
+__global__ void __launch_bounds__(256) unpatchify_splitk_kernel(const float* __restrict__ part,
+                                                                int splits,
+                                                                __nv_bfloat16* __restrict__ latent,
+                                                                MspShape sh, int position,
+                                                                int batch) {
+    const int b = blockIdx.z;
+    const int per = sh.C * sh.Hl * sh.Wl;
+    const int o = blockIdx.x * blockDim.x + threadIdx.x;
+    if (o >= per) return;
+    const int P = sh.patch * sh.scales[position];
+    const int PP = P * P, F = sh.C * PP, gw = sh.Wl / P;
+    const int c = o / (sh.Hl * sh.Wl), yx = o - c * (sh.Hl * sh.Wl);
+    const int y = yx / sh.Wl, x = yx - (yx / sh.Wl) * sh.Wl;
+    const int i = y / P, dy = y - i * P, j = x / P, dx = x - j * P;
+    const size_t src = (size_t)(i * gw + j) * F + c * PP + dy * P + dx;
+    float acc = 0.f;
+    for (int sp = 0; sp < splits; ++sp) acc += __ldg(part + ((size_t)sp * batch + b) * per + src);
+    latent[(size_t)b * per + o] = __float2bfloat16_rn(acc);
+}
+
+cudaError_t launch_unpatchify_splitk(const float* part, int splits, void* latent, const MspShape& sh,
+                                     int position, int batch, cudaStream_t st) {
+    const int per = sh.C * sh.Hl * sh.Wl;
+    dim3 grid((unsigned)((per + 255) / 256), 1, (unsigned)batch);
+    note_launch();
+    unpatchify_splitk_kernel<<<grid, 256, 0, st>>>(part, splits, (__nv_bfloat16*)latent, sh, position,
+                                                   batch);
+    return cudaGetLastError();
+}
+
 // --------------------------------------------------------- CUDA-core GEMM
 //
 // C[m, n] = sum_k A[m, k] * B[n, k] (both operands K-contiguous), fp32

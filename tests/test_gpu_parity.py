@@ -186,14 +186,19 @@ def test_patchify_unpatchify_raw_bit_exact(dtype):
         assert torch.equal(back.cpu(), m["latent"][:, l])
 
 
-def test_patchify_embed_and_unpatchify_deembed():
+@pytest.mark.parametrize("shared", [True, False], ids=["tier_weights", "per_position_weights"])
+def test_patchify_embed_and_unpatchify_deembed(shared):
     w = dataclasses.replace(synth.LAYER_480P, batch=2, heads=12)
     plan, _ = _msp_plan(w, BF16, True)
     m = synth.msp_inputs(w, BF16)
     lat = m["latent"].cuda()
     E = w.embed_dim
     N = plan.info.n_tokens
-    w_tier = [m["w_tier"][s].t().contiguous().cuda() for s in w.scales]  # [E, C*P^2]
+    if shared:
+        tiers = {s: m["w_tier"][s].t().contiguous().cuda() for s in set(w.scales)}  # [E, C*P^2]
+        w_tier = [tiers[s] for s in w.scales]
+    else:
+        w_tier = [m["w_tier"][s].t().contiguous().cuda() for s in w.scales]
     tok = torch.empty((w.batch, N, E), dtype=BF16, device="cuda")
     plan.patchify(lat, w_tier, tok)
     torch.cuda.synchronize()
