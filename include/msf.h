@@ -224,6 +224,26 @@ msf_status msf_history_append(msf_plan_t plan, const void* k_win, const void* v_
  * all devices), for accounting in benchmarks. Host only. */
 uint64_t msf_kernel_launches(void);
 
+/* Allocation-free variant of msf_unpatchify with a de-embedding weight. The
+ * paper has no counterpart: this exists for callers that cannot allocate
+ * device memory (hosts that hand out every device buffer from their own pool
+ * and forbid libraries to call cudaMalloc), so it needs no bound workspace.
+ * Same arguments and result as msf_unpatchify(plan, position, tokens, w_out,
+ * latent_out, stream) with w_out != NULL, for bf16 plans with an embedding.
+ * Its scratch (raw tokens and split-K fp32 partial sums) is a fixed 8 MiB
+ * device array inside the library, held by every GPU that loads it until the
+ * process exits; a problem needs B * C*Hl*Wl * 2 bytes (rounded up to 256)
+ * plus 256 bytes of it, and larger ones are rejected with
+ * MSF_ERR_UNSUPPORTED. The first call on each device looks up that array's
+ * device address (cudaGetSymbolAddress, with that device current); make that
+ * first call before any stream capture. It calls no cudaMalloc/cudaFree. Every
+ * call shares the one array and overwrites it, so calls that overlap on the
+ * GPU (different streams, or threads without ordering) race: serialise them.
+ * Errors: INVALID_ARG, UNSUPPORTED (fp32 plan, no embedding, shape too
+ * large), CUDA. */
+msf_status msf_unpatchify_noalloc(msf_plan_t plan, int32_t position, const void* tokens,
+                                  const void* w_out, void* latent_out, void* stream);
+
 /* Synchronise `stream`, read and clear the device status word. Returns
  * MSF_ERR_TIMEOUT if a kernel gave up on a bounded wait since the last
  * check, MSF_OK otherwise. */

@@ -34,7 +34,7 @@ EXPORTS = (
     "msf_status_string", "msf_last_cuda_error", "msf_plan_create", "msf_plan_destroy",
     "msf_plan_query", "msf_plan_index_map", "msf_plan_bind", "msf_patchify", "msf_unpatchify",
     "msf_kv_resample", "msf_mssa_forward", "msf_mssa_forward_simt", "msf_history_append",
-    "msf_plan_device_status", "msf_kernel_launches",
+    "msf_plan_device_status", "msf_kernel_launches", "msf_unpatchify_noalloc",
 )
 
 
@@ -94,6 +94,7 @@ def _load():
         "msf_history_append": (ctypes.c_int, [P, VP, VP, VP]),
         "msf_plan_device_status": (ctypes.c_int, [P, VP]),
         "msf_kernel_launches": (ctypes.c_uint64, []),
+        "msf_unpatchify_noalloc": (ctypes.c_int, [P, I32, VP, VP, VP, VP]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -206,6 +207,11 @@ def msf_history_append(plan: int, k_win, v_win, stream=None) -> None:
 
 def msf_plan_device_status(plan: int, stream=None) -> int:
     return _lib.msf_plan_device_status(plan, _stream(stream))
+
+
+def msf_unpatchify_noalloc(plan: int, position: int, tokens, w_out, latent_out, stream=None) -> None:
+    _check(_lib.msf_unpatchify_noalloc(plan, position, _ptr(tokens), _ptr(w_out), _ptr(latent_out),
+                                       _stream(stream)), "msf_unpatchify_noalloc")
 
 
 def msf_kernel_launches() -> int:
