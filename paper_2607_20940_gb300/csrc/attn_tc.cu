@@ -13,7 +13,8 @@
 // workspace, reset by the merger).
 //
 // Roles inside a CTA (384 threads):
-//   warp 0      TMA producer: Q0/Q1 per piece, then K_j, V_j into a 2-stage ring
+//   warp 0      TMA producer: Q0/Q1 per piece, then K_j and V_{j-1} into
+//               2-stage rings, both gated by one release per tile
 //   warp 1      MMA issuer (one thread): S_t = Q_t K_j^T into TMEM (SS form),
 //               O_t += P_t V_j with P_t read from TMEM (TS form, V MN-major)
 //   warp 2      TMEM allocation (all 512 columns)
@@ -172,7 +173,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     unsigned char* sV = sK + kStages * C::kTileBytes;          // [kStages][tile]
 
     __shared__ uint64_t q_full, q_empty, o_full, drain_bar;
-    __shared__ uint64_t k_full[kStages], k_empty[kStages], v_full[kStages], v_empty[kStages];
+    __shared__ uint64_t k_full[kStages], k_empty[kStages], v_full[kStages];
     __shared__ uint64_t s_full[2], p_full[2];
     __shared__ uint64_t epi_written, epi_decided;
     __shared__ uint32_t tmem_base_sh;
@@ -196,13 +197,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             ptx::mbar_init(&k_full[s], 1);
             ptx::mbar_init(&k_empty[s], 1);
             ptx::mbar_init(&v_full[s], 1);
-            ptx::mbar_init(&v_empty[s], 1);
         }
         for (int t = 0; t < 2; ++t) {
             ptx::mbar_init(&s_full[t], 1);
-            ptx::mbar_init(&p_full[t], 128);
+            ptx::mbar_init(&p_full[t], 4);   // one arrival per softmax warp
         }
-        ptx::mbar_init(&epi_written, 256);
+        ptx::mbar_init(&epi_written, 8);
         ptx::mbar_init(&epi_decided, 1);
         ptx::fence_mbar_init();
     }
@@ -227,6 +227,22 @@ __global__ void __launch_bounds__(kThreads, 1)
             long long js = 0;  // global K/V step
             int piece = 0;
             bool q_in_flight = false;
+            // V of tile j is issued right after K of tile j+1: both wait for the
+            // same release, the k_empty commit that follows S1 of tile j-1 (it
+            // covers the PV of tile j-2, the last reader of V's slot).
+            bool v_pending = false;
+            const CUtensorMap* pv_map = nullptr;
+            int pv_row = 0, pv_h = 0, pv_b = 0;
+            long long v_issued = 0;
+            auto issue_v = [&]() {
+                const int st = (int)(v_issued % kStages);
+                ptx::mbar_arrive_expect_tx(&v_full[st], C::kTileBytes);
+                for (int c = 0; c < C::kChunks; ++c)
+                    ptx::tma_load_4d(sV + st * C::kTileBytes + c * (kBlockN * 128), pv_map,
+                                     &v_full[st], c * 64, pv_h, pv_row, pv_b);
+                ++v_issued;
+                v_pending = false;
+            };
             for (long long t = r0; t < r1 && ok; ++piece) {
                 const Piece pc = locate(p, t, r1);
                 const TcGroup& G = p.g[pc.gi];
@@ -245,7 +261,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                     int seg, row, valid;
                     tile_info(G, u, seg, row, valid);
                     const CUtensorMap* mk = &maps.k[G.seg[seg].map];
-                    const CUtensorMap* mv = &maps.v[G.seg[seg].map];
                     const int st = (int)(js % kStages);
                     const uint32_t ph = (uint32_t)((js / kStages) & 1);
                     if (!ptx::mbar_wait_bounded(&k_empty[st], ph ^ 1u, abort_p, p.wait_limit)) {
@@ -256,28 +271,34 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int c = 0; c < C::kChunks; ++c)
                         ptx::tma_load_4d(sK + st * C::kTileBytes + c * (kBlockN * 128), mk,
                                          &k_full[st], c * 64, pc.h, row, pc.b);
-                    if (!ptx::mbar_wait_bounded(&v_empty[st], ph ^ 1u, abort_p, p.wait_limit)) {
-                        ptx::mbar_wait_bounded(&k_full[st], ph, &never, kWaitLimit);
-                        ok = false;
-                        break;
-                    }
-                    ptx::mbar_arrive_expect_tx(&v_full[st], C::kTileBytes);
-                    for (int c = 0; c < C::kChunks; ++c)
-                        ptx::tma_load_4d(sV + st * C::kTileBytes + c * (kBlockN * 128), mv,
-                                         &v_full[st], c * 64, pc.h, row, pc.b);
+                    if (v_pending) issue_v();
+                    v_pending = true;
+                    pv_map = &maps.v[G.seg[seg].map];
+                    pv_row = row;
+                    pv_h = pc.h;
+                    pv_b = pc.b;
                 }
                 t += pc.u1 - pc.u0;
+            }
+            if (ok && v_pending) {
+                // The last V waits for the release the next K would wait for.
+                const int st = (int)(js % kStages);
+                const uint32_t ph = (uint32_t)((js / kStages) & 1);
+                if (ptx::mbar_wait_bounded(&k_empty[st], ph ^ 1u, abort_p, p.wait_limit))
+                    issue_v();
+                else
+                    ok = false;
             }
             if (!ok) {
                 // Drain: every copy issued must land before the CTA exits.
                 if (q_in_flight)
                     ptx::mbar_wait_bounded(&q_full, (uint32_t)((piece - 1) & 1), &never, kWaitLimit);
-                for (long long j = (js > kStages ? js - kStages : 0); j < js; ++j) {
-                    const int st = (int)(j % kStages);
-                    const uint32_t ph = (uint32_t)((j / kStages) & 1);
-                    ptx::mbar_wait_bounded(&k_full[st], ph, &never, kWaitLimit);
-                    ptx::mbar_wait_bounded(&v_full[st], ph, &never, kWaitLimit);
-                }
+                for (long long j = (js > kStages ? js - kStages : 0); j < js; ++j)
+                    ptx::mbar_wait_bounded(&k_full[j % kStages], (uint32_t)((j / kStages) & 1), &never,
+                                           kWaitLimit);
+                for (long long j = (v_issued > kStages ? v_issued - kStages : 0); j < v_issued; ++j)
+                    ptx::mbar_wait_bounded(&v_full[j % kStages], (uint32_t)((j / kStages) & 1), &never,
+                                           kWaitLimit);
                 atomicOr(p.status, kDevTimeout);
             }
         }
@@ -347,7 +368,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (!ok) break;
                     ptx::tc_fence_after();
                     issue_pv(1, st, jl > 0);
-                    ptx::mma_commit(&v_empty[st]);
                     if (more) {
                         issue_s(1, st1);
                         ptx::mma_commit(&k_empty[st1]);
@@ -395,20 +415,21 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                 for (int q4 = 0; q4 < 4; ++q4) ptx::tmem_ld32(tS + 32 * q4, s[q4]);
                 ptx::tmem_wait_ld();
+                if (valid < kBlockN) {
+                    // Rows past the segment's end: score -inf, probability 0.
+#pragma unroll
+                    for (int c = 0; c < 128; ++c)
+                        if (c >= valid) s[c >> 5][c & 31] = 0xff800000u;
+                }
                 float mx[8];
 #pragma unroll
                 for (int e = 0; e < 8; ++e) mx[e] = -INFINITY;
-                if (valid == kBlockN) {
 #pragma unroll
-                    for (int c = 0; c < 128; ++c)
-                        mx[c & 7] = fmaxf(mx[c & 7], __uint_as_float(s[c >> 5][c & 31]));
-                } else {
-#pragma unroll
-                    for (int c = 0; c < 128; ++c)
-                        if (c < valid) mx[c & 7] = fmaxf(mx[c & 7], __uint_as_float(s[c >> 5][c & 31]));
-                }
-                const float m_tile = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
-                                           fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+                for (int c = 0; c < 128; c += 2)
+                    mx[(c >> 1) & 7] = ptx::fmax3(mx[(c >> 1) & 7], __uint_as_float(s[c >> 5][c & 31]),
+                                                  __uint_as_float(s[c >> 5][(c & 31) + 1]));
+                const float m_tile = fmaxf(ptx::fmax3(mx[0], mx[1], mx[2]),
+                                           fmaxf(ptx::fmax3(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7])));
                 const float m_new = fmaxf(m_used, m_tile * sl2);
                 if (u == pc.u0) {
                     m_used = m_new;
@@ -429,41 +450,34 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ptx::tmem_wait_st();
                 }
                 const float nm = -m_used;
-                float sm[4] = {0.f, 0.f, 0.f, 0.f};
-                if (valid == kBlockN) {
+                const uint64_t sl2x2 = ptx::f2_pack(sl2, sl2), nmx2 = ptx::f2_pack(nm, nm);
+                uint64_t sum2[2] = {ptx::f2_pack(0.f, 0.f), ptx::f2_pack(0.f, 0.f)};
 #pragma unroll
-                    for (int q4 = 0; q4 < 4; ++q4) {
-                        uint32_t pk[16];
+                for (int q4 = 0; q4 < 4; ++q4) {
+                    uint32_t pk[16];
 #pragma unroll
-                        for (int c = 0; c < 16; ++c) {
-                            const float p0 = ex2(fmaf(__uint_as_float(s[q4][2 * c]), sl2, nm));
-                            const float p1 = ex2(fmaf(__uint_as_float(s[q4][2 * c + 1]), sl2, nm));
-                            sm[c & 3] += p0 + p1;
-                            pk[c] = ptx::pack_bf16(p0, p1);
-                        }
-                        ptx::tmem_st16(tS + 16 * q4, pk);
+                    for (int c = 0; c < 16; ++c) {
+                        const uint64_t arg = ptx::f2_fma(
+                            ptx::f2_pack(__uint_as_float(s[q4][2 * c]), __uint_as_float(s[q4][2 * c + 1])),
+                            sl2x2, nmx2);
+                        float a0, a1;
+                        ptx::f2_unpack(arg, a0, a1);
+                        const float p0 = ex2(a0), p1 = ex2(a1);
+                        sum2[c & 1] = ptx::f2_add(sum2[c & 1], ptx::f2_pack(p0, p1));
+                        pk[c] = ptx::pack_bf16(p0, p1);
                     }
-                } else {
-#pragma unroll
-                    for (int q4 = 0; q4 < 4; ++q4) {
-                        uint32_t pk[16];
-#pragma unroll
-                        for (int c = 0; c < 16; ++c) {
-                            const int c0 = q4 * 32 + 2 * c;
-                            const float p0 =
-                                c0 < valid ? ex2(fmaf(__uint_as_float(s[q4][2 * c]), sl2, nm)) : 0.f;
-                            const float p1 =
-                                c0 + 1 < valid ? ex2(fmaf(__uint_as_float(s[q4][2 * c + 1]), sl2, nm)) : 0.f;
-                            sm[c & 3] += p0 + p1;
-                            pk[c] = ptx::pack_bf16(p0, p1);
-                        }
-                        ptx::tmem_st16(tS + 16 * q4, pk);
-                    }
+                    ptx::tmem_st16(tS + 16 * q4, pk);
                 }
-                l += (sm[0] + sm[1]) + (sm[2] + sm[3]);
+                {
+                    float a0, a1, b0, b1;
+                    ptx::f2_unpack(sum2[0], a0, a1);
+                    ptx::f2_unpack(sum2[1], b0, b1);
+                    l += (a0 + a1) + (b0 + b1);
+                }
                 ptx::tmem_wait_st();
                 ptx::tc_fence_before();
-                ptx::mbar_arrive(&p_full[t]);
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(&p_full[t]);
             }
             if (!ok) break;
             ok = ptx::mbar_wait_bounded(&o_full, (uint32_t)(piece & 1), abort_p, p.wait_limit);
@@ -515,7 +529,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 pml[0] = m_used;
                 pml[1] = l;
                 __threadfence();
-                ptx::mbar_arrive(&epi_written);
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(&epi_written);
                 const uint32_t par = (uint32_t)(nsplit & 1);
                 ++nsplit;
                 if (warp == 4 && lane == 0) {
