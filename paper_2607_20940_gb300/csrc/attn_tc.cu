@@ -98,7 +98,10 @@ struct Cfg {
     static constexpr int kChunks = D / 64;                    // 128-byte swizzle chunks per row
     static constexpr int kTileBytes = kBlockM * D * 2;        // one Q / K / V tile
     static constexpr int kSmem = (2 + 2 * kStages) * kTileBytes + 1024;
+    // Partial slot: output as [D/4 float4][256 rows] then [2][256 rows] (running
+    // max, running sum), so that the 32 rows of a warp touch consecutive words.
     static constexpr int kSlotFloats = 2 * kBlockM * (D + 2);
+    static constexpr int kSlotML = 2 * kBlockM * D;
 };
 
 __device__ __forceinline__ float ex2(float x) {
@@ -512,22 +515,22 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const long long c1 = cta_of(pc.item_start, T, ncta);
                 const long long c2 = cta_of(pc.item_start + G.n_tiles - 1, T, ncta);
                 const int slot = slot_of(blockIdx.x, c1, pc.item_start, T, ncta);
+                const int rr = t * kBlockM + r;
                 float* ps = p.partials + (size_t)slot * C::kSlotFloats;
-                float* prow = ps + (size_t)(t * kBlockM + r) * D;
+                float4* po = reinterpret_cast<float4*>(ps) + rr;
 #pragma unroll
                 for (int c = 0; c < D / 32; ++c) {
                     uint32_t o[32];
                     ptx::tmem_ld32(tO + c * 32, o);
                     ptx::tmem_wait_ld();
-                    float4* d4 = reinterpret_cast<float4*>(prow + c * 32);
 #pragma unroll
                     for (int e = 0; e < 8; ++e)
-                        d4[e] = make_float4(__uint_as_float(o[4 * e]), __uint_as_float(o[4 * e + 1]),
-                                            __uint_as_float(o[4 * e + 2]), __uint_as_float(o[4 * e + 3]));
+                        po[(size_t)(c * 8 + e) * 2 * kBlockM] =
+                            make_float4(__uint_as_float(o[4 * e]), __uint_as_float(o[4 * e + 1]),
+                                        __uint_as_float(o[4 * e + 2]), __uint_as_float(o[4 * e + 3]));
                 }
-                float* pml = ps + (size_t)2 * kBlockM * D + (size_t)(t * kBlockM + r) * 2;
-                pml[0] = m_used;
-                pml[1] = l;
+                ps[C::kSlotML + rr] = m_used;
+                ps[C::kSlotML + 2 * kBlockM + rr] = l;
                 __threadfence();
                 __syncwarp();
                 if (lane == 0) ptx::mbar_arrive(&epi_written);
@@ -554,19 +557,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!ok) break;
                 if (*(volatile int*)&merge_flag) {
                     // ---- last piece: merge every piece of this item
+                    const int rr = t * kBlockM + r;
                     float M = -INFINITY;
                     for (long long c = c1; c <= c2; ++c) {
                         const float* q = p.partials +
-                                         (size_t)slot_of(c, c1, pc.item_start, T, ncta) * C::kSlotFloats +
-                                         (size_t)2 * kBlockM * D + (size_t)(t * kBlockM + r) * 2;
-                        M = fmaxf(M, __ldcg(q));
+                                         (size_t)slot_of(c, c1, pc.item_start, T, ncta) * C::kSlotFloats;
+                        M = fmaxf(M, __ldcg(q + C::kSlotML + rr));
                     }
                     float L = 0.f;
                     for (long long c = c1; c <= c2; ++c) {
                         const float* q = p.partials +
-                                         (size_t)slot_of(c, c1, pc.item_start, T, ncta) * C::kSlotFloats +
-                                         (size_t)2 * kBlockM * D + (size_t)(t * kBlockM + r) * 2;
-                        L += ex2(__ldcg(q) - M) * __ldcg(q + 1);
+                                         (size_t)slot_of(c, c1, pc.item_start, T, ncta) * C::kSlotFloats;
+                        L += ex2(__ldcg(q + C::kSlotML + rr) - M) * __ldcg(q + C::kSlotML + 2 * kBlockM + rr);
                     }
                     const float inv = 1.0f / L;
 #pragma unroll 1
@@ -577,13 +579,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                         for (long long c = c1; c <= c2; ++c) {
                             const float* base =
                                 p.partials + (size_t)slot_of(c, c1, pc.item_start, T, ncta) * C::kSlotFloats;
-                            const float w =
-                                ex2(__ldcg(base + (size_t)2 * kBlockM * D + (size_t)(t * kBlockM + r) * 2) - M);
-                            const float4* src = reinterpret_cast<const float4*>(
-                                base + (size_t)(t * kBlockM + r) * D + ch * 32);
+                            const float w = ex2(__ldcg(base + C::kSlotML + rr) - M);
+                            const float4* src = reinterpret_cast<const float4*>(base) + rr;
 #pragma unroll
                             for (int e = 0; e < 8; ++e) {
-                                const float4 v = __ldcg(src + e);
+                                const float4 v = __ldcg(src + (size_t)(ch * 8 + e) * 2 * kBlockM);
                                 acc[4 * e] = fmaf(w, v.x, acc[4 * e]);
                                 acc[4 * e + 1] = fmaf(w, v.y, acc[4 * e + 1]);
                                 acc[4 * e + 2] = fmaf(w, v.z, acc[4 * e + 2]);
