@@ -13,8 +13,8 @@
 // workspace, reset by the merger).
 //
 // Roles inside a CTA (384 threads):
-//   warp 0      TMA producer: Q0/Q1 per piece, then K_j and V_{j-1} into
-//               2-stage rings, both gated by one release per tile
+//   warp 0      TMA producer: Q0/Q1 per piece, then K_j and V_j into a
+//               2-deep K ring and a 3-deep V ring, gated by one release per tile
 //   warp 1      MMA issuer (one thread): S_t = Q_t K_j^T into TMEM (SS form),
 //               O_t += P_t V_j with P_t read from TMEM (TS form, V MN-major)
 //   warp 2      TMEM allocation (all 512 columns)
@@ -45,7 +45,8 @@ namespace {
 
 constexpr int kBlockM = 128;   // query rows per tile
 constexpr int kBlockN = 128;   // context rows per K/V tile
-constexpr int kStages = 2;     // K/V ring depth
+constexpr int kStages = 2;     // K ring depth
+constexpr int kVStages = 3;    // V ring depth
 constexpr int kThreads = 384;  // 12 warps
 // Registers: 168 per thread at launch (12 warps x 168 = 64512 of 65536). The
 // producer/MMA warpgroup drops to 120 and the two softmax warpgroups rise to
@@ -97,7 +98,7 @@ template <int D>
 struct Cfg {
     static constexpr int kChunks = D / 64;                    // 128-byte swizzle chunks per row
     static constexpr int kTileBytes = kBlockM * D * 2;        // one Q / K / V tile
-    static constexpr int kSmem = (2 + 2 * kStages) * kTileBytes + 1024;
+    static constexpr int kSmem = (2 + kStages + kVStages) * kTileBytes + 1024;
     // Partial slot: output as [D/4 float4][256 rows] then [2][256 rows] (running
     // max, running sum), so that the 32 rows of a warp touch consecutive words.
     static constexpr int kSlotFloats = 2 * kBlockM * (D + 2);
@@ -173,10 +174,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     unsigned char* sQ = smem;                                  // [2][tile]
     unsigned char* sK = smem + 2 * C::kTileBytes;              // [kStages][tile]
-    unsigned char* sV = sK + kStages * C::kTileBytes;          // [kStages][tile]
+    unsigned char* sV = sK + kStages * C::kTileBytes;          // [kVStages][tile]
 
     __shared__ uint64_t q_full, q_empty, o_full, drain_bar;
-    __shared__ uint64_t k_full[kStages], k_empty[kStages], v_full[kStages];
+    __shared__ uint64_t k_full[kStages], k_empty[kStages], v_full[kVStages];
     __shared__ uint64_t s_full[2], p_full[2];
     __shared__ uint64_t epi_written, epi_decided;
     __shared__ uint32_t tmem_base_sh;
@@ -199,8 +200,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int s = 0; s < kStages; ++s) {
             ptx::mbar_init(&k_full[s], 1);
             ptx::mbar_init(&k_empty[s], 1);
-            ptx::mbar_init(&v_full[s], 1);
         }
+        for (int s = 0; s < kVStages; ++s) ptx::mbar_init(&v_full[s], 1);
         for (int t = 0; t < 2; ++t) {
             ptx::mbar_init(&s_full[t], 1);
             ptx::mbar_init(&p_full[t], 4);   // one arrival per softmax warp
@@ -230,22 +231,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             long long js = 0;  // global K/V step
             int piece = 0;
             bool q_in_flight = false;
-            // V of tile j is issued right after K of tile j+1: both wait for the
-            // same release, the k_empty commit that follows S1 of tile j-1 (it
-            // covers the PV of tile j-2, the last reader of V's slot).
-            bool v_pending = false;
-            const CUtensorMap* pv_map = nullptr;
-            int pv_row = 0, pv_h = 0, pv_b = 0;
-            long long v_issued = 0;
-            auto issue_v = [&]() {
-                const int st = (int)(v_issued % kStages);
-                ptx::mbar_arrive_expect_tx(&v_full[st], C::kTileBytes);
-                for (int c = 0; c < C::kChunks; ++c)
-                    ptx::tma_load_4d(sV + st * C::kTileBytes + c * (kBlockN * 128), pv_map,
-                                     &v_full[st], c * 64, pv_h, pv_row, pv_b);
-                ++v_issued;
-                v_pending = false;
-            };
+            // K(j) and V(j) wait for one release: the commit that follows S1 of
+            // tile j-2. It covers the last reader of K(j)'s slot (S of tile
+            // j-2) and of V(j)'s slot in the 3-deep V ring (PV1 of tile j-3).
             for (long long t = r0; t < r1 && ok; ++piece) {
                 const Piece pc = locate(p, t, r1);
                 const TcGroup& G = p.g[pc.gi];
@@ -274,23 +262,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int c = 0; c < C::kChunks; ++c)
                         ptx::tma_load_4d(sK + st * C::kTileBytes + c * (kBlockN * 128), mk,
                                          &k_full[st], c * 64, pc.h, row, pc.b);
-                    if (v_pending) issue_v();
-                    v_pending = true;
-                    pv_map = &maps.v[G.seg[seg].map];
-                    pv_row = row;
-                    pv_h = pc.h;
-                    pv_b = pc.b;
+                    const int sv = (int)(js % kVStages);
+                    ptx::mbar_arrive_expect_tx(&v_full[sv], C::kTileBytes);
+                    for (int c = 0; c < C::kChunks; ++c)
+                        ptx::tma_load_4d(sV + sv * C::kTileBytes + c * (kBlockN * 128),
+                                         &maps.v[G.seg[seg].map], &v_full[sv], c * 64, pc.h, row, pc.b);
                 }
                 t += pc.u1 - pc.u0;
-            }
-            if (ok && v_pending) {
-                // The last V waits for the release the next K would wait for.
-                const int st = (int)(js % kStages);
-                const uint32_t ph = (uint32_t)((js / kStages) & 1);
-                if (ptx::mbar_wait_bounded(&k_empty[st], ph ^ 1u, abort_p, p.wait_limit))
-                    issue_v();
-                else
-                    ok = false;
             }
             if (!ok) {
                 // Drain: every copy issued must land before the CTA exits.
@@ -299,8 +277,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (long long j = (js > kStages ? js - kStages : 0); j < js; ++j)
                     ptx::mbar_wait_bounded(&k_full[j % kStages], (uint32_t)((j / kStages) & 1), &never,
                                            kWaitLimit);
-                for (long long j = (v_issued > kStages ? v_issued - kStages : 0); j < v_issued; ++j)
-                    ptx::mbar_wait_bounded(&v_full[j % kStages], (uint32_t)((j / kStages) & 1), &never,
+                for (long long j = (js > kVStages ? js - kVStages : 0); j < js; ++j)
+                    ptx::mbar_wait_bounded(&v_full[j % kVStages], (uint32_t)((j / kVStages) & 1), &never,
                                            kWaitLimit);
                 atomicOr(p.status, kDevTimeout);
             }
@@ -351,16 +329,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (n == 1) ptx::mma_commit(&q_empty);
                 for (int jl = 0; jl < n; ++jl) {
                     const long long j = js + jl;
-                    const int st = (int)(j % kStages);
-                    const uint32_t ph = (uint32_t)((j / kStages) & 1);
+                    const int sv = (int)(j % kVStages);
+                    const uint32_t phv = (uint32_t)((j / kVStages) & 1);
                     const int st1 = (int)((j + 1) % kStages);
                     const uint32_t ph1 = (uint32_t)(((j + 1) / kStages) & 1);
                     const bool more = jl + 1 < n;
-                    ok = ptx::mbar_wait_bounded(&v_full[st], ph, abort_p, p.wait_limit) &&
+                    ok = ptx::mbar_wait_bounded(&v_full[sv], phv, abort_p, p.wait_limit) &&
                          ptx::mbar_wait_bounded(&p_full[0], (uint32_t)(j & 1), abort_p, p.wait_limit);
                     if (!ok) break;
                     ptx::tc_fence_after();
-                    issue_pv(0, st, jl > 0);
+                    issue_pv(0, sv, jl > 0);
                     if (more) {
                         ok = ptx::mbar_wait_bounded(&k_full[st1], ph1, abort_p, p.wait_limit);
                         if (!ok) break;
@@ -370,7 +348,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ok = ptx::mbar_wait_bounded(&p_full[1], (uint32_t)(j & 1), abort_p, p.wait_limit);
                     if (!ok) break;
                     ptx::tc_fence_after();
-                    issue_pv(1, st, jl > 0);
+                    issue_pv(1, sv, jl > 0);
                     if (more) {
                         issue_s(1, st1);
                         ptx::mma_commit(&k_empty[st1]);
