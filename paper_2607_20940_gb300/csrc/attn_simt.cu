@@ -12,6 +12,7 @@
 #include <math.h>
 
 #include "kernels.h"
+#include "ptx.cuh"
 
 namespace msf {
 
@@ -30,6 +31,8 @@ __device__ __forceinline__ __nv_bfloat16 tot(float x) { return __float2bfloat16_
 
 template <typename T, int D>
 __global__ void __launch_bounds__(128) attn_simt_kernel(const AttnArgs a) {
+    ptx::grid_dep_wait();
+    ptx::grid_dep_launch();
     constexpr int DP = D / 4;
     constexpr int KT = 32;
     __shared__ float Ks[KT][D];
@@ -107,14 +110,14 @@ cudaError_t launch_attn_simt(const AttnArgs& a, bool bf16, cudaStream_t st) {
     dim3 grid((unsigned)tiles, (unsigned)a.H, (unsigned)a.B);
     if (a.D == 128) {
         if (bf16)
-            { note_launch(); attn_simt_kernel<__nv_bfloat16, 128><<<grid, 128, 0, st>>>(a); }
+            return launch_pdl(attn_simt_kernel<__nv_bfloat16, 128>, grid, dim3(128), 0, st, a);
         else
-            { note_launch(); attn_simt_kernel<float, 128><<<grid, 128, 0, st>>>(a); }
+            return launch_pdl(attn_simt_kernel<float, 128>, grid, dim3(128), 0, st, a);
     } else {
         if (bf16)
-            { note_launch(); attn_simt_kernel<__nv_bfloat16, 64><<<grid, 128, 0, st>>>(a); }
+            return launch_pdl(attn_simt_kernel<__nv_bfloat16, 64>, grid, dim3(128), 0, st, a);
         else
-            { note_launch(); attn_simt_kernel<float, 64><<<grid, 128, 0, st>>>(a); }
+            return launch_pdl(attn_simt_kernel<float, 64>, grid, dim3(128), 0, st, a);
     }
     return cudaGetLastError();
 }

@@ -220,6 +220,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tbase = tmem_base_sh;
     volatile int* abort_p = &abort_flag;
     volatile int never = 0;
+    ptx::grid_dep_wait();  // q/k/v and the pyramid of the previous kernels are visible
+    ptx::grid_dep_launch();
 
     if (warp < 4) {
         ptx::setmaxnreg_dec<kCtrlRegs>();
@@ -790,8 +792,8 @@ msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st) {
             }
             cache.attr_set[1] = true;
         }
-        note_launch();
-        mssa_tc_kernel<128><<<(unsigned)ncta, kThreads, Cfg<128>::kSmem, st>>>(cache.maps, tp);
+        e = launch_pdl(mssa_tc_kernel<128>, dim3((unsigned)ncta), dim3(kThreads), Cfg<128>::kSmem, st,
+                       cache.maps, tp);
     } else {
         if (!cache.attr_set[0]) {
             cudaFuncAttributes fa;
@@ -809,10 +811,10 @@ msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st) {
             }
             cache.attr_set[0] = true;
         }
-        note_launch();
-        mssa_tc_kernel<64><<<(unsigned)ncta, kThreads, Cfg<64>::kSmem, st>>>(cache.maps, tp);
+        e = launch_pdl(mssa_tc_kernel<64>, dim3((unsigned)ncta), dim3(kThreads), Cfg<64>::kSmem, st,
+                       cache.maps, tp);
     }
-    e = cudaGetLastError();
+    if (e == cudaSuccess) e = cudaGetLastError();
     if (e != cudaSuccess) {
         set_cuda_error((int)e);
         return MSF_ERR_CUDA;

@@ -20,6 +20,7 @@
 #include <string.h>
 
 #include "gemm_tc.h"
+#include "kernels.h"
 #include "ptx.cuh"
 
 namespace msf {
@@ -87,6 +88,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     ptx::tc_fence_after();
     const uint32_t tbase = tmem_base_sh;
     volatile int* abort_p = &abort_flag;
+    ptx::grid_dep_wait();  // inputs written by the previous kernel are visible
+    ptx::grid_dep_launch();
 
     if (warp == 0 && lane == 0) {
         ptx::prefetch_tmap(&maps.a);
@@ -268,9 +271,8 @@ cudaError_t launch_bn(const GemmTcArgs& g, int batch, int splits, cudaStream_t s
     }
     dim3 grid((unsigned)((g.M + 127) / 128), (unsigned)((g.N + BN - 1) / BN),
               (unsigned)(batch * splits));
-    note_launch();
-    gemm_tc_kernel<BN, STAGES><<<grid, kThreads, GCfg<BN, STAGES>::kSmem, st>>>(maps, p);
-    return cudaGetLastError();
+    return launch_pdl(gemm_tc_kernel<BN, STAGES>, grid, dim3(kThreads), GCfg<BN, STAGES>::kSmem, st,
+                      maps, p);
 }
 
 }  // namespace

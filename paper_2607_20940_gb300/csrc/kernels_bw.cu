@@ -6,6 +6,7 @@
 #include <cuda_runtime.h>
 
 #include "kernels.h"
+#include "ptx.cuh"
 
 namespace msf {
 
@@ -56,6 +57,8 @@ struct Vec<float> {
 
 template <typename T>
 __global__ void __launch_bounds__(256) pool_kernel(const PoolBatch jobs) {
+    ptx::grid_dep_wait();
+    ptx::grid_dep_launch();
     const PoolJob& jb = jobs.j[blockIdx.y];
     const int b = blockIdx.z;
     const int idx = blockIdx.x * blockDim.x + threadIdx.x;
@@ -100,9 +103,9 @@ cudaError_t launch_pool(const PoolBatch& jobs, int batch, bool bf16, cudaStream_
     long long work = (long long)max_n * jobs.row_vecs;
     dim3 grid((unsigned)((work + 255) / 256), (unsigned)jobs.n, (unsigned)batch);
     if (bf16)
-        { note_launch(); pool_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(jobs); }
+        return launch_pdl(pool_kernel<__nv_bfloat16>, grid, dim3(256), 0, st, jobs);
     else
-        { note_launch(); pool_kernel<float><<<grid, 256, 0, st>>>(jobs); }
+        return launch_pdl(pool_kernel<float>, grid, dim3(256), 0, st, jobs);
     return cudaGetLastError();
 }
 
@@ -115,6 +118,8 @@ cudaError_t launch_pool(const PoolBatch& jobs, int batch, bool bf16, cudaStream_
 template <typename T>
 __global__ void __launch_bounds__(256) patchify_raw_kernel(const T* __restrict__ latent,
                                                            T* __restrict__ raw, MspShape sh) {
+    ptx::grid_dep_wait();
+    ptx::grid_dep_launch();
     const int l = blockIdx.y, b = blockIdx.z;
     const int per = sh.C * sh.Hl * sh.Wl;
     const int o = blockIdx.x * blockDim.x + threadIdx.x;
@@ -133,6 +138,8 @@ __global__ void __launch_bounds__(256) unpatchify_raw_kernel(const T* __restrict
                                                              T* __restrict__ latent, MspShape sh,
                                                              int position, long long raw_bstride,
                                                              int raw_offset) {
+    ptx::grid_dep_wait();
+    ptx::grid_dep_launch();
     const int b = blockIdx.z;
     const int per = sh.C * sh.Hl * sh.Wl;
     const int o = blockIdx.x * blockDim.x + threadIdx.x;
@@ -150,13 +157,11 @@ cudaError_t launch_patchify_raw(const void* latent, void* raw, const MspShape& s
                                 bool bf16, cudaStream_t st) {
     const int per = sh.C * sh.Hl * sh.Wl;
     dim3 grid((unsigned)((per + 255) / 256), (unsigned)sh.T, (unsigned)batch);
-    note_launch();
     if (bf16)
-        patchify_raw_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(
-            (const __nv_bfloat16*)latent, (__nv_bfloat16*)raw, sh);
-    else
-        patchify_raw_kernel<float><<<grid, 256, 0, st>>>((const float*)latent, (float*)raw, sh);
-    return cudaGetLastError();
+        return launch_pdl(patchify_raw_kernel<__nv_bfloat16>, grid, dim3(256), 0, st,
+                          (const __nv_bfloat16*)latent, (__nv_bfloat16*)raw, sh);
+    return launch_pdl(patchify_raw_kernel<float>, grid, dim3(256), 0, st, (const float*)latent,
+                      (float*)raw, sh);
 }
 
 cudaError_t launch_unpatchify_raw(const void* raw, void* latent, const MspShape& sh, int position,
@@ -164,15 +169,12 @@ cudaError_t launch_unpatchify_raw(const void* raw, void* latent, const MspShape&
                                   cudaStream_t st) {
     const int per = sh.C * sh.Hl * sh.Wl;
     dim3 grid((unsigned)((per + 255) / 256), 1, (unsigned)batch);
-    note_launch();
     if (bf16)
-        unpatchify_raw_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(
-            (const __nv_bfloat16*)raw, (__nv_bfloat16*)latent, sh, position, raw_bstride,
-            raw_offset);
-    else
-        unpatchify_raw_kernel<float><<<grid, 256, 0, st>>>((const float*)raw, (float*)latent, sh,
-                                                           position, raw_bstride, raw_offset);
-    return cudaGetLastError();
+        return launch_pdl(unpatchify_raw_kernel<__nv_bfloat16>, grid, dim3(256), 0, st,
+                          (const __nv_bfloat16*)raw, (__nv_bfloat16*)latent, sh, position, raw_bstride,
+                          raw_offset);
+    return launch_pdl(unpatchify_raw_kernel<float>, grid, dim3(256), 0, st, (const float*)raw,
+                      (float*)latent, sh, position, raw_bstride, raw_offset);
 }
 
 __global__ void __launch_bounds__(256) unpatchify_splitk_kernel(const float* __restrict__ part,
@@ -180,6 +182,8 @@ __global__ void __launch_bounds__(256) unpatchify_splitk_kernel(const float* __r
                                                                 __nv_bfloat16* __restrict__ latent,
                                                                 MspShape sh, int position,
                                                                 int batch) {
+    ptx::grid_dep_wait();
+    ptx::grid_dep_launch();
     const int b = blockIdx.z;
     const int per = sh.C * sh.Hl * sh.Wl;
     const int o = blockIdx.x * blockDim.x + threadIdx.x;
@@ -199,10 +203,8 @@ cudaError_t launch_unpatchify_splitk(const float* part, int splits, void* latent
                                      int position, int batch, cudaStream_t st) {
     const int per = sh.C * sh.Hl * sh.Wl;
     dim3 grid((unsigned)((per + 255) / 256), 1, (unsigned)batch);
-    note_launch();
-    unpatchify_splitk_kernel<<<grid, 256, 0, st>>>(part, splits, (__nv_bfloat16*)latent, sh, position,
-                                                   batch);
-    return cudaGetLastError();
+    return launch_pdl(unpatchify_splitk_kernel, grid, dim3(256), 0, st, part, splits,
+                      (__nv_bfloat16*)latent, sh, position, batch);
 }
 
 // --------------------------------------------------------- CUDA-core GEMM
@@ -226,6 +228,8 @@ __device__ __forceinline__ __nv_bfloat16 to_t(float x) { return __float2bfloat16
 
 template <typename T>
 __global__ void __launch_bounds__(256) gemm_nt_simt_kernel(GemmArgs g) {
+    ptx::grid_dep_wait();
+    ptx::grid_dep_launch();
     __shared__ float As[16][65];
     __shared__ float Bs[16][65];
     const int b = blockIdx.z;
@@ -270,9 +274,9 @@ __global__ void __launch_bounds__(256) gemm_nt_simt_kernel(GemmArgs g) {
 cudaError_t launch_gemm_nt_simt(const GemmArgs& g, int batch, bool bf16, cudaStream_t st) {
     dim3 grid((unsigned)((g.N + 63) / 64), (unsigned)((g.M + 63) / 64), (unsigned)batch);
     if (bf16)
-        { note_launch(); gemm_nt_simt_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(g); }
+        return launch_pdl(gemm_nt_simt_kernel<__nv_bfloat16>, grid, dim3(256), 0, st, g);
     else
-        { note_launch(); gemm_nt_simt_kernel<float><<<grid, 256, 0, st>>>(g); }
+        return launch_pdl(gemm_nt_simt_kernel<float>, grid, dim3(256), 0, st, g);
     return cudaGetLastError();
 }
 

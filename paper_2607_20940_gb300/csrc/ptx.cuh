@@ -25,6 +25,18 @@ __device__ __forceinline__ uint32_t elect_one_sync() {
     return pred;
 }
 
+// ----------------------------------------------------- programmatic launch
+// With programmatic stream serialisation the next kernel in the stream may
+// start before this one ends. Every kernel calls grid_dep_wait() before its
+// first access to global memory (which returns once the previous kernel has
+// completed and its writes are visible), so each kernel still sees all work
+// queued before it; grid_dep_launch() lets the next kernel start its launch
+// and prologue early.
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dep_launch() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ------------------------------------------------------------------ mbarrier
 
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
