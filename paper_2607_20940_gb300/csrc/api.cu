@@ -315,15 +315,17 @@ extern "C" msf_status msf_patchify(msf_plan_t plan, const void* latent, const vo
     const long long per = (long long)sh.C * sh.Hl * sh.Wl;
     const int E = p.d.embed_dim;
     if (bf16) {
-        // One tensor-core GEMM per run of consecutive states that share a tier
-        // (same scale, same weight): their raw blocks and output rows are
-        // contiguous.
+        // One tensor-core GEMM problem per run of consecutive states that
+        // share a tier (same scale, same weight): their raw blocks and output
+        // rows are contiguous. All runs go out in one grouped launch.
+        msf::GemmTcArgs runs[MSF_MAX_STATES];
+        int n_runs = 0;
         bool all_tc = true;
         for (int l0 = 0; l0 < p.T && all_tc;) {
             int l1 = l0 + 1;
             while (l1 < p.T && p.d.scales[l1] == p.d.scales[l0] && w_tier[l1] == w_tier[l0]) ++l1;
             const int P = p.d.patch * p.d.scales[l0];
-            msf::GemmTcArgs g;
+            msf::GemmTcArgs& g = runs[n_runs++];
             g.K = sh.C * P * P;
             g.A = raw + (size_t)l0 * per * p.elem;
             g.B = w_tier[l0];
@@ -340,26 +342,10 @@ extern "C" msf_status msf_patchify(msf_plan_t plan, const void* latent, const vo
             l0 = l1;
         }
         if (all_tc) {
-            for (int l0 = 0; l0 < p.T;) {
-                int l1 = l0 + 1;
-                while (l1 < p.T && p.d.scales[l1] == p.d.scales[l0] && w_tier[l1] == w_tier[l0]) ++l1;
-                const int P = p.d.patch * p.d.scales[l0];
-                msf::GemmTcArgs g;
-                g.K = sh.C * P * P;
-                g.A = raw + (size_t)l0 * per * p.elem;
-                g.B = w_tier[l0];
-                g.C = (char*)tokens + (size_t)p.st_off[l0] * E * p.elem;
-                g.M = p.st_off[l1 - 1] + p.st_n[l1 - 1] - p.st_off[l0];
-                g.N = E;
-                g.lda = g.K;
-                g.ldb = g.K;
-                g.ldc = E;
-                g.a_bstride = (long long)p.T * per;
-                g.c_bstride = (long long)p.N * E;
-                g.status = msf::status_word(p);
-                e = msf::launch_gemm_tc(g, p.B, s);
+            for (int r0 = 0; r0 < n_runs; r0 += msf::kMaxGemmProblems) {
+                const int n = n_runs - r0 < msf::kMaxGemmProblems ? n_runs - r0 : msf::kMaxGemmProblems;
+                e = msf::launch_gemm_tc_grouped(runs + r0, n, p.B, s);
                 if (e != cudaSuccess) return cuda_status(e);
-                l0 = l1;
             }
             return MSF_OK;
         }

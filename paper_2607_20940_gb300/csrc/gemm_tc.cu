@@ -40,18 +40,26 @@ struct GCfg {
     static constexpr int kTmemCols = BN < 32 ? 32 : BN;
 };
 
-struct GemmTcParams {
+// Up to kMaxProblems independent problems (e.g. the tiers of one window) share
+// one launch; blockIdx.x runs over all their 128 x BN tiles.
+struct GemmTcProblem {
     int M, N, K;
-    int batch, splits;    // grid.z = batch * splits
+    int m_tiles;
+    int tile_base;        // first tile of this problem in blockIdx.x
     __nv_bfloat16* C;     // splits == 1: bf16 output
     long long ldc;        // elements
     long long c_bstride;  // elements
+};
+struct GemmTcParams {
+    int n_prob;
+    GemmTcProblem pr[kMaxGemmProblems];
+    int batch, splits;    // grid.z = batch * splits (splits > 1: one problem)
     float* C32;           // splits > 1: fp32 partial sums [split][batch][M][N]
     unsigned int* status;
 };
 struct GemmTcMaps {
-    CUtensorMap a;  // {K, rows, B}
-    CUtensorMap b;  // {K, N}
+    CUtensorMap a[kMaxGemmProblems];  // {K, rows, B}
+    CUtensorMap b[kMaxGemmProblems];  // {K, N}
 };
 
 template <int BN, int STAGES>
@@ -64,9 +72,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     __shared__ uint32_t tmem_base_sh;
     __shared__ int abort_flag;
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-    const int m0 = blockIdx.x * 128, n0 = blockIdx.y * BN;
+    int pi = 0;
+    while (pi < p.n_prob - 1 && (int)blockIdx.x >= p.pr[pi + 1].tile_base) ++pi;
+    const GemmTcProblem& P = p.pr[pi];
+    const int local = (int)blockIdx.x - P.tile_base;
+    const int m0 = (local % P.m_tiles) * 128, n0 = (local / P.m_tiles) * BN;
     const int b = blockIdx.z % p.batch, split = blockIdx.z / p.batch;
-    const int nk_all = (p.K + 63) / 64;
+    const int nk_all = (P.K + 63) / 64;
     const int kc0 = (int)((long long)split * nk_all / p.splits);
     const int nk = (int)((long long)(split + 1) * nk_all / p.splits) - kc0;
 
@@ -92,8 +104,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     ptx::grid_dep_launch();
 
     if (warp == 0 && lane == 0) {
-        ptx::prefetch_tmap(&maps.a);
-        ptx::prefetch_tmap(&maps.b);
+        ptx::prefetch_tmap(&maps.a[pi]);
+        ptx::prefetch_tmap(&maps.b[pi]);
         int issued = 0;
         bool ok = true;
         for (int kc = 0; kc < nk; ++kc) {
@@ -105,8 +117,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             unsigned char* sa = smem + st * C::kStageBytes;
             ptx::mbar_arrive_expect_tx(&full[st], C::kStageBytes);
-            ptx::tma_load_3d(sa, &maps.a, &full[st], (kc0 + kc) * 64, m0, b);
-            ptx::tma_load_2d(sa + C::kABytes, &maps.b, &full[st], (kc0 + kc) * 64, n0);
+            ptx::tma_load_3d(sa, &maps.a[pi], &full[st], (kc0 + kc) * 64, m0, b);
+            ptx::tma_load_2d(sa + C::kABytes, &maps.b[pi], &full[st], (kc0 + kc) * 64, n0);
             ++issued;
         }
         if (!ok) {
@@ -151,10 +163,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (ok) {
             ptx::tc_fence_after();
             const int m = m0 + r;
-            const bool store = m < p.M;
+            const bool store = m < P.M;
             const uint32_t taddr = tbase + ((uint32_t)(wq * 32) << 16);
             if (p.splits == 1) {
-                __nv_bfloat16* crow = p.C + (size_t)b * p.c_bstride + (size_t)m * p.ldc + n0;
+                __nv_bfloat16* crow = P.C + (size_t)b * P.c_bstride + (size_t)m * P.ldc + n0;
 #pragma unroll 1
                 for (int c = 0; c < BN / 32; ++c) {
                     uint32_t v[32];
@@ -165,32 +177,32 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int e = 0; e < 16; ++e)
                         pk[e] = ptx::pack_bf16(__uint_as_float(v[2 * e]), __uint_as_float(v[2 * e + 1]));
                     const int ncol = n0 + c * 32;
-                    if (store && ncol + 32 <= p.N) {
+                    if (store && ncol + 32 <= P.N) {
                         uint4* d4 = reinterpret_cast<uint4*>(crow + c * 32);
 #pragma unroll
                         for (int e = 0; e < 4; ++e)
                             d4[e] = make_uint4(pk[4 * e], pk[4 * e + 1], pk[4 * e + 2], pk[4 * e + 3]);
                     } else if (store) {
                         const __nv_bfloat16* hb = reinterpret_cast<const __nv_bfloat16*>(pk);
-                        for (int e = 0; e < 32 && ncol + e < p.N; ++e) crow[c * 32 + e] = hb[e];
+                        for (int e = 0; e < 32 && ncol + e < P.N; ++e) crow[c * 32 + e] = hb[e];
                     }
                 }
             } else {
-                float* crow = p.C32 + (((size_t)split * p.batch + b) * p.M + m) * p.N + n0;
+                float* crow = p.C32 + (((size_t)split * p.batch + b) * P.M + m) * P.N + n0;
 #pragma unroll 1
                 for (int c = 0; c < BN / 32; ++c) {
                     uint32_t v[32];
                     ptx::tmem_ld32(taddr + c * 32, v);
                     ptx::tmem_wait_ld();
                     const int ncol = n0 + c * 32;
-                    if (store && ncol + 32 <= p.N) {
+                    if (store && ncol + 32 <= P.N) {
                         float4* d4 = reinterpret_cast<float4*>(crow + c * 32);
 #pragma unroll
                         for (int e = 0; e < 8; ++e)
                             d4[e] = make_float4(__uint_as_float(v[4 * e]), __uint_as_float(v[4 * e + 1]),
                                                 __uint_as_float(v[4 * e + 2]), __uint_as_float(v[4 * e + 3]));
                     } else if (store) {
-                        for (int e = 0; e < 32 && ncol + e < p.N; ++e) crow[c * 32 + e] = __uint_as_float(v[e]);
+                        for (int e = 0; e < 32 && ncol + e < P.N; ++e) crow[c * 32 + e] = __uint_as_float(v[e]);
                     }
                 }
             }
@@ -225,42 +237,47 @@ EncodeTiledFn encoder() {
 }
 
 template <int BN, int STAGES>
-cudaError_t launch_bn(const GemmTcArgs& g, int batch, int splits, cudaStream_t st) {
+cudaError_t launch_bn(const GemmTcArgs* gs, int n, int batch, int splits, cudaStream_t st) {
     EncodeTiledFn enc = encoder();
     if (!enc) return cudaErrorNotSupported;
     GemmTcMaps maps;
     memset(&maps, 0, sizeof(maps));
-    {
-        cuuint64_t dims[3] = {(cuuint64_t)g.K, (cuuint64_t)g.M, (cuuint64_t)batch};
-        cuuint64_t strides[2] = {(cuuint64_t)g.lda * 2, (cuuint64_t)g.a_bstride * 2};
-        cuuint32_t box[3] = {64, 128, 1};
-        cuuint32_t es[3] = {1, 1, 1};
-        if (enc(&maps.a, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(g.A), dims, strides,
-                box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-            return cudaErrorInvalidValue;
-    }
-    {
-        cuuint64_t dims[2] = {(cuuint64_t)g.K, (cuuint64_t)g.N};
-        cuuint64_t strides[1] = {(cuuint64_t)g.ldb * 2};
-        cuuint32_t box[2] = {64, (cuuint32_t)BN};
-        cuuint32_t es[2] = {1, 1};
-        if (enc(&maps.b, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(g.B), dims, strides,
-                box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-            return cudaErrorInvalidValue;
-    }
     GemmTcParams p;
-    p.M = g.M;
-    p.N = g.N;
-    p.K = g.K;
+    memset(&p, 0, sizeof(p));
+    int tiles = 0;
+    for (int i = 0; i < n; ++i) {
+        const GemmTcArgs& g = gs[i];
+        cuuint64_t adims[3] = {(cuuint64_t)g.K, (cuuint64_t)g.M, (cuuint64_t)batch};
+        cuuint64_t astrides[2] = {(cuuint64_t)g.lda * 2, (cuuint64_t)g.a_bstride * 2};
+        cuuint32_t abox[3] = {64, 128, 1};
+        cuuint32_t es[3] = {1, 1, 1};
+        if (enc(&maps.a[i], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(g.A), adims, astrides,
+                abox, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+        cuuint64_t bdims[2] = {(cuuint64_t)g.K, (cuuint64_t)g.N};
+        cuuint64_t bstrides[1] = {(cuuint64_t)g.ldb * 2};
+        cuuint32_t bbox[2] = {64, (cuuint32_t)BN};
+        if (enc(&maps.b[i], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(g.B), bdims, bstrides,
+                bbox, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+        GemmTcProblem& pr = p.pr[i];
+        pr.M = g.M;
+        pr.N = g.N;
+        pr.K = g.K;
+        pr.m_tiles = (g.M + 127) / 128;
+        pr.tile_base = tiles;
+        pr.C = (__nv_bfloat16*)g.C;
+        pr.ldc = g.ldc;
+        pr.c_bstride = g.c_bstride;
+        tiles += pr.m_tiles * ((g.N + BN - 1) / BN);
+    }
+    p.n_prob = n;
     p.batch = batch;
     p.splits = splits;
-    p.C = (__nv_bfloat16*)g.C;
-    p.ldc = g.ldc;
-    p.c_bstride = g.c_bstride;
-    p.C32 = g.C32;
-    p.status = g.status;
+    p.C32 = gs[0].C32;
+    p.status = gs[0].status;
     static bool attr = false;
     if (!attr) {
         cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES>,
@@ -269,8 +286,7 @@ cudaError_t launch_bn(const GemmTcArgs& g, int batch, int splits, cudaStream_t s
         if (e != cudaSuccess) return e;
         attr = true;
     }
-    dim3 grid((unsigned)((g.M + 127) / 128), (unsigned)((g.N + BN - 1) / BN),
-              (unsigned)(batch * splits));
+    dim3 grid((unsigned)tiles, 1, (unsigned)(batch * splits));
     return launch_pdl(gemm_tc_kernel<BN, STAGES>, grid, dim3(kThreads), GCfg<BN, STAGES>::kSmem, st,
                       maps, p);
 }
@@ -297,13 +313,24 @@ cudaError_t launch_gemm_tc(const GemmTcArgs& g, int batch, cudaStream_t st) {
             splits *= 2;
         g.splits_used = splits;
         if (splits > 1) {
-            if (g.N <= 64) return launch_bn<64, 4>(g, batch, splits, st);
-            return launch_bn<128, 4>(g, batch, splits, st);
+            if (g.N <= 64) return launch_bn<64, 4>(&g, 1, batch, splits, st);
+            return launch_bn<128, 4>(&g, 1, batch, splits, st);
         }
     }
     g.splits_used = 1;
-    if (g.N <= 64) return launch_bn<64, 4>(g, batch, 1, st);
-    return launch_bn<128, 2>(g, batch, 1, st);
+    if (g.N <= 64) return launch_bn<64, 4>(&g, 1, batch, 1, st);
+    return launch_bn<128, 2>(&g, 1, batch, 1, st);
+}
+
+cudaError_t launch_gemm_tc_grouped(const GemmTcArgs* gs, int n, int batch, cudaStream_t st) {
+    if (n < 1 || n > kMaxGemmProblems) return cudaErrorInvalidValue;
+    bool narrow = true;
+    for (int i = 0; i < n; ++i) {
+        gs[i].splits_used = 1;
+        narrow = narrow && gs[i].N <= 64;
+    }
+    if (narrow) return launch_bn<64, 4>(gs, n, batch, 1, st);
+    return launch_bn<128, 2>(gs, n, batch, 1, st);
 }
 
 }  // namespace msf

@@ -24,7 +24,11 @@ struct GemmTcArgs {
     mutable int splits_used = 1;
 };
 
+constexpr int kMaxGemmProblems = 4;
+
 bool gemm_tc_supported(const GemmTcArgs& g);
 cudaError_t launch_gemm_tc(const GemmTcArgs& g, int batch, cudaStream_t st);
+// Several independent problems (no K split) in one launch.
+cudaError_t launch_gemm_tc_grouped(const GemmTcArgs* gs, int n, int batch, cudaStream_t st);
 
 }  // namespace msf
