@@ -287,86 +287,111 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         } else if (warp == 1) {
         // ============================ MMA issuer ============================
-        if (lane == 0) {
+        // The whole warp runs the loop, so its control flow, barrier waits and
+        // descriptors stay warp-uniform; one elected lane (the same lane every
+        // time in a converged warp, so every commit covers every MMA before
+        // it) issues the MMAs and commits. The tensor pipe queues only a few
+        // MMAs, so the loop waits at two points per K/V step and issues 16
+        // MMAs after each.
+        {
             constexpr uint32_t idS = ptx::idesc_bf16(kBlockM, kBlockN, false, false);
             constexpr uint32_t idO = ptx::idesc_bf16(kBlockM, D, false, true);
-            const uint32_t q_addr = ptx::smem_u32(sQ);
-            const uint32_t k_addr = ptx::smem_u32(sK);
-            const uint32_t v_addr = ptx::smem_u32(sV);
+            // Descriptors are built once; a K step or another stage only adds a
+            // constant to the 14-bit start-address field (shared memory offsets
+            // stay below 256 KB, so the field never carries).
+            constexpr uint64_t kTileDesc = (uint64_t)(C::kTileBytes >> 4);
+            const uint64_t q_desc = ptx::sdesc_sw128(ptx::smem_u32(sQ), 16, 1024);
+            const uint64_t k_desc = ptx::sdesc_sw128(ptx::smem_u32(sK), 16, 1024);
+            const uint64_t v_desc = ptx::sdesc_sw128(ptx::smem_u32(sV), kBlockN * 128, 1024);
             auto issue_s = [&](int t, int st) {
-                const uint32_t qa = q_addr + t * C::kTileBytes;
-                const uint32_t ka = k_addr + st * C::kTileBytes;
+                const uint64_t qd = q_desc + (uint64_t)t * kTileDesc;
+                const uint64_t kd = k_desc + (uint64_t)st * kTileDesc;
+                const uint32_t d = tbase + t * 128;
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk) {
-                    const uint32_t off = (kk / 4) * (kBlockM * 128) + (kk % 4) * 32;
-                    ptx::mma_ss(tbase + t * 128, ptx::sdesc_sw128(qa + off, 16, 1024),
-                                ptx::sdesc_sw128(ka + off, 16, 1024), idS, kk > 0 ? 1u : 0u);
+                    constexpr int kChunk = kBlockM * 128;
+                    const uint64_t off = (uint64_t)(((kk / 4) * kChunk + (kk % 4) * 32) >> 4);
+                    ptx::mma_ss(d, qd + off, kd + off, idS, kk > 0 ? 1u : 0u);
                 }
                 ptx::mma_commit(&s_full[t]);
             };
             auto issue_pv = [&](int t, int st, bool acc) {
-                const uint32_t va = v_addr + st * C::kTileBytes;
+                const uint64_t vd = v_desc + (uint64_t)st * kTileDesc;
+                const uint32_t d = tbase + 256 + t * 128, a = tbase + t * 128;
 #pragma unroll
-                for (int kk = 0; kk < kBlockN / 16; ++kk) {
-                    ptx::mma_ts(tbase + 256 + t * 128, tbase + t * 128 + kk * 8,
-                                ptx::sdesc_sw128(va + kk * 2048, kBlockN * 128, 1024), idO,
+                for (int kk = 0; kk < kBlockN / 16; ++kk)
+                    ptx::mma_ts(d, a + kk * 8, vd + (uint64_t)(kk * (2048 >> 4)), idO,
                                 (acc || kk > 0) ? 1u : 0u);
-                }
+            };
+            // Warp-wide bounded wait: every lane waits, the warp agrees.
+            auto wait_all = [&](uint64_t* bar, uint32_t parity) {
+                const bool r = ptx::mbar_wait_bounded(bar, parity, abort_p, p.wait_limit);
+                return __all_sync(0xffffffffu, r);
             };
             bool ok = true;
-            long long js = 0;
+            // Ring positions of the next K/V tile: K slot and phase (2-deep),
+            // V slot and phase (3-deep), P/S phase (one per tile).
+            int ks = 0, vs = 0;
+            uint32_t kph = 0, vph = 0, pph = 0;
             int piece = 0;
             for (long long t = r0; t < r1 && ok; ++piece) {
                 const Piece pc = locate(p, t, r1);
                 const int n = pc.u1 - pc.u0;
-                const int st0 = (int)(js % kStages);
-                ok = ptx::mbar_wait_bounded(&q_full, (uint32_t)(piece & 1), abort_p, p.wait_limit) &&
-                     ptx::mbar_wait_bounded(&k_full[st0], (uint32_t)((js / kStages) & 1), abort_p,
-                                            p.wait_limit);
+                ok = wait_all(&q_full, (uint32_t)(piece & 1)) && wait_all(&k_full[ks], kph);
                 if (!ok) break;
                 ptx::tc_fence_after();
-                issue_s(0, st0);
-                issue_s(1, st0);
-                ptx::mma_commit(&k_empty[st0]);
-                if (n == 1) ptx::mma_commit(&q_empty);
+                if (ptx::elect_one_sync()) {
+                    issue_s(0, ks);
+                    issue_s(1, ks);
+                    ptx::mma_commit(&k_empty[ks]);
+                    if (n == 1) ptx::mma_commit(&q_empty);
+                }
+                __syncwarp();
                 for (int jl = 0; jl < n; ++jl) {
-                    const long long j = js + jl;
-                    const int sv = (int)(j % kVStages);
-                    const uint32_t phv = (uint32_t)((j / kVStages) & 1);
-                    const int st1 = (int)((j + 1) % kStages);
-                    const uint32_t ph1 = (uint32_t)(((j + 1) / kStages) & 1);
                     const bool more = jl + 1 < n;
-                    ok = ptx::mbar_wait_bounded(&v_full[sv], phv, abort_p, p.wait_limit) &&
-                         ptx::mbar_wait_bounded(&p_full[0], (uint32_t)(j & 1), abort_p, p.wait_limit);
+                    const int ks1 = ks ^ 1;
+                    const uint32_t kph1 = ks1 == 0 ? kph ^ 1u : kph;
+                    // V of this tile, K of the next one and P0 of this tile.
+                    ok = wait_all(&v_full[vs], vph) && (!more || wait_all(&k_full[ks1], kph1)) &&
+                         wait_all(&p_full[0], pph);
                     if (!ok) break;
                     ptx::tc_fence_after();
-                    issue_pv(0, sv, jl > 0);
-                    if (more) {
-                        ok = ptx::mbar_wait_bounded(&k_full[st1], ph1, abort_p, p.wait_limit);
-                        if (!ok) break;
-                        ptx::tc_fence_after();
-                        issue_s(0, st1);
+                    if (ptx::elect_one_sync()) {
+                        issue_pv(0, vs, jl > 0);
+                        if (more) issue_s(0, ks1);
                     }
-                    ok = ptx::mbar_wait_bounded(&p_full[1], (uint32_t)(j & 1), abort_p, p.wait_limit);
+                    __syncwarp();
+                    ok = wait_all(&p_full[1], pph);
                     if (!ok) break;
                     ptx::tc_fence_after();
-                    issue_pv(1, sv, jl > 0);
-                    if (more) {
-                        issue_s(1, st1);
-                        ptx::mma_commit(&k_empty[st1]);
-                        if (jl + 2 == n) ptx::mma_commit(&q_empty);  // last use of Q issued
+                    if (ptx::elect_one_sync()) {
+                        issue_pv(1, vs, jl > 0);
+                        if (more) {
+                            issue_s(1, ks1);
+                            ptx::mma_commit(&k_empty[ks1]);
+                            if (jl + 2 == n) ptx::mma_commit(&q_empty);  // last use of Q issued
+                        }
+                    }
+                    __syncwarp();
+                    ks = ks1;
+                    kph = kph1;
+                    pph ^= 1u;
+                    if (++vs == kVStages) {
+                        vs = 0;
+                        vph ^= 1u;
                     }
                 }
                 if (!ok) break;
-                ptx::mma_commit(&o_full);
-                js += n;
+                if (ptx::elect_one_sync()) ptx::mma_commit(&o_full);
+                __syncwarp();
                 t += n;
             }
             if (!ok) {
                 // drain_bar covers every MMA issued: TMEM is never released under one.
-                ptx::mma_commit(&drain_bar);
+                if (ptx::elect_one_sync()) ptx::mma_commit(&drain_bar);
+                __syncwarp();
                 ptx::mbar_wait_bounded(&drain_bar, 0, &never, kWaitLimit);
-                atomicOr(p.status, kDevTimeout);
+                if (lane == 0) atomicOr(p.status, kDevTimeout);
             }
         }
         }
