@@ -351,9 +351,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const bool more = jl + 1 < n;
                     const int ks1 = ks ^ 1;
                     const uint32_t kph1 = ks1 == 0 ? kph ^ 1u : kph;
-                    // V of this tile, K of the next one and P0 of this tile.
-                    ok = wait_all(&v_full[vs], vph) && (!more || wait_all(&k_full[ks1], kph1)) &&
-                         wait_all(&p_full[0], pph);
+                    // V of this tile, K of the next one and P0 of this tile: the
+                    // three probes go out together; the bounded waits run only
+                    // if one of them is not ready yet.
+                    {
+                        const bool rv = ptx::mbar_try_wait(&v_full[vs], vph);
+                        const bool rk = !more || ptx::mbar_try_wait(&k_full[ks1], kph1);
+                        const bool rp = ptx::mbar_try_wait(&p_full[0], pph);
+                        if (!__all_sync(0xffffffffu, rv && rk && rp))
+                            ok = wait_all(&v_full[vs], vph) && (!more || wait_all(&k_full[ks1], kph1)) &&
+                                 wait_all(&p_full[0], pph);
+                    }
                     if (!ok) break;
                     ptx::tc_fence_after();
                     if (ptx::elect_one_sync()) {
