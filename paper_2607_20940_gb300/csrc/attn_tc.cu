@@ -437,20 +437,55 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int c = 0; c < 128; ++c)
                         if (c >= valid) s[c >> 5][c & 31] = 0xff800000u;
                 }
-                float mx[8];
+                // Exponentials use the running maximum m_used, which may lag
+                // the row's true maximum: P = 2^(s - m_used) then exceeds 1,
+                // which changes nothing but a power-of-two scale common to
+                // P, O and l. The tile's sum shows how far it lags; only when
+                // it passes 2^32 (or is not finite) is the exact maximum found
+                // and O rescaled, so most tiles skip the max pass entirely.
+                // The first tile of a piece starts from its exact maximum.
+                auto tile_max = [&]() -> float {
+                    float mx[8];
 #pragma unroll
-                for (int e = 0; e < 8; ++e) mx[e] = -INFINITY;
+                    for (int e = 0; e < 8; ++e) mx[e] = -INFINITY;
 #pragma unroll
-                for (int c = 0; c < 128; c += 2)
-                    mx[(c >> 1) & 7] = ptx::fmax3(mx[(c >> 1) & 7], __uint_as_float(s[c >> 5][c & 31]),
-                                                  __uint_as_float(s[c >> 5][(c & 31) + 1]));
-                const float m_tile = fmaxf(ptx::fmax3(mx[0], mx[1], mx[2]),
-                                           fmaxf(ptx::fmax3(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7])));
-                const float m_new = fmaxf(m_used, m_tile * sl2);
-                if (u == pc.u0) {
-                    m_used = m_new;
-                } else if (__any_sync(0xffffffffu, m_new > m_used + 8.0f)) {
+                    for (int c = 0; c < 128; c += 2)
+                        mx[(c >> 1) & 7] = ptx::fmax3(mx[(c >> 1) & 7], __uint_as_float(s[c >> 5][c & 31]),
+                                                      __uint_as_float(s[c >> 5][(c & 31) + 1]));
+                    return fmaxf(ptx::fmax3(mx[0], mx[1], mx[2]),
+                                 fmaxf(ptx::fmax3(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7]))) * sl2;
+                };
+                if (u == pc.u0) m_used = tile_max();
+                uint64_t sum2[2];
+#pragma unroll 1
+                for (int pass = 0; pass < 2; ++pass) {
+                    const float nm = -m_used;
+                    const uint64_t sl2x2 = ptx::f2_pack(sl2, sl2), nmx2 = ptx::f2_pack(nm, nm);
+                    sum2[0] = sum2[1] = ptx::f2_pack(0.f, 0.f);
+#pragma unroll
+                    for (int q4 = 0; q4 < 4; ++q4) {
+                        uint32_t pk[16];
+#pragma unroll
+                        for (int c = 0; c < 16; ++c) {
+                            const uint64_t arg = ptx::f2_fma(
+                                ptx::f2_pack(__uint_as_float(s[q4][2 * c]), __uint_as_float(s[q4][2 * c + 1])),
+                                sl2x2, nmx2);
+                            float a0, a1;
+                            ptx::f2_unpack(arg, a0, a1);
+                            const float p0 = ex2(a0), p1 = ex2(a1);
+                            sum2[c & 1] = ptx::f2_add(sum2[c & 1], ptx::f2_pack(p0, p1));
+                            pk[c] = ptx::pack_bf16(p0, p1);
+                        }
+                        ptx::tmem_st16(tS + 16 * q4, pk);
+                    }
+                    if (pass == 1) break;
+                    float a0, a1, b0, b1;
+                    ptx::f2_unpack(sum2[0], a0, a1);
+                    ptx::f2_unpack(sum2[1], b0, b1);
+                    const float tile_sum = (a0 + a1) + (b0 + b1);
+                    if (!__any_sync(0xffffffffu, !(tile_sum <= 4294967296.0f))) break;
                     // O_t holds every PV up to the previous step (the S_t commit covers it).
+                    const float m_new = fmaxf(m_used, tile_max());
                     const float f = ex2(m_used - m_new);
                     l *= f;
                     m_used = m_new;
@@ -463,26 +498,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         for (int e = 0; e < 16; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * f);
                         ptx::tmem_st16(tO + c * 16, o);
                     }
-                    ptx::tmem_wait_st();
-                }
-                const float nm = -m_used;
-                const uint64_t sl2x2 = ptx::f2_pack(sl2, sl2), nmx2 = ptx::f2_pack(nm, nm);
-                uint64_t sum2[2] = {ptx::f2_pack(0.f, 0.f), ptx::f2_pack(0.f, 0.f)};
-#pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) {
-                    uint32_t pk[16];
-#pragma unroll
-                    for (int c = 0; c < 16; ++c) {
-                        const uint64_t arg = ptx::f2_fma(
-                            ptx::f2_pack(__uint_as_float(s[q4][2 * c]), __uint_as_float(s[q4][2 * c + 1])),
-                            sl2x2, nmx2);
-                        float a0, a1;
-                        ptx::f2_unpack(arg, a0, a1);
-                        const float p0 = ex2(a0), p1 = ex2(a1);
-                        sum2[c & 1] = ptx::f2_add(sum2[c & 1], ptx::f2_pack(p0, p1));
-                        pk[c] = ptx::pack_bf16(p0, p1);
-                    }
-                    ptx::tmem_st16(tS + 16 * q4, pk);
+                    ptx::tmem_wait_st();  // P of the first pass is overwritten after this
                 }
                 {
                     float a0, a1, b0, b1;
