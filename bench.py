@@ -6,6 +6,8 @@ tokens, history ring of 2 frames):
   MSP patchify + tier embedding of the 5 latent states (16x60x104 -> 4290x1536)
   -> window part of the K/V pyramid -> MSSA attention (Eq. 4)
   -> de-embed + unpatchify of the head state -> history append (head K/V).
+The embedding runs on a second stream beside the pyramid, and the
+de-embedding beside the history append; attention waits for both inputs.
 `value` is the MSSA FLOPs the schedule requires (4*D*H*sum_g Nq_g*Nkv_g =
 202.79 GFLOP) divided by the device time of the whole step, in TFLOP/s.
 Inputs are resident in HBM; the L2 is flushed (a 256 MiB write) between
@@ -244,20 +246,36 @@ def main():
     flops = info.attention_flops
 
     ev_a = []  # attention start/end events of timed steps
+    side = torch.cuda.Stream(device=dev)
 
     def step(q, k, v, latent, timed_attn=False):
-        plan.patchify(latent, w_tier, tok)
-        plan.kv_resample(k, v, msf.MSF_RESAMPLE_WINDOW_ONLY)
+        # Two streams: the MSP embedding of the window runs beside the K/V
+        # pyramid, and the de-embedding of the head state beside the history
+        # update. Attention waits for both of its inputs.
+        fork = torch.cuda.Event()
+        fork.record(stream)
+        side.wait_event(fork)
+        plan.patchify(latent, w_tier, tok, stream=side)
+        embedded = torch.cuda.Event()
+        embedded.record(side)
+        plan.kv_resample(k, v, msf.MSF_RESAMPLE_WINDOW_ONLY, stream=stream)
+        stream.wait_event(embedded)
         if timed_attn:
             a0 = torch.cuda.Event(enable_timing=True)
             a1 = torch.cuda.Event(enable_timing=True)
             a0.record(stream)
-        plan.mssa_forward(q, k, v, out)
+        plan.mssa_forward(q, k, v, out, stream=stream)
         if timed_attn:
             a1.record(stream)
             ev_a.append((a0, a1))
-        plan.unpatchify(0, out.view(w.batch, N, E), w_out, lat_out)
-        plan.history_append(k, v)
+        attended = torch.cuda.Event()
+        attended.record(stream)
+        side.wait_event(attended)
+        plan.unpatchify(0, out.view(w.batch, N, E), w_out, lat_out, stream=side)
+        plan.history_append(k, v, stream=stream)
+        joined = torch.cuda.Event()
+        joined.record(side)
+        stream.wait_event(joined)
 
     plan.kv_resample(d["k_win"], d["v_win"], msf.MSF_RESAMPLE_FULL)
     for _ in range(args.warmup):

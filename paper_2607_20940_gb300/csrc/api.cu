@@ -5,6 +5,7 @@
 
 #include "attn_tc.h"
 #include "gemm_tc.h"
+#include "msp_tc.h"
 #include "internal.h"
 #include "kernels.h"
 
@@ -309,11 +310,45 @@ extern "C" msf_status msf_patchify(msf_plan_t plan, const void* latent, const vo
     if (!p.bound) return MSF_ERR_STATE;  // the raw tokens go through the workspace
     for (int l = 0; l < p.T; ++l)
         if (!w_tier[l] || !aligned16(w_tier[l])) return MSF_ERR_INVALID_ARG;
+    const long long per = (long long)sh.C * sh.Hl * sh.Wl;
+    const int E = p.d.embed_dim;
+    if (bf16) {
+        // Fused gather + embedding: one problem per run of consecutive states
+        // that share a tier (same scale, same weight), all runs in one launch.
+        msf::MspEmbedRun runs[MSF_MAX_STATES];
+        int n_runs = 0;
+        for (int l0 = 0; l0 < p.T;) {
+            int l1 = l0 + 1;
+            while (l1 < p.T && p.d.scales[l1] == p.d.scales[l0] && w_tier[l1] == w_tier[l0]) ++l1;
+            msf::MspEmbedRun& r = runs[n_runs++];
+            r.w = w_tier[l0];
+            r.P = p.d.patch * p.d.scales[l0];
+            r.K = sh.C * r.P * r.P;
+            r.l0 = l0;
+            r.n_l = p.st_n[l0];
+            r.M = p.st_off[l1 - 1] + p.st_n[l1 - 1] - p.st_off[l0];
+            r.gw = sh.Wl / r.P;
+            r.tok_off = p.st_off[l0];
+            l0 = l1;
+        }
+        bool fused = true;
+        for (int r0 = 0; r0 < n_runs && fused; r0 += msf::kMaxGemmProblems) {
+            const int n = n_runs - r0 < msf::kMaxGemmProblems ? n_runs - r0 : msf::kMaxGemmProblems;
+            fused = msf::msp_embed_supported(runs + r0, n, E);
+        }
+        if (fused) {
+            for (int r0 = 0; r0 < n_runs; r0 += msf::kMaxGemmProblems) {
+                const int n = n_runs - r0 < msf::kMaxGemmProblems ? n_runs - r0 : msf::kMaxGemmProblems;
+                cudaError_t e = msf::launch_msp_embed(runs + r0, n, sh, E, latent, tokens, (long long)p.N * E,
+                                                      p.B, msf::status_word(p), s);
+                if (e != cudaSuccess) return cuda_status(e);
+            }
+            return MSF_OK;
+        }
+    }
     char* raw = msf::msp_scratch(p);
     cudaError_t e = msf::launch_patchify_raw(latent, raw, sh, p.B, bf16, s);
     if (e != cudaSuccess) return cuda_status(e);
-    const long long per = (long long)sh.C * sh.Hl * sh.Wl;
-    const int E = p.d.embed_dim;
     if (bf16) {
         // One tensor-core GEMM problem per run of consecutive states that
         // share a tier (same scale, same weight): their raw blocks and output

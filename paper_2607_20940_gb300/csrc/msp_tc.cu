@@ -1,0 +1,369 @@
+// Fused Multi-Scale Patchification kernel on the sm_103a tensor cores
+// (Sec. 3.2: a latent state of scale s_l is cut into patches of edge
+// P = patch * s_l; Eq. 3 token counts; feature order (c, dy, dx)).
+//
+// msp_embed_kernel    patchify + tier embedding in one pass. The A operand
+//                     (raw patch vectors, K = C*P^2) is gathered from the
+//                     latent straight into 128-byte-swizzled shared memory by
+//                     four warps, B (the tier's [E, K] weight) arrives by TMA,
+//                     and the accumulator is written once as bf16 tokens.
+//
+// Roles (256 threads): warp 0 TMA producer, warp 1 MMA issuer (one elected
+// lane of the converged warp), warp 2 TMEM allocation, warps 4-7 gather and
+// epilogue. Every wait is bounded and winds down through the status word.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <string.h>
+
+#include "gemm_tc.h"
+#include "kernels.h"
+#include "msp_tc.h"
+#include "ptx.cuh"
+
+namespace msf {
+
+namespace {
+
+constexpr int kThreads = 256;
+constexpr long long kWaitLimit = 2000000000LL;
+constexpr int kChunkA = 128 * 128;  // 128 rows x 64 bf16 (one K chunk), swizzled
+constexpr int kEmbedBN = 128;
+constexpr int kEmbedStages = 2;
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encoder() {
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        void* ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = (EncodeTiledFn)ptr;
+    }
+    return fn;
+}
+
+bool encode_2d(CUtensorMap* m, const void* base, int inner, int outer, long long stride_bytes,
+               int box_inner, int box_outer) {
+    EncodeTiledFn enc = encoder();
+    if (!enc) return false;
+    cuuint64_t dims[2] = {(cuuint64_t)inner, (cuuint64_t)outer};
+    cuuint64_t strides[1] = {(cuuint64_t)stride_bytes};
+    cuuint32_t box[2] = {(cuuint32_t)box_inner, (cuuint32_t)box_outer};
+    cuuint32_t es[2] = {1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Byte offset of bf16 element (row, k) inside one 128-row x 64-column K chunk
+// in the 128-byte swizzle layout the tensor core and TMA use: rows are 128
+// bytes, eight rows form a 1024-byte atom, and the 16-byte unit index is
+// XOR-ed with the row's position in its atom.
+__device__ __forceinline__ uint32_t swz_offset(int row, int k) {
+    const int byte = k * 2;
+    return (uint32_t)((row >> 3) * 1024 + (row & 7) * 128 + (((byte >> 4) ^ (row & 7)) << 4) + (byte & 15));
+}
+
+// ----------------------------------------------------------------- embedding
+
+// Features [64 kc, 64 kc + 64) of one token row in (c, dy, dx) order: 64 / P
+// runs of P pixels, each run one row segment of one channel. All loads of the
+// chunk are issued before the first store so that they overlap.
+template <int P, typename V>
+__device__ __forceinline__ void gather_chunk(unsigned char* dst, const __nv_bfloat16* base, size_t plane,
+                                             int Wl, int r, int kc, bool valid) {
+    constexpr int kRuns = 64 / P;
+    V v[kRuns];
+#pragma unroll
+    for (int g = 0; g < kRuns; ++g) {
+        const int f0 = kc * 64 + g * P;
+        const int c = f0 / (P * P), dy = (f0 % (P * P)) / P;
+        if (valid)
+            v[g] = __ldg(reinterpret_cast<const V*>(base + c * plane + (size_t)dy * Wl));
+        else
+            memset(&v[g], 0, sizeof(V));
+    }
+#pragma unroll
+    for (int g = 0; g < kRuns; ++g) *reinterpret_cast<V*>(dst + swz_offset(r, g * P)) = v[g];
+}
+
+struct EmbedRun {
+    int tile_base;  // first CTA of this run in blockIdx.x
+    int m_tiles;
+    int M;          // tokens of the run (per stream)
+    int l0;         // first state of the run
+    int n_l;        // tokens per state
+    int gw;         // tokens per grid row (Wl / P)
+    int P;          // patch edge in latent pixels
+    int K;          // C * P * P
+    int tok_off;    // first token row of the run in the output
+};
+struct EmbedParams {
+    int n_runs;
+    EmbedRun run[kMaxGemmProblems];
+    int T, C, Hl, Wl, E;
+    const __nv_bfloat16* latent;  // [B, T, C, Hl, Wl]
+    __nv_bfloat16* tokens;        // [B, N, E]
+    long long tok_bstride;        // elements
+    unsigned int* status;
+};
+struct EmbedMaps {
+    CUtensorMap w[kMaxGemmProblems];    // [E, K] weight of each run: dims {K, E}
+    CUtensorMap out[kMaxGemmProblems];  // the run's tokens: dims {E, M, B}, rows past M clipped
+};
+
+__global__ void __launch_bounds__(kThreads, 1)
+    msp_embed_kernel(const __grid_constant__ EmbedMaps maps, const __grid_constant__ EmbedParams p) {
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    unsigned char* sA = smem;                                   // [stage][chunk]
+    unsigned char* sB = smem + kEmbedStages * kChunkA;          // [stage][BN rows x 128 B]
+    constexpr int kBBytes = kEmbedBN * 128;
+    __shared__ uint64_t a_full[kEmbedStages], a_empty[kEmbedStages];
+    __shared__ uint64_t b_full[kEmbedStages], b_empty[kEmbedStages], acc_full;
+    __shared__ uint32_t tmem_base_sh;
+    __shared__ int abort_flag;
+
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    int ri = 0;
+    while (ri < p.n_runs - 1 && (int)blockIdx.x >= p.run[ri + 1].tile_base) ++ri;
+    const EmbedRun& R = p.run[ri];
+    const int local = (int)blockIdx.x - R.tile_base;
+    const int mt = local % R.m_tiles, nt = local / R.m_tiles;
+    const int b = blockIdx.z;
+    const int nk = R.K / 64;
+
+    if (threadIdx.x == 0) {
+        abort_flag = 0;
+        for (int s = 0; s < kEmbedStages; ++s) {
+            ptx::mbar_init(&a_full[s], 128);  // one arrival per gathering thread
+            ptx::mbar_init(&a_empty[s], 1);
+            ptx::mbar_init(&b_full[s], 1);
+            ptx::mbar_init(&b_empty[s], 1);
+        }
+        ptx::mbar_init(&acc_full, 1);
+        ptx::fence_mbar_init();
+    }
+    if (warp == 2) {
+        ptx::tmem_alloc(&tmem_base_sh, kEmbedBN);
+        ptx::tmem_relinquish();
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tbase = tmem_base_sh;
+    volatile int* abort_p = &abort_flag;
+    volatile int never = 0;
+    ptx::grid_dep_wait();  // the latent and weights written before are visible
+    ptx::grid_dep_launch();
+
+    if (warp == 0) {
+        if (lane == 0) {
+            ptx::prefetch_tmap(&maps.w[ri]);
+            int issued = 0;
+            bool ok = true;
+            for (int kc = 0; kc < nk; ++kc) {
+                const int st = kc % kEmbedStages;
+                const uint32_t ph = (uint32_t)((kc / kEmbedStages) & 1);
+                if (!ptx::mbar_wait_bounded(&b_empty[st], ph ^ 1u, abort_p, kWaitLimit)) {
+                    ok = false;
+                    break;
+                }
+                ptx::mbar_arrive_expect_tx(&b_full[st], kBBytes);
+                ptx::tma_load_2d(sB + st * kBBytes, &maps.w[ri], &b_full[st], kc * 64, nt * kEmbedBN);
+                ++issued;
+            }
+            if (!ok) {
+                for (int kc = (issued > kEmbedStages ? issued - kEmbedStages : 0); kc < issued; ++kc)
+                    ptx::mbar_wait_bounded(&b_full[kc % kEmbedStages],
+                                           (uint32_t)((kc / kEmbedStages) & 1), &never, kWaitLimit);
+                atomicOr(p.status, kDevTimeout);
+            }
+        }
+    } else if (warp == 1) {
+        constexpr uint32_t idesc = ptx::idesc_bf16(128, kEmbedBN, false, false);
+        const uint64_t a_desc = ptx::sdesc_sw128(ptx::smem_u32(sA), 16, 1024);
+        const uint64_t b_desc = ptx::sdesc_sw128(ptx::smem_u32(sB), 16, 1024);
+        bool ok = true;
+        for (int kc = 0; kc < nk && ok; ++kc) {
+            const int st = kc % kEmbedStages;
+            const uint32_t ph = (uint32_t)((kc / kEmbedStages) & 1);
+            const bool ra = ptx::mbar_wait_bounded(&a_full[st], ph, abort_p, kWaitLimit);
+            const bool rb = ra && ptx::mbar_wait_bounded(&b_full[st], ph, abort_p, kWaitLimit);
+            ok = __all_sync(0xffffffffu, rb);
+            if (!ok) break;
+            ptx::tc_fence_after();
+            if (ptx::elect_one_sync()) {
+                const uint64_t ad = a_desc + (uint64_t)(st * (kChunkA >> 4));
+                const uint64_t bd = b_desc + (uint64_t)(st * (kBBytes >> 4));
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk)
+                    ptx::mma_ss(tbase, ad + (uint64_t)(kk * 2), bd + (uint64_t)(kk * 2), idesc,
+                                (kc > 0 || kk > 0) ? 1u : 0u);
+                ptx::mma_commit(&a_empty[st]);
+                ptx::mma_commit(&b_empty[st]);
+            }
+            __syncwarp();
+        }
+        if (ptx::elect_one_sync()) ptx::mma_commit(&acc_full);  // also after an abort: drains the MMAs
+        __syncwarp();
+        if (!ok && lane == 0) atomicOr(p.status, kDevTimeout);
+    } else if (warp >= 4) {
+        // ---- gather: one token row per thread
+        const int r = (warp - 4) * 32 + lane;
+        const int m = mt * 128 + r;
+        const bool valid = m < R.M;
+        const int P = R.P;
+        const __nv_bfloat16* base = p.latent;
+        if (valid) {
+            const int l = R.l0 + m / R.n_l;
+            const int loc = m % R.n_l;
+            const int i = loc / R.gw, jj = loc % R.gw;
+            base = p.latent + ((size_t)b * p.T + l) * p.C * p.Hl * p.Wl + (size_t)(P * i) * p.Wl + P * jj;
+        }
+        const size_t plane = (size_t)p.Hl * p.Wl;
+        bool ok = true;
+        for (int kc = 0; kc < nk; ++kc) {
+            const int st = kc % kEmbedStages;
+            const uint32_t ph = (uint32_t)((kc / kEmbedStages) & 1);
+            ok = ptx::mbar_wait_bounded(&a_empty[st], ph ^ 1u, abort_p, kWaitLimit);
+            ok = __all_sync(0xffffffffu, ok);
+            if (!ok) break;
+            unsigned char* dst = sA + st * kChunkA;
+            if (P == 2) {
+                gather_chunk<2, uint32_t>(dst, base, plane, p.Wl, r, kc, valid);
+            } else if (P == 4) {
+                gather_chunk<4, uint2>(dst, base, plane, p.Wl, r, kc, valid);
+            } else if (P == 8) {
+                gather_chunk<8, uint4>(dst, base, plane, p.Wl, r, kc, valid);
+            } else {
+                for (int g = 0; g < 64 / P; ++g) {
+                    const int f0 = kc * 64 + g * P;
+                    const int c = f0 / (P * P), dy = (f0 % (P * P)) / P;
+                    const __nv_bfloat16* src = base + c * plane + (size_t)dy * p.Wl;
+                    for (int x = 0; x < P; ++x)
+                        *reinterpret_cast<__nv_bfloat16*>(dst + swz_offset(r, g * P + x)) =
+                            valid ? src[x] : __float2bfloat16(0.f);
+                }
+            }
+            ptx::fence_proxy_async_smem();  // the tensor core reads through the async proxy
+            ptx::mbar_arrive(&a_full[st]);
+        }
+        // ---- epilogue: bf16 tile staged in the (now idle) A stages in the
+        // 128-byte swizzle layout, then two TMA stores of 128 rows x 64 columns.
+        ok = ok && ptx::mbar_wait_bounded(&acc_full, 0, abort_p, kWaitLimit);
+        ok = __all_sync(0xffffffffu, ok);
+        if (ok) {
+            ptx::tc_fence_after();
+            const uint32_t taddr = tbase + ((uint32_t)((warp - 4) * 32) << 16);
+#pragma unroll 1
+            for (int c = 0; c < kEmbedBN / 32; ++c) {
+                uint32_t v[32];
+                ptx::tmem_ld32(taddr + c * 32, v);
+                ptx::tmem_wait_ld();
+                unsigned char* stage = sA + (c / 2) * kChunkA;
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    *reinterpret_cast<uint4*>(stage + swz_offset(r, (c % 2) * 32 + 8 * e)) =
+                        make_uint4(ptx::pack_bf16(__uint_as_float(v[8 * e]), __uint_as_float(v[8 * e + 1])),
+                                   ptx::pack_bf16(__uint_as_float(v[8 * e + 2]), __uint_as_float(v[8 * e + 3])),
+                                   ptx::pack_bf16(__uint_as_float(v[8 * e + 4]), __uint_as_float(v[8 * e + 5])),
+                                   ptx::pack_bf16(__uint_as_float(v[8 * e + 6]), __uint_as_float(v[8 * e + 7])));
+            }
+            ptx::fence_proxy_async_smem();
+        }
+        // The four epilogue warps meet before one thread stores the tile.
+        ok = ptx::named_bar_and(1, 128, ok);
+        if (ok && warp == 4 && lane == 0) {
+            for (int h = 0; h < kEmbedBN / 64; ++h)
+                ptx::tma_store_3d(&maps.out[ri], sA + h * kChunkA, nt * kEmbedBN + h * 64, mt * 128, b);
+            ptx::bulk_commit();
+            ptx::bulk_wait_read_all();
+        }
+        if (!ok && lane == 0) atomicOr(p.status, kDevTimeout);
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    if (warp == 2) {
+        ptx::tc_fence_after();
+        ptx::tmem_dealloc(tbase, kEmbedBN);
+    }
+}
+
+constexpr int kEmbedSmem = kEmbedStages * (kChunkA + kEmbedBN * 128) + 1024;
+
+}  // namespace
+
+bool msp_embed_supported(const MspEmbedRun* runs, int n, int E) {
+    if (n < 1 || n > kMaxGemmProblems || E % kEmbedBN != 0) return false;
+    for (int i = 0; i < n; ++i) {
+        const MspEmbedRun& r = runs[i];
+        if (r.K % 64 != 0 || r.P < 1 || 64 % r.P != 0 || ((uintptr_t)r.w & 15) || r.M <= 0) return false;
+    }
+    return true;
+}
+
+cudaError_t launch_msp_embed(const MspEmbedRun* runs, int n, const MspShape& sh, int E, const void* latent,
+                             void* tokens, long long tok_bstride, int batch, unsigned int* status,
+                             cudaStream_t st) {
+    EmbedMaps maps;
+    memset(&maps, 0, sizeof(maps));
+    EmbedParams p;
+    memset(&p, 0, sizeof(p));
+    int tiles = 0;
+    for (int i = 0; i < n; ++i) {
+        const MspEmbedRun& r = runs[i];
+        if (!encode_2d(&maps.w[i], r.w, r.K, E, (long long)r.K * 2, 64, kEmbedBN)) return cudaErrorInvalidValue;
+        {
+            EncodeTiledFn enc = encoder();
+            cuuint64_t dims[3] = {(cuuint64_t)E, (cuuint64_t)r.M, (cuuint64_t)batch};
+            cuuint64_t strides[2] = {(cuuint64_t)E * 2, (cuuint64_t)tok_bstride * 2};
+            cuuint32_t box[3] = {64, 128, 1};
+            cuuint32_t es[3] = {1, 1, 1};
+            if (!enc || enc(&maps.out[i], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3,
+                            (char*)tokens + (size_t)r.tok_off * E * 2, dims, strides, box, es,
+                            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+                return cudaErrorInvalidValue;
+        }
+        EmbedRun& R = p.run[i];
+        R.tile_base = tiles;
+        R.m_tiles = (r.M + 127) / 128;
+        R.M = r.M;
+        R.l0 = r.l0;
+        R.n_l = r.n_l;
+        R.gw = r.gw;
+        R.P = r.P;
+        R.K = r.K;
+        R.tok_off = r.tok_off;
+        tiles += R.m_tiles * (E / kEmbedBN);
+    }
+    p.n_runs = n;
+    p.T = sh.T;
+    p.C = sh.C;
+    p.Hl = sh.Hl;
+    p.Wl = sh.Wl;
+    p.E = E;
+    p.latent = (const __nv_bfloat16*)latent;
+    p.tokens = (__nv_bfloat16*)tokens;
+    p.tok_bstride = tok_bstride;
+    p.status = status;
+    static bool attr = false;
+    if (!attr) {
+        cudaError_t e = cudaFuncSetAttribute(msp_embed_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             kEmbedSmem);
+        if (e != cudaSuccess) return e;
+        attr = true;
+    }
+    return launch_pdl(msp_embed_kernel, dim3((unsigned)tiles, 1, (unsigned)batch), dim3(kThreads), kEmbedSmem,
+                      st, maps, p);
+}
+
+}  // namespace msf
