@@ -193,6 +193,163 @@ def _traffic_from_profile(kernel_src: str):
     return None
 
 
+def _timed(fn, flush, reps=5, warm=2, sleep=True):
+    """Median device time (ms) of fn() between two events; the L2 is flushed
+    and the GPU kept busy while the host enqueues, so launch latency counts
+    but host gaps do not."""
+    import torch
+    ts = []
+    for i in range(warm + reps):
+        flush.fill_(1)
+        if sleep:
+            torch.cuda._sleep(1000000)
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record()
+        fn()
+        b.record()
+        torch.cuda.synchronize()
+        if i >= warm:
+            ts.append(a.elapsed_time(b))
+    return statistics.median(ts)
+
+
+def other_configs(msf, synth, dev, flush, peaks, rank):
+    """The remaining configurations of the workload family, measured after the
+    timed region: the three-scale 48x80 window, the B=4 streaming rollout
+    (120 steps, history 2 -> capacity 4), the 30-layer window pass, and the
+    bandwidth of the pyramid and embedding kernels."""
+    import torch
+    out = {}
+    hbm = float(peaks["hbm_gbs"])
+    bf16 = float(peaks["bf16_tflops"])
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(1234 + rank)
+
+    def rnd(shape):
+        return torch.randn(shape, generator=gen, device=dev, dtype=torch.float32).to(torch.bfloat16)
+
+    def setup(w, embed=False):
+        plan = msf.Plan(msf.make_desc(w.scales, w.grid_h, w.grid_w, w.heads, w.head_dim, w.sink_tokens,
+                                      w.history_frames, w.history_capacity, batch=w.batch,
+                                      latent_channels=w.latent_channels, patch=w.patch,
+                                      embed_dim=w.embed_dim if embed else 0))
+        N, G, H, D, B = plan.info.n_tokens, w.grid_h * w.grid_w, w.heads, w.head_dim, w.batch
+        t = {k: rnd((B, N, H, D)) for k in ("q", "k_win", "v_win")}
+        t["k_sink"], t["v_sink"] = rnd((B, w.sink_tokens, H, D)), rnd((B, w.sink_tokens, H, D))
+        for k in ("k_hist", "v_hist"):
+            ring = torch.zeros((B, max(w.history_capacity, 1), G, H, D), dtype=torch.bfloat16, device=dev)
+            ring[:, :w.history_frames] = rnd((B, w.history_frames, G, H, D))
+            t[k] = ring
+        ws = plan.workspace(dev)
+        plan.bind(ws, t["k_sink"], t["v_sink"], t["k_hist"], t["v_hist"])
+        t["out"] = torch.empty_like(t["q"])
+        t["ws"] = ws
+        return plan, t
+
+    # ---- three-scale window (T=6, 48x80, scales (1,1,2,2,4,4), 16 heads)
+    w3 = synth.THREE_SCALE
+    plan, t = setup(w3)
+    pyr_ms = _timed(lambda: plan.kv_resample(t["k_win"], t["v_win"], msf.MSF_RESAMPLE_FULL), flush)
+    attn_ms = _timed(lambda: plan.mssa_forward(t["q"], t["k_win"], t["v_win"], t["out"]), flush)
+    fl = plan.info.attention_flops
+    out["three_scale"] = {"workload": w3.name, "attention_us": attn_ms * 1e3, "gflop": fl / 1e9,
+                          "tflops": fl / (attn_ms * 1e-3) / 1e12, "frac": fl / (attn_ms * 1e-3) / 1e12 / bf16,
+                          "pyramid_full_us": pyr_ms * 1e3}
+    if plan.device_status() != msf.MSF_OK:
+        raise RuntimeError("device status error (three-scale)")
+    plan.close()
+    del t
+
+    # ---- streaming rollout: B=4, 120 steps, history 2 -> cap 4, sink fixed
+    ws4 = synth.STREAM_480P
+    plan, t = setup(ws4)
+    sets = [{k: rnd(t[k].shape) for k in ("q", "k_win", "v_win")} for _ in range(4)]
+    plan.kv_resample(t["k_win"], t["v_win"], msf.MSF_RESAMPLE_FULL)
+    step_ev, attn_ev, fl_steps = [], [], 0.0
+    torch.cuda.synchronize()
+    for i in range(ws4.steps):
+        x = sets[i % len(sets)]
+        e0, e1, e2, e3 = (torch.cuda.Event(enable_timing=True) for _ in range(4))
+        e0.record()
+        plan.kv_resample(x["k_win"], x["v_win"], msf.MSF_RESAMPLE_WINDOW_ONLY)
+        e1.record()
+        plan.mssa_forward(x["q"], x["k_win"], x["v_win"], t["out"])
+        e2.record()
+        fl_steps += plan.info.attention_flops
+        plan.history_append(x["k_win"], x["v_win"])
+        e3.record()
+        step_ev.append((e0, e3))
+        attn_ev.append((e1, e2))
+    torch.cuda.synchronize()
+    steps_us = sorted(a.elapsed_time(b) * 1e3 for a, b in step_ev)
+    attn_s = sum(a.elapsed_time(b) for a, b in attn_ev) * 1e-3
+    out["stream_b4"] = {"workload": ws4.name, "steps": ws4.steps, "streams": ws4.batch,
+                        "step_us_p50": steps_us[len(steps_us) // 2],
+                        "step_us_p99": steps_us[min(len(steps_us) - 1, int(0.99 * len(steps_us)))],
+                        "attention_frames_per_s": ws4.batch * ws4.steps / attn_s,
+                        "attention_tflops": fl_steps / attn_s / 1e12,
+                        "history_frames_end": plan.info.history_count,
+                        "note": "steps back to back without an L2 flush (a sustained rollout)"}
+    if plan.device_status() != msf.MSF_OK:
+        raise RuntimeError("device status error (stream)")
+    plan.close()
+    del t, sets
+
+    # ---- 30-layer window pass at 480p shapes (MSP embed -> pyramid -> MSSA -> de-embed per layer)
+    wp = synth.PASS_480P
+    plan, t = setup(wp, embed=True)
+    mi = synth.msp_inputs(wp, torch.bfloat16)
+    lat = mi["latent"].to(dev)
+    tiers = {sc: mi["w_tier"][sc].t().contiguous().to(dev) for sc in set(wp.scales)}
+    w_tier = [tiers[sc] for sc in wp.scales]
+    w_out = mi["w_out"].t().contiguous().to(dev)
+    N, E = plan.info.n_tokens, wp.embed_dim
+    tok = torch.empty((wp.batch, N, E), dtype=torch.bfloat16, device=dev)
+    lat_out = torch.empty((wp.batch, wp.latent_channels, wp.grid_h * wp.patch, wp.grid_w * wp.patch),
+                          dtype=torch.bfloat16, device=dev)
+    plan.kv_resample(t["k_win"], t["v_win"], msf.MSF_RESAMPLE_FULL)
+
+    def one_pass():
+        for _ in range(wp.layers):
+            plan.patchify(lat, w_tier, tok)
+            plan.kv_resample(t["k_win"], t["v_win"], msf.MSF_RESAMPLE_WINDOW_ONLY)
+            plan.mssa_forward(t["q"], t["k_win"], t["v_win"], t["out"])
+            plan.unpatchify(0, t["out"].view(wp.batch, N, E), w_out, lat_out)
+
+    pass_ms = _timed(one_pass, flush, reps=3, warm=1, sleep=False)
+    fl = plan.info.attention_flops * wp.layers
+    out["window_pass_30"] = {"workload": wp.name, "layers": wp.layers, "pass_ms": pass_ms,
+                             "us_per_layer": pass_ms * 1e3 / wp.layers, "tflops": fl / (pass_ms * 1e-3) / 1e12}
+
+    # ---- bandwidth of the pyramid and embedding kernels (480p layer, B=1 and the B=4 streams)
+    bw = {}
+    for w in (synth.LAYER_480P, synth.STREAM_480P):
+        plan_b, tb = setup(w, embed=True)
+        G, H, D, B = w.grid_h * w.grid_w, w.heads, w.head_dim, w.batch
+        row = H * D * 2
+        # window part: every fine state read once, pooled to G/4 tokens per coarse group (K and V)
+        fine_states = sum(1 for sc in w.scales if sc == 1)
+        win_bytes = 2 * B * fine_states * G * row * (1 + 0.25)
+        win_ms = _timed(lambda: plan_b.kv_resample(tb["k_win"], tb["v_win"], msf.MSF_RESAMPLE_WINDOW_ONLY),
+                        flush)
+        mi_b = synth.msp_inputs(w, torch.bfloat16)
+        lat_b = mi_b["latent"].to(dev)
+        tiers_b = {sc: mi_b["w_tier"][sc].t().contiguous().to(dev) for sc in set(w.scales)}
+        tok_b = torch.empty((B, plan_b.info.n_tokens, w.embed_dim), dtype=torch.bfloat16, device=dev)
+        emb_ms = _timed(lambda: plan_b.patchify(lat_b, [tiers_b[sc] for sc in w.scales], tok_b), flush)
+        emb_bytes = lat_b.numel() * 2 + tok_b.numel() * 2
+        for name, by, ms in (("pyramid_window", win_bytes, win_ms), ("embed", emb_bytes, emb_ms)):
+            gbs = by / (ms * 1e-3) / 1e9
+            bw[f"{name}_{w.name}"] = {"us": ms * 1e3, "bytes": by, "gbs": gbs, "frac_of_measured": gbs / hbm,
+                                     "frac_of_8tbs": gbs / 8000.0}
+        plan_b.close()
+    out["bandwidth"] = bw
+    out["bandwidth_note"] = ("event time per call including ~4 us of launch latency; bytes are the "
+                             "algorithmic reads + writes")
+    return out
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -361,6 +518,10 @@ def main():
     torch.cuda.synchronize()
     fine_attn_ms = statistics.mean(a.elapsed_time(b) for a, b in fine_ms)
     fine_flops = plan_f.info.attention_flops
+    plan_f.close()
+    del df, wsf, outf
+    peaks, peak_src = _peaks()
+    others = other_configs(msf, synth, dev, flush, peaks, rank)
 
     if rank != 0:
         if world > 1:
@@ -416,6 +577,7 @@ def main():
                      "tflops": fine_flops / (fine_attn_ms * 1e-3) / 1e12,
                      "speedup_vs_all_fine": fine_attn_ms / attn_avg_ms},
         "cpu_baseline": cpu,
+        "other_configs": others,
         "e2e": {"value": world * flops * args.steps / (e2e_ms * 1e-3) / 1e12, "unit": UNIT,
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": e2e_ms / args.steps},
