@@ -119,7 +119,9 @@ struct EmbedMaps {
     CUtensorMap out[kMaxGemmProblems];  // the run's tokens: dims {E, M, B}, rows past M clipped
 };
 
-__global__ void __launch_bounds__(kThreads, 1)
+// Three CTAs per SM (registers <= 85, 67.5 KB of shared memory each) so the
+// 480p window's 420 tiles run in one wave on 152 SMs.
+__global__ void __launch_bounds__(kThreads, 3)
     msp_embed_kernel(const __grid_constant__ EmbedMaps maps, const __grid_constant__ EmbedParams p) {
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -359,6 +361,8 @@ cudaError_t launch_msp_embed(const MspEmbedRun* runs, int n, const MspShape& sh,
     if (!attr) {
         cudaError_t e = cudaFuncSetAttribute(msp_embed_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              kEmbedSmem);
+        if (e != cudaSuccess) return e;
+        e = cudaFuncSetAttribute(msp_embed_kernel, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
         if (e != cudaSuccess) return e;
         attr = true;
     }
