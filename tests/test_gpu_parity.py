@@ -247,3 +247,84 @@ def test_patchify_embed_and_unpatchify_deembed(shared):
                                     w.grid_h * w.patch, w.grid_w * w.patch, synth.to_f64(m["w_out"]))
     e2 = np.abs(lat_out.double().cpu().numpy() - ref_lat)
     assert e2.max() <= 2.0 ** -7 * np.abs(ref_lat).max() + 1e-3, e2.max()
+
+
+# ------------------------------------------------- full-size configurations
+
+def test_streaming_rollout_480p_b4():
+    """The B=4 streaming rollout at its real shapes: history starts at 2 fine
+    frames, grows to the capacity of 4, then evicts the oldest; the sink stays
+    fixed. Five steps cover the growth and two replacements. Each step's
+    attention (one sampled head per step) matches a from-scratch oracle pass
+    over the oracle's own cache, and the ring matches it bit for bit."""
+    w = synth.STREAM_480P
+    x = synth.attention_inputs(w, BF16)
+    plan = make_plan(w, BF16)
+    dx = device_inputs(x, w.history_capacity)
+    bind(plan, dx)
+    hist = ostream.History(synth.to_f64(x["k_hist"]), synth.to_f64(x["v_hist"]), w.history_capacity)
+    G = w.grid_h * w.grid_w
+    for step in range(5):
+        kv = synth.step_kv(w, 4000 + step, BF16)
+        dkv = {k: v.cuda() for k, v in kv.items()}
+        plan.kv_resample(dkv["k_win"], dkv["v_win"],
+                         msf().MSF_RESAMPLE_FULL if step == 0 else msf().MSF_RESAMPLE_WINDOW_ONLY)
+        out = torch.empty_like(dkv["q"])
+        plan.mssa_forward(dkv["q"], dkv["k_win"], dkv["v_win"], out)
+        heads = [(5 * step) % w.heads]
+        hk, hv = hist.frames()
+        ref = omssa.mssa_forward(synth.to_f64(kv["q"]), synth.to_f64(kv["k_win"]), synth.to_f64(kv["v_win"]),
+                                 synth.to_f64(x["k_sink"]), synth.to_f64(x["v_sink"]), hk, hv, w.scales,
+                                 w.grid_h, w.grid_w, heads=heads)
+        mx, mean = err_stats(out, ref, heads=heads)
+        assert mx <= BF16_MAX and mean <= BF16_MEAN, (step, mx, mean)
+        plan.history_append(dkv["k_win"], dkv["v_win"])
+        hist.append(synth.to_f64(kv["k_win"][:, :G]), synth.to_f64(kv["v_win"][:, :G]))
+        torch.cuda.synchronize()
+        n = hist.count
+        assert plan.info.history_count == n
+        assert np.array_equal(dx["k_hist"][:, :n].double().cpu().numpy(), hist.k[:, :n])
+        assert np.array_equal(dx["v_hist"][:, :n].double().cpu().numpy(), hist.v[:, :n])
+    assert hist.count == w.history_capacity
+    assert plan.device_status() == msf().MSF_OK
+
+
+@pytest.mark.parametrize("layer", [0, 29])
+def test_window_pass_layer(layer):
+    """One layer of the 30-layer window pass (q/k/v of std 0.5, layer seed
+    100 + l): MSP embedding of the five states, MSSA (sampled heads) and the
+    de-embedding + unpatchify of the head state, each against the oracle."""
+    w = synth.PASS_480P
+    seed = w.seed + layer
+    x = synth.attention_inputs(w, BF16, seed=seed)
+    m = synth.msp_inputs(w, BF16, seed=seed)
+    plan = make_plan(w, BF16, embed=True)
+    dx = device_inputs(x, w.history_capacity)
+    bind(plan, dx)
+    N, E = plan.info.n_tokens, w.embed_dim
+    tiers = {s: m["w_tier"][s].t().contiguous().cuda() for s in set(w.scales)}
+    tok = torch.empty((w.batch, N, E), dtype=BF16, device="cuda")
+    plan.patchify(m["latent"].cuda(), [tiers[s] for s in w.scales], tok)
+    plan.kv_resample(dx["k_win"], dx["v_win"])
+    out = torch.empty_like(dx["q"])
+    plan.mssa_forward(dx["q"], dx["k_win"], dx["v_win"], out)
+    w_out = m["w_out"].t().contiguous().cuda()
+    lat_out = torch.empty((w.batch, w.latent_channels, w.grid_h * w.patch, w.grid_w * w.patch),
+                          dtype=BF16, device="cuda")
+    plan.unpatchify(0, out.view(w.batch, N, E), w_out, lat_out)
+    torch.cuda.synchronize()
+    assert plan.device_status() == msf().MSF_OK
+    ref_tok = omsp.patchify_window(synth.to_f64(m["latent"]), w.scales, w.patch,
+                                   {s: synth.to_f64(m["w_tier"][s]) for s in set(w.scales)})
+    e = np.abs(tok.double().cpu().numpy() - ref_tok)
+    assert e.max() <= 2.0 ** -7 * np.abs(ref_tok).max() + 1e-3, e.max()
+    heads = [layer % w.heads]
+    ref = oracle_mssa(x, w, 0, heads=heads)
+    mx, mean = err_stats(out, ref, heads=heads)
+    assert mx <= BF16_MAX and mean <= BF16_MEAN, (mx, mean)
+    n0 = plan.info.state_tokens[0]
+    ref_lat = omsp.unpatchify_state(synth.to_f64(out.view(w.batch, N, E)[:, :n0].cpu()), w.patch,
+                                    w.latent_channels, w.grid_h * w.patch, w.grid_w * w.patch,
+                                    synth.to_f64(m["w_out"]))
+    e2 = np.abs(lat_out.double().cpu().numpy() - ref_lat)
+    assert e2.max() <= 2.0 ** -7 * np.abs(ref_lat).max() + 1e-3, e2.max()
