@@ -12,11 +12,11 @@ namespace msf {
 
 // ----------------------------------------------------------------- pooling
 //
-// One thread produces one 16-byte vector of one pooled token's [H*D] row, for
-// K and V together: it loads sigma^2 source vectors of each (all independent
-// 128-bit loads of rows that are contiguous in [B, N, H, D]), sums them in
-// fp32 in a fixed (dy, dx) order, scales by 1/sigma^2 (exact) and rounds
-// once. STRIDED copies the block's top-left vector.
+// One thread produces two adjacent 16-byte vectors of one pooled token's
+// [H*D] row, for K and V together: it loads sigma^2 source vectors of each
+// (independent 128-bit loads of rows that are contiguous in [B, N, H, D]),
+// sums them in fp32 in a fixed (dy, dx) order, scales by 1/sigma^2 (exact)
+// and rounds once. STRIDED copies the block's top-left vectors.
 
 template <typename T>
 struct Vec;
@@ -55,6 +55,48 @@ struct Vec<float> {
     }
 };
 
+// Two adjacent 16-byte vectors of one pooled token, K and V. With the stride
+// known at compile time every source load is issued before the first add, so
+// a thread keeps 4*S*S loads in flight.
+template <typename T, int S>
+__device__ __forceinline__ void pool_pair(const char* sk, const char* sv, char* dk, char* dv, int src_gw,
+                                          int i, int jj, size_t row, int mode) {
+    uint4 xk[S * S][2], xv[S * S][2];
+    const int taps = mode == MSF_RESAMPLE_STRIDED ? 1 : S * S;
+#pragma unroll
+    for (int t = 0; t < S * S; ++t) {
+        if (t < taps) {
+            const int dy = t / S, dx = t % S;
+            const size_t src = (size_t)((S * i + dy) * src_gw + S * jj + dx) * row;
+            xk[t][0] = __ldg(reinterpret_cast<const uint4*>(sk + src));
+            xk[t][1] = __ldg(reinterpret_cast<const uint4*>(sk + src + 16));
+            xv[t][0] = __ldg(reinterpret_cast<const uint4*>(sv + src));
+            xv[t][1] = __ldg(reinterpret_cast<const uint4*>(sv + src + 16));
+        }
+    }
+    if (taps == 1) {
+        *reinterpret_cast<uint4*>(dk) = xk[0][0];
+        *reinterpret_cast<uint4*>(dk + 16) = xk[0][1];
+        *reinterpret_cast<uint4*>(dv) = xv[0][0];
+        *reinterpret_cast<uint4*>(dv + 16) = xv[0][1];
+        return;
+    }
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        float ak[Vec<T>::n], av[Vec<T>::n];
+#pragma unroll
+        for (int e = 0; e < Vec<T>::n; ++e) ak[e] = av[e] = 0.f;
+#pragma unroll
+        for (int t = 0; t < S * S; ++t) {  // fixed (dy, dx) order
+            Vec<T>::add(ak, xk[t][h]);
+            Vec<T>::add(av, xv[t][h]);
+        }
+        const float mul = 1.0f / (float)(S * S);
+        *reinterpret_cast<uint4*>(dk + 16 * h) = Vec<T>::pack(ak, mul);
+        *reinterpret_cast<uint4*>(dv + 16 * h) = Vec<T>::pack(av, mul);
+    }
+}
+
 template <typename T>
 __global__ void __launch_bounds__(256) pool_kernel(const PoolBatch jobs) {
     ptx::grid_dep_wait();
@@ -62,45 +104,51 @@ __global__ void __launch_bounds__(256) pool_kernel(const PoolBatch jobs) {
     const PoolJob& jb = jobs.j[blockIdx.y];
     const int b = blockIdx.z;
     const int idx = blockIdx.x * blockDim.x + threadIdx.x;
-    const int rv = jobs.row_vecs;
-    const int tok = idx / rv;
+    const int rp = jobs.row_vecs / 2;  // vector pairs per token row
+    const int tok = idx / rp;
     if (tok >= jb.out_n) return;
-    const int vec = idx - tok * rv;
+    const int vec = 2 * (idx - tok * rp);
     const int i = tok / jb.out_gw, jj = tok - (tok / jb.out_gw) * jb.out_gw;
-    const int s = jb.sigma;
-    const size_t row = (size_t)rv * 16;
+    const size_t row = (size_t)jobs.row_vecs * 16;
     const char* sk = jb.src_k + (size_t)b * jb.src_bstride + (size_t)vec * 16;
     const char* sv = jb.src_v + (size_t)b * jb.src_bstride + (size_t)vec * 16;
     char* dk = jb.dst_k + (size_t)b * jb.dst_bstride + (size_t)tok * row + (size_t)vec * 16;
     char* dv = jb.dst_v + (size_t)b * jb.dst_bstride + (size_t)tok * row + (size_t)vec * 16;
-    if (jobs.mode == MSF_RESAMPLE_STRIDED || s == 1) {
-        const size_t src = (size_t)((s * i) * jb.src_gw + s * jj) * row;
-        *reinterpret_cast<uint4*>(dk) = __ldg(reinterpret_cast<const uint4*>(sk + src));
-        *reinterpret_cast<uint4*>(dv) = __ldg(reinterpret_cast<const uint4*>(sv + src));
-        return;
-    }
-    float ak[Vec<T>::n], av[Vec<T>::n];
-#pragma unroll
-    for (int e = 0; e < Vec<T>::n; ++e) ak[e] = av[e] = 0.f;
-    for (int dy = 0; dy < s; ++dy) {
-        for (int dx = 0; dx < s; ++dx) {
-            const size_t src = (size_t)((s * i + dy) * jb.src_gw + s * jj + dx) * row;
-            uint4 xk = __ldg(reinterpret_cast<const uint4*>(sk + src));
-            uint4 xv = __ldg(reinterpret_cast<const uint4*>(sv + src));
-            Vec<T>::add(ak, xk);
-            Vec<T>::add(av, xv);
+    switch (jb.sigma) {
+    case 1: pool_pair<T, 1>(sk, sv, dk, dv, jb.src_gw, i, jj, row, jobs.mode); break;
+    case 2: pool_pair<T, 2>(sk, sv, dk, dv, jb.src_gw, i, jj, row, jobs.mode); break;
+    case 4: pool_pair<T, 4>(sk, sv, dk, dv, jb.src_gw, i, jj, row, jobs.mode); break;
+    default: {
+        // Larger strides: same arithmetic, loads issued per tap.
+        const int s = jb.sigma;
+        for (int h = 0; h < 2; ++h) {
+            if (jobs.mode == MSF_RESAMPLE_STRIDED) {
+                const size_t src = (size_t)((s * i) * jb.src_gw + s * jj) * row + 16 * h;
+                *reinterpret_cast<uint4*>(dk + 16 * h) = __ldg(reinterpret_cast<const uint4*>(sk + src));
+                *reinterpret_cast<uint4*>(dv + 16 * h) = __ldg(reinterpret_cast<const uint4*>(sv + src));
+                continue;
+            }
+            float ak[Vec<T>::n], av[Vec<T>::n];
+            for (int e = 0; e < Vec<T>::n; ++e) ak[e] = av[e] = 0.f;
+            for (int dy = 0; dy < s; ++dy)
+                for (int dx = 0; dx < s; ++dx) {
+                    const size_t src = (size_t)((s * i + dy) * jb.src_gw + s * jj + dx) * row + 16 * h;
+                    Vec<T>::add(ak, __ldg(reinterpret_cast<const uint4*>(sk + src)));
+                    Vec<T>::add(av, __ldg(reinterpret_cast<const uint4*>(sv + src)));
+                }
+            const float mul = 1.0f / (float)(s * s);
+            *reinterpret_cast<uint4*>(dk + 16 * h) = Vec<T>::pack(ak, mul);
+            *reinterpret_cast<uint4*>(dv + 16 * h) = Vec<T>::pack(av, mul);
         }
     }
-    const float mul = 1.0f / (float)(s * s);
-    *reinterpret_cast<uint4*>(dk) = Vec<T>::pack(ak, mul);
-    *reinterpret_cast<uint4*>(dv) = Vec<T>::pack(av, mul);
+    }
 }
 
 cudaError_t launch_pool(const PoolBatch& jobs, int batch, bool bf16, cudaStream_t st) {
     if (jobs.n == 0) return cudaSuccess;
     int max_n = 0;
     for (int k = 0; k < jobs.n; ++k) max_n = jobs.j[k].out_n > max_n ? jobs.j[k].out_n : max_n;
-    long long work = (long long)max_n * jobs.row_vecs;
+    long long work = (long long)max_n * (jobs.row_vecs / 2);
     dim3 grid((unsigned)((work + 255) / 256), (unsigned)jobs.n, (unsigned)batch);
     if (bf16)
         return launch_pdl(pool_kernel<__nv_bfloat16>, grid, dim3(256), 0, st, jobs);
