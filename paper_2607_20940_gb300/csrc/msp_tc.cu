@@ -28,7 +28,7 @@ namespace {
 constexpr int kThreads = 256;
 constexpr long long kWaitLimit = 2000000000LL;
 constexpr int kChunkA = 128 * 128;  // 128 rows x 64 bf16 (one K chunk), swizzled
-constexpr int kEmbedBN = 128;
+constexpr int kEmbedBN = 256;
 constexpr int kEmbedStages = 2;
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
@@ -119,9 +119,10 @@ struct EmbedMaps {
     CUtensorMap out[kMaxGemmProblems];  // the run's tokens: dims {E, M, B}, rows past M clipped
 };
 
-// Three CTAs per SM (registers <= 85, 67.5 KB of shared memory each) so the
-// 480p window's 420 tiles run in one wave on 152 SMs.
-__global__ void __launch_bounds__(kThreads, 3)
+// 128 tokens x 256 embedding columns per CTA (one N=256 MMA per K step, half
+// the gathers of 128-column tiles); two CTAs per SM (97 KB of shared memory
+// each), so the 480p window's 210 tiles run in one wave on 152 SMs.
+__global__ void __launch_bounds__(kThreads, 2)
     msp_embed_kernel(const __grid_constant__ EmbedMaps maps, const __grid_constant__ EmbedParams p) {
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -258,8 +259,8 @@ __global__ void __launch_bounds__(kThreads, 3)
             ptx::fence_proxy_async_smem();  // the tensor core reads through the async proxy
             ptx::mbar_arrive(&a_full[st]);
         }
-        // ---- epilogue: bf16 tile staged in the (now idle) A stages in the
-        // 128-byte swizzle layout, then two TMA stores of 128 rows x 64 columns.
+        // ---- epilogue: bf16 tile staged in the (now idle) A and B stages in
+        // the 128-byte swizzle layout, then TMA stores of 128 rows x 64 columns.
         ok = ok && ptx::mbar_wait_bounded(&acc_full, 0, abort_p, kWaitLimit);
         ok = __all_sync(0xffffffffu, ok);
         if (ok) {

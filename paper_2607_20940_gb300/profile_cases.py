@@ -1,0 +1,78 @@
+"""Profiling driver: runs one kernel family of the window pass on seeded
+synthetic inputs so that `ncu -k <kernel>` can capture it in isolation.
+
+    python -m paper_2607_20940_gb300.profile_cases pool     # K/V pyramid at three sizes
+    python -m paper_2607_20940_gb300.profile_cases embed    # MSP patchify + tier embedding
+    python -m paper_2607_20940_gb300.profile_cases deembed  # de-embedding + unpatchify
+
+Each case runs twice after an L2 flush (a 256 MiB write) and checks the
+device status word. Nothing here is timed; the numbers come from the
+profiler.
+"""
+from __future__ import annotations
+
+import sys
+
+import torch
+
+from paper_2607_20940_gb300 import msf, synth
+
+
+def _setup(w, embed=False):
+    dev = torch.device("cuda", 0)
+    x = synth.attention_inputs(w)
+    plan = msf.Plan(msf.make_desc(w.scales, w.grid_h, w.grid_w, w.heads, w.head_dim, w.sink_tokens,
+                                  w.history_frames, w.history_capacity, batch=w.batch,
+                                  latent_channels=w.latent_channels, patch=w.patch,
+                                  embed_dim=w.embed_dim if embed else 0))
+    d = {k: v.to(dev) for k, v in x.items()}
+    for k in ("k_hist", "v_hist"):
+        ring = torch.zeros((w.batch, max(w.history_capacity, 1)) + tuple(d[k].shape[2:]),
+                           dtype=d[k].dtype, device=dev)
+        ring[:, :w.history_frames] = d[k]
+        d[k] = ring
+    ws = plan.workspace(dev)
+    plan.bind(ws, d["k_sink"], d["v_sink"], d["k_hist"], d["v_hist"])
+    return plan, d, ws
+
+
+def run(case: str) -> None:
+    dev = torch.device("cuda", 0)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    if case == "pool":
+        for w, mode in ((synth.LAYER_480P, msf.MSF_RESAMPLE_WINDOW_ONLY),
+                        (synth.STREAM_480P, msf.MSF_RESAMPLE_WINDOW_ONLY),
+                        (synth.THREE_SCALE, msf.MSF_RESAMPLE_FULL)):
+            plan, d, _ = _setup(w)
+            for _ in range(2):
+                flush.fill_(1)
+                plan.kv_resample(d["k_win"], d["v_win"], mode)
+            torch.cuda.synchronize()
+            assert plan.device_status() == msf.MSF_OK
+            plan.close()
+    elif case in ("embed", "deembed"):
+        for w in (synth.LAYER_480P, synth.STREAM_480P):
+            plan, d, _ = _setup(w, embed=True)
+            mi = synth.msp_inputs(w)
+            lat = mi["latent"].to(dev)
+            tiers = {s: mi["w_tier"][s].t().contiguous().to(dev) for s in set(w.scales)}
+            w_out = mi["w_out"].t().contiguous().to(dev)
+            N, E = plan.info.n_tokens, w.embed_dim
+            tok = torch.randn((w.batch, N, E), device=dev).to(torch.bfloat16)
+            lat_out = torch.empty((w.batch, w.latent_channels, w.grid_h * w.patch, w.grid_w * w.patch),
+                                  dtype=torch.bfloat16, device=dev)
+            for _ in range(2):
+                flush.fill_(1)
+                if case == "embed":
+                    plan.patchify(lat, [tiers[s] for s in w.scales], tok)
+                else:
+                    plan.unpatchify(0, tok, w_out, lat_out)
+            torch.cuda.synchronize()
+            assert plan.device_status() == msf.MSF_OK
+            plan.close()
+    else:
+        raise SystemExit(f"unknown case {case!r}: pool, embed or deembed")
+
+
+if __name__ == "__main__":
+    run(sys.argv[1] if len(sys.argv) > 1 else "pool")
