@@ -6,8 +6,8 @@ tokens, history ring of 2 frames):
   MSP patchify + tier embedding of the 5 latent states (16x60x104 -> 4290x1536)
   -> window part of the K/V pyramid -> MSSA attention (Eq. 4)
   -> de-embed + unpatchify of the head state -> history append (head K/V).
-The embedding runs on a second stream beside the pyramid, and the
-de-embedding beside the history append; attention waits for both inputs.
+The embedding runs on a second stream beside the pyramid, and the history
+append beside the de-embedding; attention waits for both of its inputs.
 `value` is the MSSA FLOPs the schedule requires (4*D*H*sum_g Nq_g*Nkv_g =
 202.79 GFLOP) divided by the device time of the whole step, in TFLOP/s.
 Inputs are resident in HBM; the L2 is flushed (a 256 MiB write) between
@@ -407,8 +407,8 @@ def main():
 
     def step(q, k, v, latent, timed_attn=False):
         # Two streams: the MSP embedding of the window runs beside the K/V
-        # pyramid, and the de-embedding of the head state beside the history
-        # update. Attention waits for both of its inputs.
+        # pyramid, and the history update beside the de-embedding of the head
+        # state. Attention waits for both of its inputs.
         fork = torch.cuda.Event()
         fork.record(stream)
         side.wait_event(fork)
@@ -428,8 +428,8 @@ def main():
         attended = torch.cuda.Event()
         attended.record(stream)
         side.wait_event(attended)
-        plan.unpatchify(0, out.view(w.batch, N, E), w_out, lat_out, stream=side)
-        plan.history_append(k, v, stream=stream)
+        plan.history_append(k, v, stream=side)
+        plan.unpatchify(0, out.view(w.batch, N, E), w_out, lat_out, stream=stream)
         joined = torch.cuda.Event()
         joined.record(side)
         stream.wait_event(joined)

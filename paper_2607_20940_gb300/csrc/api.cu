@@ -428,6 +428,11 @@ extern "C" msf_status msf_unpatchify(msf_plan_t plan, int32_t position, const vo
     const int F = sh.C * P * P;
     const int E = p.d.embed_dim;
     char* raw = msf::msp_scratch(p);
+    if (bf16 && msf::msp_deembed_supported(p.st_n[position], F, E)) {
+        return cuda_status(msf::launch_msp_deembed(tokens, (long long)p.N * E, p.N, p.st_off[position], w_out,
+                                                   p.st_n[position], F, E, sh, P, latent_out, p.B,
+                                                   msf::status_word(p), s));
+    }
     if (bf16) {
         msf::GemmTcArgs t;
         t.A = (const char*)tokens + (size_t)p.st_off[position] * E * p.elem;

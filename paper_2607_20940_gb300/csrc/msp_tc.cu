@@ -1,4 +1,4 @@
-// Fused Multi-Scale Patchification kernel on the sm_103a tensor cores
+// Fused Multi-Scale Patchification kernels on the sm_103a tensor cores
 // (Sec. 3.2: a latent state of scale s_l is cut into patches of edge
 // P = patch * s_l; Eq. 3 token counts; feature order (c, dy, dx)).
 //
@@ -7,6 +7,10 @@
 //                     latent straight into 128-byte-swizzled shared memory by
 //                     four warps, B (the tier's [E, K] weight) arrives by TMA,
 //                     and the accumulator is written once as bf16 tokens.
+//
+// msp_deembed_kernel  de-embedding + unpatchify of one window position,
+//                     split-K over a thread-block cluster and reduced over
+//                     distributed shared memory (see its section below).
 //
 // Roles (256 threads): warp 0 TMA producer, warp 1 MMA issuer (one elected
 // lane of the converged warp), warp 2 TMEM allocation, warps 4-7 gather and
@@ -300,6 +304,199 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
 }
 
+
+// ------------------------------------------------------------ de-embedding
+//
+// msp_deembed_kernel: de-embedding + unpatchify of one window position. The
+// K = E contraction is split over the S CTAs of a thread-block cluster
+// (S <= 8 divides 128). Each CTA leaves its fp32 partial 128 x 64 tile in its
+// own shared memory; after a cluster barrier CTA r sums rows [r*128/S,
+// (r+1)*128/S) of all S partials in split order over distributed shared
+// memory, rounds once to bf16 and scatters them into the latent layout
+// [B, C, Hl, Wl]. No partial sums go through global memory and no second
+// kernel is needed.
+
+constexpr int kDeBN = 64;
+constexpr int kDeStages = 4;
+constexpr int kDePartStride = kDeBN + 4;  // floats per staged row (padding spreads the banks)
+
+struct DeembedParams {
+    int M;              // tokens of the position (per stream)
+    int K;              // embedding width E
+    int m_tiles;
+    int splits;         // cluster size along y
+    int P, gw, C, Hl, Wl;
+    int tok_row0;       // first token row of the position
+    __nv_bfloat16* latent;  // [B, C, Hl, Wl]
+    unsigned int* status;
+};
+struct DeembedMaps {
+    CUtensorMap a;  // tokens {E, rows, B}
+    CUtensorMap b;  // W_out {E, F}
+};
+
+__global__ void __launch_bounds__(kThreads, 1)
+    msp_deembed_kernel(const __grid_constant__ DeembedMaps maps, const __grid_constant__ DeembedParams p) {
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    constexpr int kBBytes = kDeBN * 128;
+    constexpr int kStageBytes = kChunkA + kBBytes;
+    float* part = reinterpret_cast<float*>(smem);  // reuses the ring once every MMA is done
+    __shared__ uint64_t full[kDeStages], empty[kDeStages], acc_full;
+    __shared__ uint32_t tmem_base_sh;
+    __shared__ int abort_flag;
+
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    const int tile = blockIdx.x;
+    const int mt = tile % p.m_tiles, nt = tile / p.m_tiles;
+    const int split = (int)ptx::cluster_rank();
+    const int b = blockIdx.z;
+    const int nk_all = p.K / 64;
+    const int kc0 = (int)((long long)split * nk_all / p.splits);
+    const int nk = (int)((long long)(split + 1) * nk_all / p.splits) - kc0;
+
+    if (threadIdx.x == 0) {
+        abort_flag = 0;
+        for (int s = 0; s < kDeStages; ++s) {
+            ptx::mbar_init(&full[s], 1);
+            ptx::mbar_init(&empty[s], 1);
+        }
+        ptx::mbar_init(&acc_full, 1);
+        ptx::fence_mbar_init();
+    }
+    if (warp == 2) {
+        ptx::tmem_alloc(&tmem_base_sh, kDeBN);
+        ptx::tmem_relinquish();
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tbase = tmem_base_sh;
+    volatile int* abort_p = &abort_flag;
+    volatile int never = 0;
+    ptx::grid_dep_wait();  // the tokens written by the attention kernel are visible
+    ptx::grid_dep_launch();
+
+    bool ok = true;
+    if (warp == 0) {
+        if (lane == 0) {
+            ptx::prefetch_tmap(&maps.a);
+            ptx::prefetch_tmap(&maps.b);
+            int issued = 0;
+            for (int kc = 0; kc < nk; ++kc) {
+                const int st = kc % kDeStages;
+                const uint32_t ph = (uint32_t)((kc / kDeStages) & 1);
+                if (!ptx::mbar_wait_bounded(&empty[st], ph ^ 1u, abort_p, kWaitLimit)) {
+                    ok = false;
+                    break;
+                }
+                unsigned char* sa = smem + st * kStageBytes;
+                ptx::mbar_arrive_expect_tx(&full[st], kStageBytes);
+                ptx::tma_load_3d(sa, &maps.a, &full[st], (kc0 + kc) * 64, p.tok_row0 + mt * 128, b);
+                ptx::tma_load_2d(sa + kChunkA, &maps.b, &full[st], (kc0 + kc) * 64, nt * kDeBN);
+                ++issued;
+            }
+            if (!ok) {
+                for (int kc = (issued > kDeStages ? issued - kDeStages : 0); kc < issued; ++kc)
+                    ptx::mbar_wait_bounded(&full[kc % kDeStages], (uint32_t)((kc / kDeStages) & 1), &never,
+                                           kWaitLimit);
+                atomicOr(p.status, kDevTimeout);
+            }
+        }
+    } else if (warp == 1) {
+        constexpr uint32_t idesc = ptx::idesc_bf16(128, kDeBN, false, false);
+        const uint64_t desc0 = ptx::sdesc_sw128(ptx::smem_u32(smem), 16, 1024);
+        for (int kc = 0; kc < nk && ok; ++kc) {
+            const int st = kc % kDeStages;
+            const uint32_t ph = (uint32_t)((kc / kDeStages) & 1);
+            ok = __all_sync(0xffffffffu, ptx::mbar_wait_bounded(&full[st], ph, abort_p, kWaitLimit));
+            if (!ok) break;
+            ptx::tc_fence_after();
+            if (ptx::elect_one_sync()) {
+                const uint64_t ad = desc0 + (uint64_t)(st * (kStageBytes >> 4));
+                const uint64_t bd = ad + (uint64_t)(kChunkA >> 4);
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk)
+                    ptx::mma_ss(tbase, ad + (uint64_t)(kk * 2), bd + (uint64_t)(kk * 2), idesc,
+                                (kc > 0 || kk > 0) ? 1u : 0u);
+                ptx::mma_commit(&empty[st]);
+            }
+            __syncwarp();
+        }
+        if (ptx::elect_one_sync()) ptx::mma_commit(&acc_full);  // also after an abort: drains the MMAs
+        __syncwarp();
+        if (!ok && lane == 0) atomicOr(p.status, kDevTimeout);
+    } else if (warp >= 4) {
+        // ---- this split's partial tile into shared memory (row-major, padded rows)
+        const int r = (warp - 4) * 32 + lane;
+        ok = __all_sync(0xffffffffu, ptx::mbar_wait_bounded(&acc_full, 0, abort_p, kWaitLimit));
+        if (ok) {
+            ptx::tc_fence_after();
+            const uint32_t taddr = tbase + ((uint32_t)((warp - 4) * 32) << 16);
+#pragma unroll
+            for (int c = 0; c < kDeBN / 32; ++c) {
+                uint32_t v[32];
+                ptx::tmem_ld32(taddr + c * 32, v);
+                ptx::tmem_wait_ld();
+                float4* d4 = reinterpret_cast<float4*>(part + r * kDePartStride + c * 32);
+#pragma unroll
+                for (int e = 0; e < 8; ++e)
+                    d4[e] = make_float4(__uint_as_float(v[4 * e]), __uint_as_float(v[4 * e + 1]),
+                                        __uint_as_float(v[4 * e + 2]), __uint_as_float(v[4 * e + 3]));
+            }
+        } else if (lane == 0) {
+            atomicOr(p.status, kDevTimeout);
+        }
+    }
+    // Every thread of every CTA of the cluster: partials are staged.
+    __syncwarp();
+    ptx::tc_fence_before();
+    ptx::cluster_sync();
+    {
+        // ---- rows [rank*R, rank*R + R) of the tile: sum the S partials in
+        // split order, round once, scatter into the latent.
+        const int R = 128 / p.splits;             // rows per CTA
+        const int per_row = kDeBN / 4;            // float4 per row
+        const int P = p.P, PP = P * P;
+        const size_t plane = (size_t)p.Hl * p.Wl;
+        for (int q = threadIdx.x; q < R * per_row; q += kThreads) {
+            const int row = split * R + q / per_row;
+            const int c4 = q % per_row;
+            const int m = mt * 128 + row;
+            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int s = 0; s < p.splits; ++s) {
+                const float4 v = ptx::ld_cluster_f4(part + row * kDePartStride + 4 * c4, (uint32_t)s);
+                acc.x += v.x;
+                acc.y += v.y;
+                acc.z += v.z;
+                acc.w += v.w;
+            }
+            if (m < p.M) {
+                const int i = m / p.gw, jj = m % p.gw;
+                __nv_bfloat16* lat =
+                    p.latent + (size_t)b * p.C * plane + (size_t)(P * i) * p.Wl + (size_t)P * jj;
+                const float vals[4] = {acc.x, acc.y, acc.z, acc.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const int f = nt * kDeBN + 4 * c4 + e;
+                    const int ch = f / PP, dy = (f % PP) / P, dx = f % P;
+                    lat[(size_t)ch * plane + (size_t)dy * p.Wl + dx] = __float2bfloat16_rn(vals[e]);
+                }
+            }
+        }
+    }
+    // No CTA leaves while another may still read its shared memory.
+    ptx::cluster_sync();
+    __syncthreads();
+    if (warp == 2) {
+        ptx::tc_fence_after();
+        ptx::tmem_dealloc(tbase, kDeBN);
+    }
+}
+
+constexpr int kDeSmem = kDeStages * (kChunkA + kDeBN * 128) + 1024;
+static_assert(128 * kDePartStride * 4 <= kDeStages * (kChunkA + kDeBN * 128), "partial tile fits the ring");
+
 constexpr int kEmbedSmem = kEmbedStages * (kChunkA + kEmbedBN * 128) + 1024;
 
 }  // namespace
@@ -369,6 +566,57 @@ cudaError_t launch_msp_embed(const MspEmbedRun* runs, int n, const MspShape& sh,
     }
     return launch_pdl(msp_embed_kernel, dim3((unsigned)tiles, 1, (unsigned)batch), dim3(kThreads), kEmbedSmem,
                       st, maps, p);
+}
+
+
+bool msp_deembed_supported(int M, int F, int E) {
+    return M > 0 && F % kDeBN == 0 && E % 64 == 0 && E >= 64;
+}
+
+cudaError_t launch_msp_deembed(const void* tokens, long long tok_bstride_elems, int tok_rows, int tok_row0,
+                               const void* w_out, int M, int F, int E, const MspShape& sh, int P, void* latent,
+                               int batch, unsigned int* status, cudaStream_t st) {
+    DeembedMaps maps;
+    memset(&maps, 0, sizeof(maps));
+    EncodeTiledFn enc = encoder();
+    if (!enc) return cudaErrorNotSupported;
+    {
+        cuuint64_t dims[3] = {(cuuint64_t)E, (cuuint64_t)tok_rows, (cuuint64_t)batch};
+        cuuint64_t strides[2] = {(cuuint64_t)E * 2, (cuuint64_t)tok_bstride_elems * 2};
+        cuuint32_t box[3] = {64, 128, 1};
+        cuuint32_t es[3] = {1, 1, 1};
+        if (enc(&maps.a, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(tokens), dims, strides, box, es,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+    }
+    if (!encode_2d(&maps.b, w_out, E, F, (long long)E * 2, 64, kDeBN)) return cudaErrorInvalidValue;
+    // The largest power of two <= 8 that leaves each split at least one K chunk.
+    int splits = 8;
+    while (splits > 1 && splits > E / 64) splits /= 2;
+    DeembedParams p;
+    memset(&p, 0, sizeof(p));
+    p.M = M;
+    p.K = E;
+    p.m_tiles = (M + 127) / 128;
+    p.splits = splits;
+    p.P = P;
+    p.gw = sh.Wl / P;
+    p.C = sh.C;
+    p.Hl = sh.Hl;
+    p.Wl = sh.Wl;
+    p.tok_row0 = tok_row0;
+    p.latent = (__nv_bfloat16*)latent;
+    p.status = status;
+    static bool attr = false;
+    if (!attr) {
+        cudaError_t e = cudaFuncSetAttribute(msp_deembed_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             kDeSmem);
+        if (e != cudaSuccess) return e;
+        attr = true;
+    }
+    const dim3 grid((unsigned)(p.m_tiles * (F / kDeBN)), (unsigned)splits, (unsigned)batch);
+    return launch_pdl_cluster(msp_deembed_kernel, grid, dim3(kThreads), kDeSmem, st, dim3(1, splits, 1), maps, p);
 }
 
 }  // namespace msf

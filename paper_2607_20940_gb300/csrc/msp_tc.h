@@ -1,5 +1,5 @@
-// Fused MSP patchify + tier embedding on the sm_103a tensor cores; see
-// msp_tc.cu.
+// Fused MSP kernels (patchify + tier embedding, de-embedding + unpatchify) on
+// the sm_103a tensor cores; see msp_tc.cu.
 #pragma once
 #include <cuda_runtime.h>
 
@@ -25,5 +25,12 @@ bool msp_embed_supported(const MspEmbedRun* runs, int n, int E);
 cudaError_t launch_msp_embed(const MspEmbedRun* runs, int n, const MspShape& sh, int E, const void* latent,
                              void* tokens, long long tok_bstride, int batch, unsigned int* status,
                              cudaStream_t st);
+
+// De-embedding + unpatchify of M tokens (F = C*P*P features, E = K) of one
+// window position; the split-K reduction stays inside a thread-block cluster.
+bool msp_deembed_supported(int M, int F, int E);
+cudaError_t launch_msp_deembed(const void* tokens, long long tok_bstride_elems, int tok_rows, int tok_row0,
+                               const void* w_out, int M, int F, int E, const MspShape& sh, int P, void* latent,
+                               int batch, unsigned int* status, cudaStream_t st);
 
 }  // namespace msf

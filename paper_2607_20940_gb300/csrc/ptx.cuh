@@ -298,6 +298,18 @@ __device__ __forceinline__ void cluster_sync() {
             : "memory");
 }
 
+// Load 16 bytes from the same shared-memory offset in CTA `rank` of the cluster.
+__device__ __forceinline__ float4 ld_cluster_f4(const void* local, uint32_t rank) {
+    uint32_t remote;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
+    float4 v;
+    asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "r"(remote)
+                 : "memory");
+    return v;
+}
+
 // Store a 32-bit value to the same shared-memory offset in CTA `rank` of the cluster.
 __device__ __forceinline__ void st_cluster_u32(const void* local, uint32_t rank, uint32_t v) {
     uint32_t remote;
