@@ -6,7 +6,7 @@ tokens, history ring of 2 frames):
   MSP patchify + tier embedding of the 5 latent states (16x60x104 -> 4290x1536)
   -> window part of the K/V pyramid -> MSSA attention (Eq. 4)
   -> de-embed + unpatchify of the head state -> history append (head K/V).
-The embedding runs on a second stream beside the pyramid, and the history
+The K/V pyramid runs on a second stream beside the embedding, and the history
 append beside the de-embedding; attention waits for both of its inputs.
 `value` is the MSSA FLOPs the schedule requires (4*D*H*sum_g Nq_g*Nkv_g =
 202.79 GFLOP) divided by the device time of the whole step, in TFLOP/s.
@@ -406,17 +406,17 @@ def main():
     side = torch.cuda.Stream(device=dev)
 
     def step(q, k, v, latent, timed_attn=False):
-        # Two streams: the MSP embedding of the window runs beside the K/V
-        # pyramid, and the history update beside the de-embedding of the head
+        # Two streams: the K/V pyramid runs beside the MSP embedding of the
+        # window, and the history update beside the de-embedding of the head
         # state. Attention waits for both of its inputs.
         fork = torch.cuda.Event()
         fork.record(stream)
         side.wait_event(fork)
-        plan.patchify(latent, w_tier, tok, stream=side)
-        embedded = torch.cuda.Event()
-        embedded.record(side)
-        plan.kv_resample(k, v, msf.MSF_RESAMPLE_WINDOW_ONLY, stream=stream)
-        stream.wait_event(embedded)
+        plan.kv_resample(k, v, msf.MSF_RESAMPLE_WINDOW_ONLY, stream=side)
+        pooled = torch.cuda.Event()
+        pooled.record(side)
+        plan.patchify(latent, w_tier, tok, stream=stream)
+        stream.wait_event(pooled)
         if timed_attn:
             a0 = torch.cuda.Event(enable_timing=True)
             a1 = torch.cuda.Event(enable_timing=True)
