@@ -58,6 +58,10 @@ constexpr int kCtrlRegs = 120;
 constexpr int kSoftmaxRegs = 192;
 static_assert(4 * kCtrlRegs + 8 * kSoftmaxRegs == 12 * kLaunchRegs, "register split");
 constexpr long long kWaitLimit = 2000000000LL;  // ~1 s of SM clock
+// Lead tiles per item in the stream-K sequence: the fixed cost of a piece
+// (Q load and pipeline fill, epilogue or partial write) measured as ~5 K/V
+// tiles, so CTAs whose ranges hold many short items get fewer tiles.
+constexpr int kItemLeadTiles = 5;
 
 struct TcSeg {
     int map;
@@ -71,6 +75,7 @@ struct TcGroup {
     int n_items;     // B * H * n_qb
     int n_seg;
     int n_tiles;     // tiles per item
+    int n_virt;      // item stride in the tile sequence: n_tiles + lead tiles
     long long tile_base;  // first tile of this group in the global sequence
     int item_base;        // first item index of this group (merge counters)
     TcSeg seg[kMaxSeg];
@@ -115,7 +120,8 @@ __device__ __forceinline__ float ex2(float x) {
 struct Piece {
     int gi, item, b, h, q_row0, u0, u1;
     bool whole;
-    long long item_start;  // global index of the item's first tile
+    long long item_start;  // global index of the item's first real tile
+    long long t_next;      // sequence position after this piece
 };
 
 __device__ __forceinline__ long long cta_begin(long long c, long long T, long long n) {
@@ -132,20 +138,24 @@ __device__ __forceinline__ Piece locate(const TcParams& p, long long t, long lon
     while (gi < p.n_groups - 1 && t >= p.g[gi + 1].tile_base) ++gi;
     const TcGroup& G = p.g[gi];
     const long long rel = t - G.tile_base;
-    const int item = (int)(rel / G.n_tiles);
-    const int u0 = (int)(rel - (long long)item * G.n_tiles);
-    long long u1 = u0 + (r1 - t);
-    if (u1 > G.n_tiles) u1 = G.n_tiles;
+    const int item = (int)(rel / G.n_virt);
+    const int v0 = (int)(rel - (long long)item * G.n_virt);
+    long long v1 = v0 + (r1 - t);
+    if (v1 > G.n_virt) v1 = G.n_virt;
+    // Each item starts with lead tiles that stand for the fixed cost of a
+    // piece (Q load, pipeline fill, epilogue); they carry no work.
+    const int lead = G.n_virt - G.n_tiles;
     pc.gi = gi;
     pc.item = item;
     const int qb = item % G.n_qb;
     pc.h = (item / G.n_qb) % p.H;
     pc.b = item / (G.n_qb * p.H);
     pc.q_row0 = G.q_begin + qb * 2 * kBlockM;
-    pc.u0 = u0;
-    pc.u1 = (int)u1;
-    pc.whole = (u0 == 0 && u1 == G.n_tiles);
-    pc.item_start = G.tile_base + (long long)item * G.n_tiles;
+    pc.u0 = v0 > lead ? v0 - lead : 0;
+    pc.u1 = (int)v1 > lead ? (int)v1 - lead : 0;
+    pc.whole = (pc.u0 == 0 && pc.u1 == G.n_tiles);
+    pc.item_start = G.tile_base + (long long)item * G.n_virt + lead;
+    pc.t_next = t + (v1 - v0);
     return pc;
 }
 
@@ -236,8 +246,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             // K(j) and V(j) wait for one release: the commit that follows S1 of
             // tile j-2. It covers the last reader of K(j)'s slot (S of tile
             // j-2) and of V(j)'s slot in the 3-deep V ring (PV1 of tile j-3).
-            for (long long t = r0; t < r1 && ok; ++piece) {
+            for (long long t = r0; t < r1 && ok;) {
                 const Piece pc = locate(p, t, r1);
+                t = pc.t_next;
+                if (pc.u0 == pc.u1) continue;  // lead tiles only
                 const TcGroup& G = p.g[pc.gi];
                 if (!ptx::mbar_wait_bounded(&q_empty, (uint32_t)((piece & 1) ^ 1), abort_p,
                                             p.wait_limit)) {
@@ -270,7 +282,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         ptx::tma_load_4d(sV + sv * C::kTileBytes + c * (kBlockN * 128),
                                          &maps.v[G.seg[seg].map], &v_full[sv], c * 64, pc.h, row, pc.b);
                 }
-                t += pc.u1 - pc.u0;
+                ++piece;
             }
             if (!ok) {
                 // Drain: every copy issued must land before the CTA exits.
@@ -334,9 +346,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             int ks = 0, vs = 0;
             uint32_t kph = 0, vph = 0, pph = 0;
             int piece = 0;
-            for (long long t = r0; t < r1 && ok; ++piece) {
+            for (long long t = r0; t < r1 && ok;) {
                 const Piece pc = locate(p, t, r1);
+                t = pc.t_next;
                 const int n = pc.u1 - pc.u0;
+                if (n == 0) continue;  // lead tiles only
                 ok = wait_all(&q_full, (uint32_t)(piece & 1)) && wait_all(&k_full[ks], kph);
                 if (!ok) break;
                 ptx::tc_fence_after();
@@ -392,7 +406,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!ok) break;
                 if (ptx::elect_one_sync()) ptx::mma_commit(&o_full);
                 __syncwarp();
-                t += n;
+                ++piece;
             }
             if (!ok) {
                 // drain_bar covers every MMA issued: TMEM is never released under one.
@@ -416,8 +430,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool ok = true;
         long long js = 0;
         int piece = 0, nsplit = 0;
-        for (long long tt = r0; tt < r1 && ok; ++piece) {
+        for (long long tt = r0; tt < r1 && ok;) {
             const Piece pc = locate(p, tt, r1);
+            tt = pc.t_next;
+            if (pc.u0 == pc.u1) continue;  // lead tiles only
             const TcGroup& G = p.g[pc.gi];
             float m_used = -INFINITY, l = 0.f;
             for (int u = pc.u0; u < pc.u1; ++u, ++js) {
@@ -631,7 +647,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 }
             }
-            tt += pc.u1 - pc.u0;
+            ++piece;
         }
         if (!ok && lane == 0) atomicOr(p.status, kDevTimeout);
     }
@@ -809,9 +825,10 @@ msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st) {
             ts.tile0 = tg.n_tiles;
             tg.n_tiles += (sg.len + kBlockN - 1) / kBlockN;
         }
+        tg.n_virt = tg.n_tiles + kItemLeadTiles;
         tg.tile_base = total_tiles;
         tg.item_base = item_base;
-        total_tiles += (long long)tg.n_items * tg.n_tiles;
+        total_tiles += (long long)tg.n_items * tg.n_virt;
         item_base += tg.n_items;
     }
     tp.n_groups = a.n_groups;
