@@ -244,6 +244,16 @@ uint64_t msf_kernel_launches(void);
 msf_status msf_unpatchify_noalloc(msf_plan_t plan, int32_t position, const void* tokens,
                                   const void* w_out, void* latent_out, void* stream);
 
+/* Failure-path self test (no counterpart in the paper): launches one block
+ * that waits on an mbarrier nothing ever arrives at, with the same bounded
+ * wait every tcgen05 kernel of this library uses, for `limit_cycles` SM
+ * clock cycles (1 .. 2^31). The wait gives up, the block raises the TIMEOUT
+ * bit of the plan's device status word and returns; the next
+ * msf_plan_device_status reports MSF_ERR_TIMEOUT and clears the word, and
+ * the context stays usable. The plan must be bound. Asynchronous on
+ * `stream`. Errors: INVALID_ARG, STATE (not bound), CUDA. */
+msf_status msf_selftest_wait_timeout(msf_plan_t plan, int64_t limit_cycles, void* stream);
+
 /* Synchronise `stream`, read and clear the device status word. Returns
  * MSF_ERR_TIMEOUT if a kernel gave up on a bounded wait since the last
  * check, MSF_OK otherwise. */

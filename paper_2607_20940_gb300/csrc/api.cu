@@ -8,6 +8,7 @@
 #include "msp_tc.h"
 #include "internal.h"
 #include "kernels.h"
+#include "ptx.cuh"
 
 using msf::Plan;
 
@@ -474,6 +475,32 @@ extern "C" msf_status msf_unpatchify(msf_plan_t plan, int32_t position, const vo
     cudaError_t e = msf::launch_gemm_nt_simt(g, p.B, bf16, s);
     if (e != cudaSuccess) return cuda_status(e);
     return cuda_status(msf::launch_unpatchify_raw(raw, latent_out, sh, position, per, 0, p.B, bf16, s));
+}
+
+namespace {
+// Waits on a barrier that nothing arrives at; the bounded wait must give up.
+__global__ void wait_timeout_selftest_kernel(unsigned int* status, long long limit) {
+    __shared__ uint64_t bar;
+    __shared__ int abort_flag;
+    if (threadIdx.x == 0) {
+        abort_flag = 0;
+        msf::ptx::mbar_init(&bar, 1);
+        msf::ptx::fence_mbar_init();
+    }
+    __syncthreads();
+    volatile int* abort_p = &abort_flag;
+    const bool ok = msf::ptx::mbar_wait_bounded(&bar, 0, abort_p, limit);
+    if (!__all_sync(0xffffffffu, ok) && threadIdx.x == 0) atomicOr(status, msf::kDevTimeout);
+}
+}  // namespace
+
+extern "C" msf_status msf_selftest_wait_timeout(msf_plan_t plan, int64_t limit_cycles, void* stream) {
+    if (!plan || limit_cycles < 1 || limit_cycles > (int64_t(1) << 31)) return MSF_ERR_INVALID_ARG;
+    const Plan& p = *plan;
+    if (!p.bound) return MSF_ERR_STATE;
+    msf::note_launch();
+    wait_timeout_selftest_kernel<<<1, 32, 0, (cudaStream_t)stream>>>(msf::status_word(p), (long long)limit_cycles);
+    return cuda_status(cudaGetLastError());
 }
 
 extern "C" msf_status msf_plan_device_status(msf_plan_t plan, void* stream) {

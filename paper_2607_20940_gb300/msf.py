@@ -35,6 +35,7 @@ EXPORTS = (
     "msf_plan_query", "msf_plan_index_map", "msf_plan_bind", "msf_patchify", "msf_unpatchify",
     "msf_kv_resample", "msf_mssa_forward", "msf_mssa_forward_simt", "msf_history_append",
     "msf_plan_device_status", "msf_kernel_launches", "msf_unpatchify_noalloc",
+    "msf_selftest_wait_timeout",
 )
 
 
@@ -95,6 +96,7 @@ def _load():
         "msf_plan_device_status": (ctypes.c_int, [P, VP]),
         "msf_kernel_launches": (ctypes.c_uint64, []),
         "msf_unpatchify_noalloc": (ctypes.c_int, [P, I32, VP, VP, VP, VP]),
+        "msf_selftest_wait_timeout": (ctypes.c_int, [P, ctypes.c_int64, VP]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -214,6 +216,10 @@ def msf_unpatchify_noalloc(plan: int, position: int, tokens, w_out, latent_out, 
                                        _stream(stream)), "msf_unpatchify_noalloc")
 
 
+def msf_selftest_wait_timeout(plan: int, limit_cycles: int, stream=None) -> None:
+    _check(_lib.msf_selftest_wait_timeout(plan, limit_cycles, _stream(stream)), "msf_selftest_wait_timeout")
+
+
 def msf_kernel_launches() -> int:
     return int(_lib.msf_kernel_launches())
 
@@ -292,3 +298,6 @@ class Plan:
 
     def device_status(self, stream=None) -> int:
         return msf_plan_device_status(self.handle, stream)
+
+    def selftest_wait_timeout(self, limit_cycles, stream=None):
+        msf_selftest_wait_timeout(self.handle, limit_cycles, stream)
