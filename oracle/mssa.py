@@ -8,6 +8,11 @@ Tensors: q, k_win, v_win [B, N, H, D] with the window's states concatenated
 in position order, each state row-major over its grid; k_sink, v_sink
 [B, Ns, H, D]; k_hist, v_hist [B, nh, Gh*Gw, H, D] (fine history frames in
 slot order). All inputs are widened to float64 before any arithmetic.
+
+Chunked states (Sec. 5.1, F latent frames per state): a state's tokens are
+F frame grids one after the other, and Subsample acts on each latent frame
+separately (spatial patches, so spatial resampling); ``frames`` = F, 1 by
+default. History frames then hold F*Gh*Gw tokens each.
 """
 from __future__ import annotations
 
@@ -47,19 +52,30 @@ def resample(x: np.ndarray, gh: int, gw: int, sigma: int, mode: int = AVG) -> np
     return out.reshape((B, oh * ow) + rest)
 
 
-def group_context(kv_win, kv_sink, kv_hist, scales, grid_h, grid_w, g, mode=AVG):
+def resample_frames(x: np.ndarray, frames: int, gh: int, gw: int, sigma: int,
+                    mode: int = AVG) -> np.ndarray:
+    """Subsample of a chunk: x [B, frames*gh*gw, ...] holds ``frames`` latent
+    frame grids in order; each is resampled on its own and the results are
+    concatenated in the same frame order."""
+    x = np.asarray(x, dtype=np.float64)
+    n = gh * gw
+    return np.concatenate([resample(x[:, f * n:(f + 1) * n], gh, gw, sigma, mode)
+                           for f in range(frames)], axis=1)
+
+
+def group_context(kv_win, kv_sink, kv_hist, scales, grid_h, grid_w, g, mode=AVG, frames=1):
     """C_a^MSSA of Eq. 4 for query scale g: [sink || history@g || state_l@max(1,g/s_l)].
 
     kv_* are one of K or V. Returns [B, Nctx, H, D] float64.
     """
-    offs = schedule.token_offsets(scales, grid_h, grid_w)
-    cnt = schedule.token_counts(scales, grid_h, grid_w)
+    offs = schedule.token_offsets(scales, grid_h, grid_w, frames)
+    cnt = schedule.token_counts(scales, grid_h, grid_w, frames)
     parts = [np.asarray(kv_sink, dtype=np.float64)]
     for f in range(kv_hist.shape[1]):
-        parts.append(resample(kv_hist[:, f], grid_h, grid_w, g, mode))
+        parts.append(resample_frames(kv_hist[:, f], frames, grid_h, grid_w, g, mode))
     for l, s in enumerate(scales):
         st = np.asarray(kv_win[:, offs[l]:offs[l] + cnt[l]], dtype=np.float64)
-        parts.append(resample(st, grid_h // s, grid_w // s, max(1, g // s), mode))
+        parts.append(resample_frames(st, frames, grid_h // s, grid_w // s, max(1, g // s), mode))
     return np.concatenate(parts, axis=1)
 
 
@@ -83,7 +99,7 @@ def attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float) -> np.n
 
 
 def mssa_forward(q, k_win, v_win, k_sink, v_sink, k_hist, v_hist, scales, grid_h, grid_w,
-                 mode=AVG, softmax_scale=None, heads=None):
+                 mode=AVG, softmax_scale=None, heads=None, frames=1):
     """MSSA over one window: every query group attends to its Eq. 4 context.
 
     Output [B, N, H, D] in the same token order as q. ``heads`` optionally
@@ -95,28 +111,28 @@ def mssa_forward(q, k_win, v_win, k_sink, v_sink, k_hist, v_hist, scales, grid_h
     scale = D ** -0.5 if not softmax_scale else softmax_scale
     out = np.full(q.shape, np.nan, dtype=np.float64)
     hsel = list(range(q.shape[2])) if heads is None else list(heads)
-    for grp in schedule.query_groups(scales, grid_h, grid_w):
+    for grp in schedule.query_groups(scales, grid_h, grid_w, frames):
         kc = group_context(k_win[:, :, hsel], k_sink[:, :, hsel], k_hist[:, :, :, hsel],
-                           scales, grid_h, grid_w, grp.scale, mode)
+                           scales, grid_h, grid_w, grp.scale, mode, frames)
         vc = group_context(v_win[:, :, hsel], v_sink[:, :, hsel], v_hist[:, :, :, hsel],
-                           scales, grid_h, grid_w, grp.scale, mode)
+                           scales, grid_h, grid_w, grp.scale, mode, frames)
         qg = q[:, grp.q_begin:grp.q_end][:, :, hsel]
         out[:, grp.q_begin:grp.q_end, hsel] = attention(qg, kc, vc, scale)
     return out
 
 
-def pyramid_segment(kv_win, kv_hist, scales, grid_h, grid_w, g, mode=AVG):
+def pyramid_segment(kv_win, kv_hist, scales, grid_h, grid_w, g, mode=AVG, frames=1):
     """Only the resampled part of group g's context: history@g followed by the
     window states finer than g, each pooled to scale g. [B, n, H, D] float64."""
-    offs = schedule.token_offsets(scales, grid_h, grid_w)
-    cnt = schedule.token_counts(scales, grid_h, grid_w)
+    offs = schedule.token_offsets(scales, grid_h, grid_w, frames)
+    cnt = schedule.token_counts(scales, grid_h, grid_w, frames)
     parts = []
     for f in range(kv_hist.shape[1]):
-        parts.append(resample(kv_hist[:, f], grid_h, grid_w, g, mode))
+        parts.append(resample_frames(kv_hist[:, f], frames, grid_h, grid_w, g, mode))
     for l, s in enumerate(scales):
         if s < g:
             st = np.asarray(kv_win[:, offs[l]:offs[l] + cnt[l]], dtype=np.float64)
-            parts.append(resample(st, grid_h // s, grid_w // s, g // s, mode))
+            parts.append(resample_frames(st, frames, grid_h // s, grid_w // s, g // s, mode))
     if not parts:
         return np.zeros((kv_win.shape[0], 0) + tuple(kv_win.shape[2:]))
     return np.concatenate(parts, axis=1)

@@ -5,6 +5,11 @@ Notation follows Sec. 4.1: window positions l = 1..T carry patch sizes
 p_l = s_l * p with s_l in {1, 2, 4, ...}, non-decreasing in l. A latent frame
 tokenised at the native patch p gives a fine Gh x Gw grid; at p_l it gives a
 (Gh/s_l) x (Gw/s_l) grid, so N_l = Gh*Gw / s_l^2 (Eq. 3).
+
+Chunked states (Sec. 5.1: each window state is a chunk of F latent frames):
+patchification is spatial, so a state holds F such grids, N_l = F*Gh*Gw/s_l^2,
+its tokens ordered (latent frame, row, col). Every per-frame count above is
+multiplied by F; ``frames`` defaults to 1 (one latent frame per state).
 """
 from __future__ import annotations
 
@@ -35,15 +40,16 @@ def state_grid(grid_h: int, grid_w: int, s: int) -> Tuple[int, int]:
     return grid_h // s, grid_w // s
 
 
-def token_counts(scales: Sequence[int], grid_h: int, grid_w: int) -> List[int]:
-    """N_l^MSP = HW / p_l^2 (Eq. 3), in tokens of the fine grid Gh x Gw."""
-    return [(grid_h * grid_w) // (s * s) for s in scales]
+def token_counts(scales: Sequence[int], grid_h: int, grid_w: int, frames: int = 1) -> List[int]:
+    """N_l^MSP = HW / p_l^2 (Eq. 3) per latent frame, in tokens of the fine
+    grid Gh x Gw; a chunk of F frames has F times as many."""
+    return [frames * ((grid_h // s) * (grid_w // s)) for s in scales]
 
 
-def token_offsets(scales, grid_h, grid_w) -> List[int]:
+def token_offsets(scales, grid_h, grid_w, frames: int = 1) -> List[int]:
     """Start of state l's tokens in the window sequence (states in position order)."""
     out, acc = [], 0
-    for n in token_counts(scales, grid_h, grid_w):
+    for n in token_counts(scales, grid_h, grid_w, frames):
         out.append(acc)
         acc += n
     return out
@@ -55,10 +61,11 @@ def rho_tok(scales: Sequence[int]) -> Fraction:
     return sum((Fraction(1, s * s) for s in scales), Fraction(0)) / T
 
 
-def token_of(scales, grid_h, grid_w, l: int, i: int, j: int) -> int:
-    """Index of token (row i, col j) of state l (0-based) in the window sequence."""
-    gw = grid_w // scales[l]
-    return token_offsets(scales, grid_h, grid_w)[l] + i * gw + j
+def token_of(scales, grid_h, grid_w, l: int, i: int, j: int, f: int = 0, frames: int = 1) -> int:
+    """Index of token (row i, col j) of latent frame f of state l (0-based) in
+    the window sequence."""
+    gh, gw = grid_h // scales[l], grid_w // scales[l]
+    return token_offsets(scales, grid_h, grid_w, frames)[l] + (f * gh + i) * gw + j
 
 
 class Group(NamedTuple):
@@ -68,10 +75,10 @@ class Group(NamedTuple):
     q_end: int          # one past the last
 
 
-def query_groups(scales, grid_h, grid_w) -> List[Group]:
+def query_groups(scales, grid_h, grid_w, frames: int = 1) -> List[Group]:
     """Queries that share one context: all tokens of states with equal s_l."""
-    offs = token_offsets(scales, grid_h, grid_w)
-    cnt = token_counts(scales, grid_h, grid_w)
+    offs = token_offsets(scales, grid_h, grid_w, frames)
+    cnt = token_counts(scales, grid_h, grid_w, frames)
     groups = []
     for g in sorted(set(scales)):
         st = tuple(l for l, s in enumerate(scales) if s == g)
@@ -79,7 +86,7 @@ def query_groups(scales, grid_h, grid_w) -> List[Group]:
     return groups
 
 
-def context_rows(scales, grid_h, grid_w, sink_tokens: int, n_hist: int, g: int):
+def context_rows(scales, grid_h, grid_w, sink_tokens: int, n_hist: int, g: int, frames: int = 1):
     """The rows of C_a^MSSA (Eq. 4) for queries of scale g, in context order.
 
     Each row is (kind, frame, stride, row, col): kind SINK has frame 0,
@@ -87,6 +94,9 @@ def context_rows(scales, grid_h, grid_w, sink_tokens: int, n_hist: int, g: int):
     (row, col) on the (Gh/st) x (Gw/st) grid of that frame pooled by
     st = g (history is fine, p_b = p); kind WIN has frame = window position l
     and (row, col) on the grid of state l pooled by st = max(1, g / s_l).
+    For chunked states each history frame and window state holds F latent
+    frames, each subsampled on its own; latent frame f's grid rows are
+    numbered f*gh .. f*gh + gh - 1 (gh the rows of one pooled frame).
     """
     rows = []
     for n in range(sink_tokens):
@@ -94,41 +104,45 @@ def context_rows(scales, grid_h, grid_w, sink_tokens: int, n_hist: int, g: int):
     for f in range(n_hist):
         st = max(1, g // 1)
         gh, gw = grid_h // st, grid_w // st
-        for i in range(gh):
-            for j in range(gw):
-                rows.append((HIST, f, st, i, j))
+        for lf in range(frames):
+            for i in range(gh):
+                for j in range(gw):
+                    rows.append((HIST, f, st, lf * gh + i, j))
     for l, s in enumerate(scales):
         st = max(1, g // s)
         gh, gw = grid_h // (s * st), grid_w // (s * st)
-        for i in range(gh):
-            for j in range(gw):
-                rows.append((WIN, l, st, i, j))
+        for lf in range(frames):
+            for i in range(gh):
+                for j in range(gw):
+                    rows.append((WIN, l, st, lf * gh + i, j))
     return rows
 
 
-def context_length(scales, grid_h, grid_w, sink_tokens, n_hist, g) -> int:
-    return len(context_rows(scales, grid_h, grid_w, sink_tokens, n_hist, g))
+def context_length(scales, grid_h, grid_w, sink_tokens, n_hist, g, frames: int = 1) -> int:
+    return len(context_rows(scales, grid_h, grid_w, sink_tokens, n_hist, g, frames))
 
 
-def attention_pairs(scales, grid_h, grid_w, sink_tokens, n_hist) -> int:
+def attention_pairs(scales, grid_h, grid_w, sink_tokens, n_hist, frames: int = 1) -> int:
     """Query-key pairs MSSA evaluates per (stream, head): sum_g Nq_g * Nkv_g."""
     tot = 0
-    for grp in query_groups(scales, grid_h, grid_w):
+    for grp in query_groups(scales, grid_h, grid_w, frames):
         nq = grp.q_end - grp.q_begin
-        tot += nq * context_length(scales, grid_h, grid_w, sink_tokens, n_hist, grp.scale)
+        tot += nq * context_length(scales, grid_h, grid_w, sink_tokens, n_hist, grp.scale, frames)
     return tot
 
 
-def msp_only_pairs(scales, grid_h, grid_w, sink_tokens, n_hist) -> int:
+def msp_only_pairs(scales, grid_h, grid_w, sink_tokens, n_hist, frames: int = 1) -> int:
     """Pairs when every query sees the un-resampled context (MSP without MSSA):
     each of the N_MSP queries against sink + fine history + all window tokens."""
-    n = sum(token_counts(scales, grid_h, grid_w))
-    return n * (sink_tokens + n_hist * grid_h * grid_w + n)
+    n = sum(token_counts(scales, grid_h, grid_w, frames))
+    return n * (sink_tokens + n_hist * frames * grid_h * grid_w + n)
 
 
-def attention_flops(scales, grid_h, grid_w, sink_tokens, n_hist, heads, head_dim, batch=1) -> int:
+def attention_flops(scales, grid_h, grid_w, sink_tokens, n_hist, heads, head_dim, batch=1,
+                    frames: int = 1) -> int:
     """Algorithmic FLOPs: 2 for each multiply-add of Q K^T and of P V."""
-    return 4 * head_dim * heads * batch * attention_pairs(scales, grid_h, grid_w, sink_tokens, n_hist)
+    return 4 * head_dim * heads * batch * attention_pairs(scales, grid_h, grid_w, sink_tokens,
+                                                          n_hist, frames)
 
 
 def r_mssa_eq5(scales: Sequence[int], n_sink_frames: int, n_hist: int) -> Fraction:

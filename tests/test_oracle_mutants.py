@@ -1,0 +1,113 @@
+"""Planted mistakes: each test swaps one plausible error into the fp64 oracle
+(on the CPU, through monkeypatch, so the oracle itself is untouched) and
+checks that at least one of its pins in test_oracle_pins.py then fails.
+A pin that still passed with the mistake in place would not be pinning
+that part of the oracle.
+"""
+import numpy as np
+import pytest
+
+import test_oracle_pins as pins
+from oracle import msp, mssa, schedule
+
+
+def _fails(fn, *args):
+    with pytest.raises(AssertionError):
+        fn(*args)
+
+
+def test_pool_normalised_by_sigma_not_sigma_squared(monkeypatch):
+    good = mssa.resample
+
+    def bad(x, gh, gw, sigma, mode=mssa.AVG):
+        y = good(x, gh, gw, sigma, mode)
+        return y * sigma if mode == mssa.AVG else y
+    monkeypatch.setattr(mssa, "resample", bad)
+    _fails(pins.test_resample_constant_field_is_identity, mssa.AVG, 2)
+    _fails(pins.test_equal_keys_give_weighted_value_mean)
+
+
+def test_strided_pick_off_the_corner(monkeypatch):
+    good = mssa.resample
+
+    def bad(x, gh, gw, sigma, mode=mssa.AVG):
+        if mode != mssa.STRIDED or sigma == 1:
+            return good(x, gh, gw, sigma, mode)
+        x = np.asarray(x, dtype=np.float64)
+        grid = x.reshape((x.shape[0], gh, gw) + x.shape[2:])
+        out = grid[:, 1::sigma, 1::sigma]      # bottom-right of a 2x2 block
+        return out.reshape((x.shape[0], -1) + x.shape[2:])
+    monkeypatch.setattr(mssa, "resample", bad)
+    _fails(pins.test_resample_linear_ramp, 2)
+
+
+def test_query_state_left_out_of_its_own_context(monkeypatch):
+    good = schedule.context_rows
+
+    def bad(scales, gh, gw, ns, nh, g, frames=1):
+        return [r for r in good(scales, gh, gw, ns, nh, g, frames)
+                if not (r[0] == schedule.WIN and scales[r[1]] == g)]
+    monkeypatch.setattr(schedule, "context_rows", bad)
+    _fails(pins.test_eq5_pair_reduction_matches_paper)
+
+
+def test_history_not_pooled_for_coarse_queries(monkeypatch):
+    good = mssa.group_context
+
+    def bad(kv_win, kv_sink, kv_hist, scales, gh, gw, g, mode=mssa.AVG, frames=1):
+        # the correct context, but with the history frames at full resolution
+        ctx = good(kv_win, kv_sink, kv_hist[:, :0], scales, gh, gw, g, mode, frames)
+        ns = np.asarray(kv_sink).shape[1]
+        hist = [np.asarray(kv_hist[:, f], dtype=np.float64) for f in range(kv_hist.shape[1])]
+        return np.concatenate([ctx[:, :ns]] + hist + [ctx[:, ns:]], axis=1)
+    monkeypatch.setattr(mssa, "group_context", bad)
+    _fails(pins.test_brute_force_eq4, mssa.AVG, (1, 2), 4, 4, 3, 1)
+
+
+def test_softmax_scale_dropped(monkeypatch):
+    good = mssa.attention
+    monkeypatch.setattr(mssa, "attention", lambda q, k, v, scale: good(q, k, v, 1.0))
+    _fails(pins.test_all_fine_reduces_to_plain_attention_sdpa)
+
+
+def test_patch_offsets_swapped(monkeypatch):
+    def bad(latent, P):
+        x = np.asarray(latent, dtype=np.float64)
+        B, C, Hl, Wl = x.shape
+        gh, gw = Hl // P, Wl // P
+        out = np.empty((B, gh, gw, C * P * P))
+        for c in range(C):
+            for dy in range(P):
+                for dx in range(P):
+                    out[:, :, :, c * P * P + dx * P + dy] = x[:, c, dy::P, dx::P]
+        return out.reshape(B, gh * gw, C * P * P)
+    monkeypatch.setattr(msp, "patchify", bad)
+    _fails(pins.test_patch_embedding_equals_strided_conv)
+    _fails(pins.test_chunked_patch_embedding_equals_conv3d)
+
+
+def test_chunk_pooled_across_latent_frames(monkeypatch):
+    good = mssa.resample_frames
+
+    def bad(x, frames, gh, gw, sigma, mode=mssa.AVG):
+        # per-frame pooling followed by a temporal mean over frame pairs
+        y = good(x, frames, gh, gw, sigma, mode).copy()
+        n = y.shape[1] // frames
+        for f in range(0, frames - 1, 2):
+            m = 0.5 * (y[:, f * n:(f + 1) * n] + y[:, (f + 1) * n:(f + 2) * n])
+            y[:, f * n:(f + 2) * n] = np.concatenate([m, m], axis=1)
+        return y
+    monkeypatch.setattr(mssa, "resample_frames", bad)
+    _fails(pins.test_chunked_resample_is_per_frame, mssa.AVG, 2)
+    _fails(pins.test_chunked_brute_force_eq4, mssa.AVG, (1, 2), 4, 4, 2, 3, 1)
+
+
+def test_chunk_tokens_frame_minor(monkeypatch):
+    good = msp.patchify
+
+    def bad(latent, P):
+        x = np.asarray(latent, dtype=np.float64)
+        per = [good(x[:, :, f], P) for f in range(x.shape[2])]
+        return np.stack(per, axis=2).reshape(x.shape[0], -1, per[0].shape[2])
+    monkeypatch.setattr(msp, "patchify_chunk", bad)
+    _fails(pins.test_chunked_patch_embedding_equals_conv3d)

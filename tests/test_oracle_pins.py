@@ -279,3 +279,101 @@ def test_history_ring_keeps_newest_frames():
         live = sorted(int(k[0, s, 0, 0, 0]) for s in range(k.shape[1]))
         assert live == list(range(max(0, f + 1 - cap), f + 1))
         assert np.all(v == k + 100)
+
+
+# --------------------------------------------- chunked states (Sec. 5.1) --
+# The paper's window holds T = 5 chunks of 3 latent frames each; patches are
+# spatial, so Eq. 3 applies per latent frame and Subsample acts on each
+# latent frame's grid separately.
+
+def test_chunked_counts_keep_the_printed_token_ratio():
+    g = _golden()["rho_tok"]
+    cnt = schedule.token_counts(g["scales"], 30, 52, frames=3)
+    assert cnt == [4680, 4680, 1170, 1170, 1170]
+    assert Fraction(sum(cnt), 5 * 3 * 30 * 52) == Fraction(55, 100)
+    assert 1 - sum(cnt) / (5 * 3 * 1560) == pytest.approx(g["token_reduction"], abs=1e-12)
+
+
+def test_chunked_contexts_keep_the_printed_pair_ratio():
+    """Every per-frame count scales by F, every pair count by F^2, so Eq. 5's
+    closed form (written per frame) must still equal the chunked enumeration."""
+    g = _golden()["r_mssa"]
+    scales, gh, gw, F = g["scales"], 30, 52, 3
+    sink = F * gh * gw * g["sink_frames"]
+    pairs = schedule.attention_pairs(scales, gh, gw, sink, g["history_frames"], frames=F)
+    dense = schedule.msp_only_pairs(scales, gh, gw, sink, g["history_frames"], frames=F)
+    r = 1 - Fraction(pairs, dense)
+    assert r == schedule.r_mssa_eq5(scales, g["sink_frames"], g["history_frames"])
+    assert round(float(r), g["printed_digits"]) == pytest.approx(g["value"], abs=1e-12)
+    # and exactly F^2 times the one-frame pair count
+    assert pairs == F * F * schedule.attention_pairs(scales, gh, gw, gh * gw, 1)
+
+
+@pytest.mark.parametrize("mode", [mssa.AVG, mssa.STRIDED])
+@pytest.mark.parametrize("sigma", [2, 4])
+def test_chunked_resample_is_per_frame(mode, sigma):
+    """Frame f of the chunk holds 100 f + row: pooled rows stay inside their
+    frame (no temporal mixing) and land at the block centre (AVG) or the
+    block's top row (STRIDED)."""
+    F, gh, gw = 3, 8, 4
+    f, i, _ = np.meshgrid(np.arange(F), np.arange(gh), np.arange(gw), indexing="ij")
+    x = (100.0 * f + i).reshape(1, F * gh * gw, 1, 1)
+    y = mssa.resample_frames(x, F, gh, gw, sigma, mode).reshape(F, gh // sigma, gw // sigma)
+    of, oi, _ = np.meshgrid(np.arange(F), np.arange(gh // sigma), np.arange(gw // sigma),
+                            indexing="ij")
+    off = (sigma - 1) / 2 if mode == mssa.AVG else 0
+    np.testing.assert_allclose(y, 100.0 * of + sigma * oi + off, rtol=0, atol=1e-12)
+
+
+def test_chunked_index_rows_are_bijective():
+    scales, gh, gw, F = (1, 2, 4), 8, 8, 3
+    seen = set()
+    for l, s in enumerate(scales):
+        for f in range(F):
+            for i in range(gh // s):
+                for j in range(gw // s):
+                    seen.add(schedule.token_of(scales, gh, gw, l, i, j, f=f, frames=F))
+    assert seen == set(range(sum(schedule.token_counts(scales, gh, gw, F))))
+
+
+def _rand_chunk_inputs(rng, scales, gh, gw, F, ns, nh, H, D, B=1):
+    N = sum(schedule.token_counts(scales, gh, gw, F))
+    G = F * gh * gw
+    return dict(
+        q=rng.standard_normal((B, N, H, D)), k_win=rng.standard_normal((B, N, H, D)),
+        v_win=rng.standard_normal((B, N, H, D)), k_sink=rng.standard_normal((B, ns, H, D)),
+        v_sink=rng.standard_normal((B, ns, H, D)), k_hist=rng.standard_normal((B, nh, G, H, D)),
+        v_hist=rng.standard_normal((B, nh, G, H, D)))
+
+
+@pytest.mark.parametrize("mode", [mssa.AVG, mssa.STRIDED])
+@pytest.mark.parametrize("scales,gh,gw,F,ns,nh", [
+    ((1, 2), 4, 4, 2, 3, 1),
+    ((1, 1, 2), 4, 4, 3, 2, 2),
+    ((2, 4), 4, 8, 2, 1, 1),
+])
+def test_chunked_brute_force_eq4(mode, scales, gh, gw, F, ns, nh):
+    rng = np.random.default_rng(13)
+    x = _rand_chunk_inputs(rng, scales, gh, gw, F, ns, nh, H=2, D=5)
+    out = mssa.mssa_forward(x["q"], x["k_win"], x["v_win"], x["k_sink"], x["v_sink"],
+                            x["k_hist"], x["v_hist"], scales, gh, gw, mode=mode, frames=F)
+    ref = brute.mssa_brute(x["q"].tolist(), x["k_win"].tolist(), x["v_win"].tolist(),
+                           x["k_sink"].tolist(), x["v_sink"].tolist(), x["k_hist"].tolist(),
+                           x["v_hist"].tolist(), scales, gh, gw, mode=mode, frames=F)
+    np.testing.assert_allclose(out, np.array(ref), rtol=0, atol=1e-12)
+
+
+def test_chunked_patch_embedding_equals_conv3d():
+    """A chunk's tier embedding == Conv3d with kernel = stride = (1, P, P),
+    tokens in (frame, row, col) order; the rearrangement inverts exactly."""
+    rng = np.random.default_rng(2)
+    B, C, F, Hl, Wl, P, E = 2, 3, 3, 8, 12, 4, 5
+    x = rng.standard_normal((B, C, F, Hl, Wl))
+    W = rng.standard_normal((C * P * P, E))
+    t = msp.patchify_chunk(x, P)
+    conv = torch.nn.functional.conv3d(torch.from_numpy(x),
+                                      torch.from_numpy(W.T.reshape(E, C, 1, P, P).copy()),
+                                      stride=(1, P, P))
+    ref = conv.numpy().reshape(B, E, -1).transpose(0, 2, 1)
+    np.testing.assert_allclose(t @ W, ref, rtol=0, atol=1e-12)
+    assert np.array_equal(msp.unpatchify_chunk(t, P, C, F, Hl, Wl), x)
