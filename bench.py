@@ -216,7 +216,8 @@ def _timed(fn, flush, reps=5, warm=2, sleep=True):
 
 def other_configs(msf, synth, dev, flush, peaks, rank):
     """The remaining configurations of the workload family, measured after the
-    timed region: the three-scale 48x80 window, the B=4 streaming rollout
+    timed region: the three-scale 48x80 window, the paper's chunked layout
+    (3 latent frames per state) beside its all-fine window, the B=4 streaming rollout
     (120 steps, history 2 -> capacity 4), the 30-layer window pass, and the
     bandwidth of the pyramid and embedding kernels."""
     import torch
@@ -233,8 +234,9 @@ def other_configs(msf, synth, dev, flush, peaks, rank):
         plan = msf.Plan(msf.make_desc(w.scales, w.grid_h, w.grid_w, w.heads, w.head_dim, w.sink_tokens,
                                       w.history_frames, w.history_capacity, batch=w.batch,
                                       latent_channels=w.latent_channels, patch=w.patch,
-                                      embed_dim=w.embed_dim if embed else 0))
-        N, G, H, D, B = plan.info.n_tokens, w.grid_h * w.grid_w, w.heads, w.head_dim, w.batch
+                                      embed_dim=w.embed_dim if embed else 0,
+                                      frames_per_state=w.frames))
+        N, G, H, D, B = plan.info.n_tokens, w.fine_tokens, w.heads, w.head_dim, w.batch
         t = {k: rnd((B, N, H, D)) for k in ("q", "k_win", "v_win")}
         t["k_sink"], t["v_sink"] = rnd((B, w.sink_tokens, H, D)), rnd((B, w.sink_tokens, H, D))
         for k in ("k_hist", "v_hist"):
@@ -260,6 +262,36 @@ def other_configs(msf, synth, dev, flush, peaks, rank):
         raise RuntimeError("device status error (three-scale)")
     plan.close()
     del t
+
+    # ---- the paper's chunked layout: 3 latent frames per state (12870 tokens),
+    #      sink = one chunk, one history chunk; MSSA beside the all-fine window
+    wc = synth.CHUNKED_480P
+    plan, t = setup(wc)
+    pyr_ms = _timed(lambda: plan.kv_resample(t["k_win"], t["v_win"], msf.MSF_RESAMPLE_FULL), flush)
+    attn_ms = _timed(lambda: plan.mssa_forward(t["q"], t["k_win"], t["v_win"], t["out"]), flush)
+    fl = plan.info.attention_flops
+    if plan.device_status() != msf.MSF_OK:
+        raise RuntimeError("device status error (chunked)")
+    plan.close()
+    del t
+    wcf = wc.with_scales((1,) * wc.T)
+    plan, t = setup(wcf)
+    plan.kv_resample(t["k_win"], t["v_win"], msf.MSF_RESAMPLE_FULL)
+    fine_ms = _timed(lambda: plan.mssa_forward(t["q"], t["k_win"], t["v_win"], t["out"]), flush,
+                     warm=2, reps=5)
+    fl_fine = plan.info.attention_flops
+    if plan.device_status() != msf.MSF_OK:
+        raise RuntimeError("device status error (chunked, all fine)")
+    plan.close()
+    del t
+    out["chunked_480p"] = {"workload": wc.name, "frames_per_state": wc.frames,
+                           "attention_us": attn_ms * 1e3, "gflop": fl / 1e9,
+                           "tflops": fl / (attn_ms * 1e-3) / 1e12,
+                           "frac": fl / (attn_ms * 1e-3) / 1e12 / bf16,
+                           "pyramid_full_us": pyr_ms * 1e3,
+                           "all_fine_us": fine_ms * 1e3, "all_fine_gflop": fl_fine / 1e9,
+                           "all_fine_tflops": fl_fine / (fine_ms * 1e-3) / 1e12,
+                           "speedup_vs_all_fine": fine_ms / attn_ms}
 
     # ---- streaming rollout: B=4, 120 steps, history 2 -> cap 4, sink fixed
     ws4 = synth.STREAM_480P

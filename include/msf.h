@@ -80,6 +80,13 @@ typedef struct msf_plan_desc {
     int32_t latent_channels;          /* C of the latent (patchify); 0 if unused */
     int32_t patch;                    /* native patch p in latent pixels; 0 if unused */
     int32_t embed_dim;                /* E of the tier projections; 0 = raw tokens only */
+    int32_t frames_per_state;         /* F latent frames per window state (a chunk, Sec. 5.1);
+                                         0 or 1 = one frame. Patches are spatial: each latent
+                                         frame is tokenised and subsampled on its own, a state
+                                         holds F grids in frame order, G = F * grid_h * grid_w,
+                                         history frames and ring slots hold whole chunks and the
+                                         latent of a state is [C, F, Hl, Wl]. grid_h and grid_w
+                                         are one latent frame's and must be divisible by max s_l */
 } msf_plan_desc;
 
 typedef struct msf_group_info {
@@ -95,17 +102,18 @@ typedef struct msf_plan_info {
     int32_t T;
     int32_t n_tokens;                 /* N = N_MSP (Eq. 3) */
     int32_t n_tokens_fine;            /* T * G (all-fine window, N_RF of Eq. 3) */
-    int32_t fine_tokens;              /* G */
+    int32_t fine_tokens;              /* G (tokens of one fine state, all F latent frames) */
     int32_t state_offset[MSF_MAX_STATES];
     int32_t state_tokens[MSF_MAX_STATES];
-    int32_t state_grid_h[MSF_MAX_STATES];
+    int32_t state_grid_h[MSF_MAX_STATES];  /* rows of the state's grid over all F latent
+                                              frames: F * grid_h / s_l */
     int32_t state_grid_w[MSF_MAX_STATES];
     int32_t n_groups;
     msf_group_info groups[MSF_MAX_GROUPS];
     int32_t history_count;            /* live frames in the history ring */
     int32_t history_next_slot;        /* slot the next msf_history_append writes */
     int32_t pyramid_tokens;           /* tokens per stream in the workspace pyramid */
-    int32_t _pad;
+    int32_t frames_per_state;         /* F (1 when desc.frames_per_state is 0) */
     uint64_t workspace_bytes;         /* device workspace msf_plan_bind needs */
     uint64_t attention_flops;         /* 4*D*H*B*sum_g Nq_g*Nkv_g (current history) */
     uint64_t dense_flops;             /* same window with every s_l = 1 (no MSP, no MSSA) */
@@ -143,7 +151,9 @@ msf_status msf_plan_query(msf_plan_t plan, msf_plan_info* info);
  * states 1..T). Each row is 5 int32: kind (0 sink, 1 history, 2 window),
  * frame (history slot or window position, 0-based), stride (the Subsample
  * stride applied to that frame), row, col (on the pooled grid; for the sink
- * row = sink token, col = 0). Writes at most `cap_rows` rows to `out` (host
+ * row = sink token, col = 0). With F latent frames per state the rows of
+ * latent frame f follow those of frame f-1: row = f * (pooled rows of one
+ * frame) + i. Writes at most `cap_rows` rows to `out` (host
  * memory, may be NULL when cap_rows is 0) and sets *n_rows to the total.
  * Host only. */
 msf_status msf_plan_index_map(msf_plan_t plan, int32_t group, int32_t* out, size_t cap_rows,

@@ -291,7 +291,7 @@ static msf::MspShape msp_shape(const Plan& p) {
     sh.T = p.T;
     sh.C = p.d.latent_channels;
     sh.patch = p.d.patch;
-    sh.Hl = p.d.grid_h * p.d.patch;
+    sh.Hl = p.gh * p.d.patch;  // F latent frames stacked: [C, F, Hl, Wl] = [C, F*Hl, Wl]
     sh.Wl = p.d.grid_w * p.d.patch;
     for (int l = 0; l < p.T; ++l) sh.scales[l] = p.d.scales[l];
     return sh;

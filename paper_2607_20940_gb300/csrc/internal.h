@@ -23,6 +23,8 @@ struct Group {
 struct msf_plan {
     msf_plan_desc d;
     int T, G, N, H, D, B;
+    int F;   // latent frames per state
+    int gh;  // rows of a fine state's grid: F latent frames stacked (F * grid_h)
     int elem;  // bytes per element
     int st_off[MSF_MAX_STATES], st_n[MSF_MAX_STATES];
     int st_gh[MSF_MAX_STATES], st_gw[MSF_MAX_STATES];
@@ -64,7 +66,7 @@ inline size_t pyramid_bytes(const Plan& p) {
 // Raw MSP tokens of every state: [B, T, C*Hl*Wl].
 inline size_t msp_scratch_bytes(const Plan& p) {
     if (p.d.latent_channels <= 0 || p.d.patch <= 0) return 0;
-    size_t per = (size_t)p.d.latent_channels * p.d.patch * p.d.grid_h * p.d.patch * p.d.grid_w;
+    size_t per = (size_t)p.d.latent_channels * p.d.patch * p.gh * p.d.patch * p.d.grid_w;
     return round256((size_t)p.B * p.T * per * p.elem);
 }
 // Tensor-core attention (bf16 plans): one merge counter per query block, and
@@ -83,7 +85,7 @@ inline size_t attn_partial_bytes(const Plan& p) {
 constexpr int kMaxDeembedSplits = 8;
 inline size_t msp_split_bytes(const Plan& p) {
     if (p.d.latent_channels <= 0 || p.d.patch <= 0 || p.elem != 2) return 0;
-    size_t per = (size_t)p.d.latent_channels * p.d.patch * p.d.grid_h * p.d.patch * p.d.grid_w;
+    size_t per = (size_t)p.d.latent_channels * p.d.patch * p.gh * p.d.patch * p.d.grid_w;
     return round256((size_t)kMaxDeembedSplits * p.B * per * 4);
 }
 inline size_t workspace_bytes(const Plan& p) {

@@ -75,7 +75,7 @@ extern "C" msf_status msf_unpatchify_noalloc(msf_plan_t plan, int32_t position, 
     sh.T = p.T;
     sh.C = p.d.latent_channels;
     sh.patch = p.d.patch;
-    sh.Hl = p.d.grid_h * p.d.patch;
+    sh.Hl = p.gh * p.d.patch;  // F latent frames stacked: [C, F, Hl, Wl] = [C, F*Hl, Wl]
     sh.Wl = p.d.grid_w * p.d.patch;
     for (int l = 0; l < p.T; ++l) sh.scales[l] = p.d.scales[l];
     const size_t per = (size_t)sh.C * sh.Hl * sh.Wl;  // elements per stream and state

@@ -50,7 +50,13 @@ extern "C" msf_status msf_plan_create(const msf_plan_desc* desc, msf_plan_t* out
         return MSF_ERR_INVALID_ARG;
     if (d.head_dim != 64 && d.head_dim != 128) return MSF_ERR_UNSUPPORTED;
     if (d.softmax_scale < 0.f || !isfinite(d.softmax_scale)) return MSF_ERR_INVALID_ARG;
-    if (d.latent_channels < 0 || d.patch < 0 || d.embed_dim < 0) return MSF_ERR_INVALID_ARG;
+    if (d.latent_channels < 0 || d.patch < 0 || d.embed_dim < 0 || d.frames_per_state < 0)
+        return MSF_ERR_INVALID_ARG;
+    // Chunked states (Sec. 5.1): F latent frames per state, patches and
+    // Subsample spatial. Since every stride divides one frame's grid_h, no
+    // patch or pooling block crosses a frame boundary, so a chunk is handled
+    // as one grid of F * grid_h rows (frames stacked in order).
+    const int F = d.frames_per_state > 0 ? d.frames_per_state : 1;
     // Sec. 4.1: p_l in {p, 2p, 4p, ...}, p_1 <= ... <= p_T.
     int smax = 1;
     for (int l = 0; l < d.T; ++l) {
@@ -61,7 +67,7 @@ extern "C" msf_status msf_plan_create(const msf_plan_desc* desc, msf_plan_t* out
     if (d.grid_h % smax || d.grid_w % smax) return MSF_ERR_UNSUPPORTED;
     // Index arithmetic in the kernels is 32-bit per stream; keep every
     // per-stream element count well inside that range.
-    long long G = (long long)d.grid_h * d.grid_w;
+    long long G = (long long)F * d.grid_h * d.grid_w;
     long long row = (long long)d.heads * d.head_dim;
     if (G * row * (d.T + d.history_capacity + 8) > (1LL << 31)) return MSF_ERR_UNSUPPORTED;
     if ((long long)d.sink_tokens * row > (1LL << 31)) return MSF_ERR_UNSUPPORTED;
@@ -70,6 +76,8 @@ extern "C" msf_status msf_plan_create(const msf_plan_desc* desc, msf_plan_t* out
     if (!p) return MSF_ERR_INVALID_ARG;
     memset((void*)p, 0, sizeof(Plan));
     p->d = d;
+    p->F = F;
+    p->gh = F * d.grid_h;
     p->T = d.T;
     p->G = (int)G;
     p->H = d.heads;
@@ -82,7 +90,7 @@ extern "C" msf_status msf_plan_create(const msf_plan_desc* desc, msf_plan_t* out
     int acc = 0;
     for (int l = 0; l < d.T; ++l) {
         int s = d.scales[l];
-        p->st_gh[l] = d.grid_h / s;
+        p->st_gh[l] = p->gh / s;
         p->st_gw[l] = d.grid_w / s;
         p->st_n[l] = p->st_gh[l] * p->st_gw[l];
         p->st_off[l] = acc;
@@ -198,6 +206,7 @@ extern "C" msf_status msf_plan_query(msf_plan_t plan, msf_plan_info* info) {
     info->history_next_slot =
         p.hist_count < p.d.history_capacity ? p.hist_count : p.hist_oldest;
     info->pyramid_tokens = p.pyr_tokens;
+    info->frames_per_state = p.F;
     info->workspace_bytes = p.ws_bytes;
     info->attention_flops = flops_for(p);
     // Dense reference: every state fine, every query sees sink + history + T*G.
@@ -241,7 +250,7 @@ extern "C" msf_status msf_plan_index_map(msf_plan_t plan, int32_t group, int32_t
     };
     for (int t = 0; t < p.d.sink_tokens; ++t) put(0, 0, 1, t, 0);
     for (int f = 0; f < p.hist_count; ++f)
-        for (int i = 0; i < p.d.grid_h / g; ++i)
+        for (int i = 0; i < p.gh / g; ++i)
             for (int j = 0; j < p.d.grid_w / g; ++j) put(1, f, g, i, j);
     for (int l = 0; l < p.T; ++l) {
         int s = p.d.scales[l];

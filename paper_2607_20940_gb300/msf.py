@@ -48,6 +48,7 @@ class msf_plan_desc(ctypes.Structure):
         ("batch", ctypes.c_int32), ("dtype", ctypes.c_int32), ("resample", ctypes.c_int32),
         ("softmax_scale", ctypes.c_float), ("latent_channels", ctypes.c_int32),
         ("patch", ctypes.c_int32), ("embed_dim", ctypes.c_int32),
+        ("frames_per_state", ctypes.c_int32),
     ]
 
 
@@ -66,7 +67,7 @@ class msf_plan_info(ctypes.Structure):
         ("state_grid_w", ctypes.c_int32 * MSF_MAX_STATES),
         ("n_groups", ctypes.c_int32), ("groups", msf_group_info * MSF_MAX_GROUPS),
         ("history_count", ctypes.c_int32), ("history_next_slot", ctypes.c_int32),
-        ("pyramid_tokens", ctypes.c_int32), ("_pad", ctypes.c_int32),
+        ("pyramid_tokens", ctypes.c_int32), ("frames_per_state", ctypes.c_int32),
         ("workspace_bytes", ctypes.c_uint64), ("attention_flops", ctypes.c_uint64),
         ("dense_flops", ctypes.c_uint64), ("resample_bytes", ctypes.c_uint64),
         ("pyramid_k_offset", ctypes.c_uint64), ("pyramid_v_offset", ctypes.c_uint64),
@@ -228,7 +229,8 @@ def msf_kernel_launches() -> int:
 
 def make_desc(scales, grid_h, grid_w, heads, head_dim, sink_tokens, history_frames,
               history_capacity=None, batch=1, dtype=MSF_DTYPE_BF16, resample=MSF_RESAMPLE_AVG,
-              softmax_scale=0.0, latent_channels=0, patch=0, embed_dim=0) -> msf_plan_desc:
+              softmax_scale=0.0, latent_channels=0, patch=0, embed_dim=0,
+              frames_per_state=1) -> msf_plan_desc:
     d = msf_plan_desc()
     d.T = len(scales)
     for i, s in enumerate(scales):
@@ -238,6 +240,7 @@ def make_desc(scales, grid_h, grid_w, heads, head_dim, sink_tokens, history_fram
     d.history_capacity = history_frames if history_capacity is None else history_capacity
     d.batch, d.dtype, d.resample, d.softmax_scale = batch, dtype, resample, softmax_scale
     d.latent_channels, d.patch, d.embed_dim = latent_channels, patch, embed_dim
+    d.frames_per_state = frames_per_state
     return d
 
 

@@ -44,10 +44,11 @@ class Workload:
     latent_channels: int = 16
     patch: int = 2
     embed_dim: int = 0
+    frames: int = 1   # latent frames per window state (a chunk)
 
     @property
     def fine_tokens(self) -> int:
-        return self.grid_h * self.grid_w
+        return self.frames * self.grid_h * self.grid_w
 
     def with_scales(self, scales: Sequence[int]) -> "Workload":
         return dataclasses.replace(self, scales=tuple(scales))
@@ -69,7 +70,17 @@ THREE_SCALE = Workload("mssa_3scale_t6_48x80_h16_d128", 6, (1, 1, 2, 2, 4, 4), 4
 STREAM_480P = dataclasses.replace(LAYER_480P, name="stream_480p_b4_cap4_120_steps", batch=4,
                                   history_capacity=4, seed=4, steps=120)
 
-WORKLOADS = {w.name: w for w in (TINY, LAYER_480P, PASS_480P, THREE_SCALE, STREAM_480P)}
+# The paper's own window layout (Sec. 5.1): every state a chunk of 3 latent
+# frames (4680 fine tokens at 480p), sink = one chunk, one history chunk.
+CHUNKED_480P = dataclasses.replace(LAYER_480P, name="mssa_480p_chunk3_t5_30x52_h12_d128",
+                                   frames=3, sink_tokens=3 * 1560, history_frames=1,
+                                   history_capacity=1, seed=5)
+# Small chunked case for element-wise parity: 2 frames per state, 8x12 grid.
+CHUNKED_SMALL = Workload("chunk2_t3_8x12_h2_d128", 3, (1, 2, 4), 8, 12, 2, 128, 70, 1, 2, 1, 6,
+                         patch=2, latent_channels=16, embed_dim=256, frames=2)
+
+WORKLOADS = {w.name: w for w in (TINY, LAYER_480P, PASS_480P, THREE_SCALE, STREAM_480P,
+                                 CHUNKED_480P, CHUNKED_SMALL)}
 
 
 def _randn(gen: torch.Generator, shape, std: float, dtype: torch.dtype) -> torch.Tensor:
@@ -81,7 +92,7 @@ def _randn(gen: torch.Generator, shape, std: float, dtype: torch.dtype) -> torch
 
 def window_tokens(w: Workload) -> int:
     """Sum of per-state grid sizes; plain shape bookkeeping for allocation."""
-    return sum((w.grid_h // s) * (w.grid_w // s) for s in w.scales)
+    return sum(w.frames * (w.grid_h // s) * (w.grid_w // s) for s in w.scales)
 
 
 def attention_inputs(w: Workload, dtype: torch.dtype = torch.bfloat16, seed: Optional[int] = None,
@@ -125,7 +136,8 @@ def msp_inputs(w: Workload, dtype: torch.dtype = torch.bfloat16, seed: Optional[
                embed_dim: Optional[int] = None) -> dict:
     """Latent window and seeded random tier projections for patchify/unpatchify.
 
-    latent ``[B, T, C, Hl, Wl]`` ~ N(0,1); for each distinct scale s a tier
+    latent ``[B, T, C, Hl, Wl]`` (``[B, T, C, F, Hl, Wl]`` for chunks of F > 1
+    latent frames) ~ N(0,1); for each distinct scale s a tier
     projection ``[C*(patch*s)^2, E]`` ~ N(0, 1/(C*(patch*s)^2)); the fine
     de-embedding ``[E, C*patch^2]`` ~ N(0, 1/E). With ``embed_dim`` 0 only
     the latent is drawn.
@@ -135,7 +147,8 @@ def msp_inputs(w: Workload, dtype: torch.dtype = torch.bfloat16, seed: Optional[
     gen = torch.Generator().manual_seed(seed)
     C, P = w.latent_channels, w.patch
     Hl, Wl = w.grid_h * P, w.grid_w * P
-    out = {"latent": _randn(gen, (w.batch, w.T, C, Hl, Wl), 1.0, dtype)}
+    lat = (w.batch, w.T, C, Hl, Wl) if w.frames == 1 else (w.batch, w.T, C, w.frames, Hl, Wl)
+    out = {"latent": _randn(gen, lat, 1.0, dtype)}
     if E:
         tiers = {}
         for s in sorted(set(w.scales)):

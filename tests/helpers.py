@@ -24,7 +24,7 @@ def make_plan(w: synth.Workload, dtype=BF16, resample=0, history_capacity=None, 
                        history_capacity=w.history_capacity if history_capacity is None else history_capacity,
                        batch=w.batch, dtype=m.MSF_DTYPE_BF16 if dtype == BF16 else m.MSF_DTYPE_F32,
                        resample=resample, latent_channels=w.latent_channels, patch=w.patch,
-                       embed_dim=w.embed_dim if embed else 0)
+                       embed_dim=w.embed_dim if embed else 0, frames_per_state=w.frames)
     return m.Plan(desc)
 
 
@@ -50,7 +50,7 @@ def oracle_mssa(x: dict, w: synth.Workload, mode=0, heads=None):
     f = synth.to_f64
     return omssa.mssa_forward(f(x["q"]), f(x["k_win"]), f(x["v_win"]), f(x["k_sink"]),
                               f(x["v_sink"]), f(x["k_hist"]), f(x["v_hist"]), w.scales,
-                              w.grid_h, w.grid_w, mode=mode, heads=heads)
+                              w.grid_h, w.grid_w, mode=mode, heads=heads, frames=w.frames)
 
 
 def err_stats(got: torch.Tensor, ref: np.ndarray, heads=None):

@@ -40,9 +40,10 @@ def test_library_exports_every_declared_symbol():
     assert declared == set(msf.EXPORTS)
 
 
-def _plan(scales, gh, gw, ns, nh, cap=None, H=2, D=64, B=1):
+def _plan(scales, gh, gw, ns, nh, cap=None, H=2, D=64, B=1, F=1):
     msf = _msf()
-    return msf.Plan(msf.make_desc(scales, gh, gw, H, D, ns, nh, history_capacity=cap, batch=B))
+    return msf.Plan(msf.make_desc(scales, gh, gw, H, D, ns, nh, history_capacity=cap, batch=B,
+                                  frames_per_state=F))
 
 
 CASES = [
@@ -55,28 +56,33 @@ CASES = [
 ]
 
 
+@pytest.mark.parametrize("F", [1, 3])
 @pytest.mark.parametrize("scales,gh,gw,ns,nh", CASES)
-def test_plan_tables_match_oracle(scales, gh, gw, ns, nh):
-    p = _plan(scales, gh, gw, ns, nh)
+def test_plan_tables_match_oracle(scales, gh, gw, ns, nh, F):
+    if F > 1 and gh * gw > 2000:
+        pytest.skip("chunked variant checked on the smaller grids")
+    p = _plan(scales, gh, gw, ns, nh, F=F)
     info = p.info
-    cnt = schedule.token_counts(scales, gh, gw)
-    offs = schedule.token_offsets(scales, gh, gw)
+    cnt = schedule.token_counts(scales, gh, gw, F)
+    offs = schedule.token_offsets(scales, gh, gw, F)
+    assert info.frames_per_state == F
     assert info.n_tokens == sum(cnt)
-    assert info.n_tokens_fine == len(scales) * gh * gw
+    assert info.n_tokens_fine == len(scales) * F * gh * gw
     assert list(info.state_tokens[:len(scales)]) == cnt
     assert list(info.state_offset[:len(scales)]) == offs
-    groups = schedule.query_groups(scales, gh, gw)
+    groups = schedule.query_groups(scales, gh, gw, F)
     assert info.n_groups == len(groups)
     for gi, g in enumerate(groups):
         gi_ = info.groups[gi]
         assert (gi_.scale, gi_.q_begin, gi_.q_end) == (g.scale, g.q_begin, g.q_end)
-        rows = schedule.context_rows(scales, gh, gw, ns, nh, g.scale)
+        rows = schedule.context_rows(scales, gh, gw, ns, nh, g.scale, F)
         assert gi_.n_kv == len(rows)
         got = p.index_map(gi)
         want = np.array(rows, dtype=np.int32).reshape(-1, 5)
         assert got.shape == want.shape
         assert np.array_equal(got, want)
-    assert info.attention_flops == schedule.attention_flops(scales, gh, gw, ns, nh, 2, 64)
+    assert info.attention_flops == schedule.attention_flops(scales, gh, gw, ns, nh, 2, 64,
+                                                            frames=F)
 
 
 def test_plan_tables_random_schedules():
@@ -102,17 +108,32 @@ def test_480p_numbers():
     assert info.resample_bytes == 2 * 4 * (1560 + 390) * 12 * 128 * 2
 
 
+def test_chunked_480p_numbers():
+    """The paper's layout (Sec. 5.1): 3 latent frames per state, sink = one
+    chunk, one history chunk; every count is the per-frame one times 3."""
+    w = synth.CHUNKED_480P
+    info = _plan(w.scales, 30, 52, w.sink_tokens, 1, H=12, D=128, F=3).info
+    assert info.fine_tokens == 4680 and info.n_tokens == 12870 and info.n_tokens_fine == 23400
+    assert [info.groups[i].n_kv for i in range(2)] == [4680 + 4680 + 12870,
+                                                      4680 + 1170 + 2 * 1170 + 3 * 1170]
+    assert info.attention_flops == 4 * 128 * 12 * (9360 * 22230 + 3510 * 11700)
+    assert list(info.state_grid_h[:5]) == [90, 90, 45, 45, 45]
+
+
 @pytest.mark.parametrize("bad", [
     dict(scales=(1, 2, 1)), dict(scales=(1, 3)), dict(scales=(1, 4), gh=30),
-    dict(D=96), dict(H=0), dict(nh=3, cap=2),
+    dict(D=96), dict(H=0), dict(nh=3, cap=2), dict(F=-1),
+    # one latent frame's grid must take the coarsest stride, even when the
+    # stacked chunk (F * gh rows) would
+    dict(scales=(1, 4), gh=2, F=2),
 ])
 def test_plan_validation(bad):
     msf = _msf()
-    args = dict(scales=(1, 2), gh=8, gw=8, ns=4, nh=1, cap=None, H=2, D=64)
+    args = dict(scales=(1, 2), gh=8, gw=8, ns=4, nh=1, cap=None, H=2, D=64, F=1)
     args.update(bad)
     with pytest.raises(msf.MsfError) as ei:
         _plan(args["scales"], args["gh"], args["gw"], args["ns"], args["nh"], cap=args["cap"],
-              H=args["H"], D=args["D"])
+              H=args["H"], D=args["D"], F=args["F"])
     assert ei.value.status in (msf.MSF_ERR_INVALID_ARG, msf.MSF_ERR_UNSUPPORTED)
 
 
