@@ -4,10 +4,12 @@ A step is one rolling-window pass of the whole hot path at the 480p layer
 shapes (T=5, 30x52 fine grid, scales (1,1,2,2,2), 12 heads of 128, sink 1560
 tokens, history ring of 2 frames):
   MSP patchify + tier embedding of the 5 latent states (16x60x104 -> 4290x1536)
-  -> window part of the K/V pyramid -> MSSA attention (Eq. 4)
-  -> de-embed + unpatchify of the head state -> history append (head K/V).
-The K/V pyramid runs on a second stream beside the embedding, and the history
-append beside the de-embedding; attention waits for both of its inputs.
+  -> window part of the K/V pyramid, with the head's K/V staged in the history
+     ring's spare slot and pooled (the history update, folded into that launch)
+  -> MSSA attention (Eq. 4) -> history commit (host) -> de-embed + unpatchify
+     of the head state.
+The K/V pyramid runs on a second stream beside the embedding; attention waits
+for both of its inputs.
 `value` is the MSSA FLOPs the schedule requires (4*D*H*sum_g Nq_g*Nkv_g =
 202.79 GFLOP) divided by the device time of the whole step, in TFLOP/s.
 Inputs are resident in HBM; the L2 is flushed (a 256 MiB write) between
@@ -230,17 +232,18 @@ def other_configs(msf, synth, dev, flush, peaks, rank):
     def rnd(shape):
         return torch.randn(shape, generator=gen, device=dev, dtype=torch.float32).to(torch.bfloat16)
 
-    def setup(w, embed=False):
+    def setup(w, embed=False, fused=False):
         plan = msf.Plan(msf.make_desc(w.scales, w.grid_h, w.grid_w, w.heads, w.head_dim, w.sink_tokens,
                                       w.history_frames, w.history_capacity, batch=w.batch,
                                       latent_channels=w.latent_channels, patch=w.patch,
                                       embed_dim=w.embed_dim if embed else 0,
-                                      frames_per_state=w.frames))
+                                      frames_per_state=w.frames, fused_append=int(fused)))
         N, G, H, D, B = plan.info.n_tokens, w.fine_tokens, w.heads, w.head_dim, w.batch
         t = {k: rnd((B, N, H, D)) for k in ("q", "k_win", "v_win")}
         t["k_sink"], t["v_sink"] = rnd((B, w.sink_tokens, H, D)), rnd((B, w.sink_tokens, H, D))
         for k in ("k_hist", "v_hist"):
-            ring = torch.zeros((B, max(w.history_capacity, 1), G, H, D), dtype=torch.bfloat16, device=dev)
+            slots = w.history_capacity + 1 if fused else max(w.history_capacity, 1)
+            ring = torch.zeros((B, slots, G, H, D), dtype=torch.bfloat16, device=dev)
             ring[:, :w.history_frames] = rnd((B, w.history_frames, G, H, D))
             t[k] = ring
         ws = plan.workspace(dev)
@@ -293,40 +296,55 @@ def other_configs(msf, synth, dev, flush, peaks, rank):
                            "all_fine_tflops": fl_fine / (fine_ms * 1e-3) / 1e12,
                            "speedup_vs_all_fine": fine_ms / attn_ms}
 
-    # ---- streaming rollout: B=4, 120 steps, history 2 -> cap 4, sink fixed
+    # ---- streaming rollout: B=4, 120 steps, history 2 -> cap 4, sink fixed.
+    #      Per step: K/V resample -> MSSA -> history update, on one stream;
+    #      the update fused into the resample (spare ring slot + host commit),
+    #      and, for comparison, as its own launch after the attention.
     ws4 = synth.STREAM_480P
-    plan, t = setup(ws4)
-    sets = [{k: rnd(t[k].shape) for k in ("q", "k_win", "v_win")} for _ in range(4)]
-    plan.kv_resample(t["k_win"], t["v_win"], msf.MSF_RESAMPLE_FULL)
-    step_ev, attn_ev, fl_steps = [], [], 0.0
-    torch.cuda.synchronize()
-    for i in range(ws4.steps):
-        x = sets[i % len(sets)]
-        e0, e1, e2, e3 = (torch.cuda.Event(enable_timing=True) for _ in range(4))
-        e0.record()
-        plan.kv_resample(x["k_win"], x["v_win"], msf.MSF_RESAMPLE_WINDOW_ONLY)
-        e1.record()
-        plan.mssa_forward(x["q"], x["k_win"], x["v_win"], t["out"])
-        e2.record()
-        fl_steps += plan.info.attention_flops
-        plan.history_append(x["k_win"], x["v_win"])
-        e3.record()
-        step_ev.append((e0, e3))
-        attn_ev.append((e1, e2))
-    torch.cuda.synchronize()
-    steps_us = sorted(a.elapsed_time(b) * 1e3 for a, b in step_ev)
-    attn_s = sum(a.elapsed_time(b) for a, b in attn_ev) * 1e-3
-    out["stream_b4"] = {"workload": ws4.name, "steps": ws4.steps, "streams": ws4.batch,
-                        "step_us_p50": steps_us[len(steps_us) // 2],
-                        "step_us_p99": steps_us[min(len(steps_us) - 1, int(0.99 * len(steps_us)))],
-                        "attention_frames_per_s": ws4.batch * ws4.steps / attn_s,
-                        "attention_tflops": fl_steps / attn_s / 1e12,
-                        "history_frames_end": plan.info.history_count,
-                        "note": "steps back to back without an L2 flush (a sustained rollout)"}
-    if plan.device_status() != msf.MSF_OK:
-        raise RuntimeError("device status error (stream)")
-    plan.close()
-    del t, sets
+
+    def rollout(fused):
+        plan, t = setup(ws4, fused=fused)
+        sets = [{k: rnd(t[k].shape) for k in ("q", "k_win", "v_win")} for _ in range(4)]
+        plan.kv_resample(t["k_win"], t["v_win"], msf.MSF_RESAMPLE_FULL)
+        step_ev, attn_ev, fl_steps = [], [], 0.0
+        torch.cuda.synchronize()
+        for i in range(ws4.steps):
+            x = sets[i % len(sets)]
+            e0, e1, e2, e3 = (torch.cuda.Event(enable_timing=True) for _ in range(4))
+            e0.record()
+            plan.kv_resample(x["k_win"], x["v_win"], msf.MSF_RESAMPLE_WINDOW_ONLY)
+            e1.record()
+            plan.mssa_forward(x["q"], x["k_win"], x["v_win"], t["out"])
+            e2.record()
+            fl_steps += plan.info.attention_flops
+            if fused:
+                plan.history_commit()
+            else:
+                plan.history_append(x["k_win"], x["v_win"])
+            e3.record()
+            step_ev.append((e0, e3))
+            attn_ev.append((e1, e2))
+        torch.cuda.synchronize()
+        if plan.device_status() != msf.MSF_OK:
+            raise RuntimeError("device status error (stream)")
+        steps_us = sorted(a.elapsed_time(b) * 1e3 for a, b in step_ev)
+        attn_s = sum(a.elapsed_time(b) for a, b in attn_ev) * 1e-3
+        res = {"step_us_p50": steps_us[len(steps_us) // 2],
+               "step_us_p99": steps_us[min(len(steps_us) - 1, int(0.99 * len(steps_us)))],
+               "attention_frames_per_s": ws4.batch * ws4.steps / attn_s,
+               "attention_tflops": fl_steps / attn_s / 1e12,
+               "history_frames_end": plan.info.history_count}
+        plan.close()
+        del t, sets
+        return res
+
+    fused_r = rollout(True)
+    sep_r = rollout(False)
+    out["stream_b4"] = dict({"workload": ws4.name, "steps": ws4.steps, "streams": ws4.batch,
+                             "history_update": "fused into the resample"}, **fused_r)
+    out["stream_b4"]["separate_append"] = {"step_us_p50": sep_r["step_us_p50"],
+                                           "step_us_p99": sep_r["step_us_p99"]}
+    out["stream_b4"]["note"] = "steps back to back without an L2 flush (a sustained rollout)"
 
     # ---- 30-layer window pass at 480p shapes (MSP embed -> pyramid -> MSSA -> de-embed per layer)
     wp = synth.PASS_480P
@@ -414,12 +432,20 @@ def main():
     # ------------------------------------------------------------ set-up
     x = synth.attention_inputs(w, torch.bfloat16, seed=w.seed + 1000 * rank)
     mi = synth.msp_inputs(w, torch.bfloat16, seed=w.seed + 1000 * rank)
+    # The history update is fused into the K/V resample: the ring has one
+    # spare slot, the resample stages the head there (copy and pooled levels
+    # from one read) and a host-side commit makes it a history frame.
     plan = msf.Plan(msf.make_desc(w.scales, w.grid_h, w.grid_w, w.heads, w.head_dim,
                                   w.sink_tokens, w.history_frames, w.history_capacity,
                                   batch=w.batch, latent_channels=w.latent_channels, patch=w.patch,
-                                  embed_dim=w.embed_dim))
+                                  embed_dim=w.embed_dim, fused_append=1))
     info = plan.info
-    d = {k: v.to(dev) for k, v in x.items()}
+    d = {k: v.to(dev) for k, v in x.items() if k not in ("k_hist", "v_hist")}
+    for k in ("k_hist", "v_hist"):
+        ring = torch.zeros((w.batch, w.history_capacity + 1) + tuple(x[k].shape[2:]),
+                           dtype=x[k].dtype, device=dev)
+        ring[:, :w.history_frames] = x[k].to(dev)
+        d[k] = ring
     ws = plan.workspace(dev)
     plan.bind(ws, d["k_sink"], d["v_sink"], d["k_hist"], d["v_hist"])
     lat = mi["latent"].to(dev)
@@ -438,9 +464,11 @@ def main():
     side = torch.cuda.Stream(device=dev)
 
     def step(q, k, v, latent, timed_attn=False):
-        # Two streams: the K/V pyramid runs beside the MSP embedding of the
-        # window, and the history update beside the de-embedding of the head
-        # state. Attention waits for both of its inputs.
+        # Two streams: the K/V pyramid (with the staged history head) runs
+        # beside the MSP embedding of the window; attention waits for both of
+        # its inputs, then the head is committed to the history (host only)
+        # and de-embedded. The next step's resample, which overwrites the new
+        # spare slot, forks from the main stream after this attention.
         fork = torch.cuda.Event()
         fork.record(stream)
         side.wait_event(fork)
@@ -457,14 +485,8 @@ def main():
         if timed_attn:
             a1.record(stream)
             ev_a.append((a0, a1))
-        attended = torch.cuda.Event()
-        attended.record(stream)
-        side.wait_event(attended)
-        plan.history_append(k, v, stream=side)
+        plan.history_commit()
         plan.unpatchify(0, out.view(w.batch, N, E), w_out, lat_out, stream=stream)
-        joined = torch.cuda.Event()
-        joined.record(side)
-        stream.wait_event(joined)
 
     plan.kv_resample(d["k_win"], d["v_win"], msf.MSF_RESAMPLE_FULL)
     for _ in range(args.warmup):
@@ -592,7 +614,8 @@ def main():
         "config": {
             "workload": w.name, "T": w.T, "scales": list(w.scales), "grid": [w.grid_h, w.grid_w],
             "heads": w.heads, "head_dim": w.head_dim, "sink_tokens": w.sink_tokens,
-            "history_frames": w.history_frames, "batch_per_gpu": w.batch,
+            "history_frames": w.history_frames, "history_update": "fused into the resample",
+            "batch_per_gpu": w.batch,
             "latent": [w.latent_channels, w.grid_h * w.patch, w.grid_w * w.patch],
             "embed_dim": w.embed_dim, "attention_gflop": flops / 1e9,
             "us_per_layer": ms_per_step * 1e3, "l2": "flushed between steps (256 MiB write)",

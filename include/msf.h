@@ -87,6 +87,15 @@ typedef struct msf_plan_desc {
                                          history frames and ring slots hold whole chunks and the
                                          latent of a state is [C, F, Hl, Wl]. grid_h and grid_w
                                          are one latent frame's and must be divisible by max s_l */
+    int32_t fused_append;             /* 0: the history update is its own launch
+                                         (msf_history_append). 1: it is folded into
+                                         msf_kv_resample: the ring has capacity + 1 slots,
+                                         every resample copies the head state (position 1)
+                                         into the spare slot and pools it there at every
+                                         coarser level from the same read, attention reads
+                                         the head from that slot, and msf_history_commit
+                                         (host only, no launch) makes it a history frame.
+                                         Needs s_1 = 1 and capacity >= 1 */
 } msf_plan_desc;
 
 typedef struct msf_group_info {
@@ -111,7 +120,8 @@ typedef struct msf_plan_info {
     int32_t n_groups;
     msf_group_info groups[MSF_MAX_GROUPS];
     int32_t history_count;            /* live frames in the history ring */
-    int32_t history_next_slot;        /* slot the next msf_history_append writes */
+    int32_t history_next_slot;        /* slot the next msf_history_append writes (with
+                                         fused_append: the spare slot the head is staged in) */
     int32_t pyramid_tokens;           /* tokens per stream in the workspace pyramid */
     int32_t frames_per_state;         /* F (1 when desc.frames_per_state is 0) */
     uint64_t workspace_bytes;         /* device workspace msf_plan_bind needs */
@@ -153,7 +163,11 @@ msf_status msf_plan_query(msf_plan_t plan, msf_plan_info* info);
  * stride applied to that frame), row, col (on the pooled grid; for the sink
  * row = sink token, col = 0). With F latent frames per state the rows of
  * latent frame f follow those of frame f-1: row = f * (pooled rows of one
- * frame) + i. Writes at most `cap_rows` rows to `out` (host
+ * frame) + i. With fused_append the same rows come in the kernels' order:
+ * sink; for g > 1 the pooled window states 2..n_finer; then ring slots
+ * 0..count in slot order (live frames as history rows, the spare slot as
+ * window position 0); then the window states the kernel reads from k_win
+ * (from position 1 for g = 1, from the group's first state for g > 1). Writes at most `cap_rows` rows to `out` (host
  * memory, may be NULL when cap_rows is 0) and sets *n_rows to the total.
  * Host only. */
 msf_status msf_plan_index_map(msf_plan_t plan, int32_t group, int32_t* out, size_t cap_rows,
@@ -164,6 +178,8 @@ msf_status msf_plan_index_map(msf_plan_t plan, int32_t group, int32_t* out, size
  *   k_sink, v_sink [B, Ns, H, D]           (read only, never resampled)
  *   k_hist, v_hist [B, capacity, G, H, D]  history ring, fine scale; the first
  *                                          history_frames slots hold live frames
+ *                                          ([B, capacity + 1, G, H, D] with
+ *                                          fused_append: one spare slot)
  * Resets the history count to desc.history_frames and zeroes the device status
  * word (a cudaMemsetAsync on the legacy stream, completed before returning).
  * Builds the TMA descriptors for the bound buffers. Errors: INVALID_ARG,
@@ -201,8 +217,10 @@ msf_status msf_unpatchify(msf_plan_t plan, int32_t position, const void* tokens,
  * group g > 1, the bound history frames (fine, pooled by g) and the window
  * states with s_l < g (pooled by g/s_l), from k_win, v_win [B, N, H, D].
  * Pooling is the plan's Subsample mode; AVG sums in fp32 and rounds once.
- * flags: MSF_RESAMPLE_FULL or MSF_RESAMPLE_WINDOW_ONLY. Errors: INVALID_ARG,
- * STATE (not bound), CUDA. */
+ * flags: MSF_RESAMPLE_FULL or MSF_RESAMPLE_WINDOW_ONLY. With fused_append the
+ * same launch also stages the head state (tokens [0, G) of k_win/v_win) in
+ * the ring's spare slot and its pyramid levels (one read of the head for the
+ * copy and the pooling). Errors: INVALID_ARG, STATE (not bound), CUDA. */
 msf_status msf_kv_resample(msf_plan_t plan, const void* k_win, const void* v_win, int32_t flags,
                            void* stream);
 
@@ -225,10 +243,20 @@ msf_status msf_mssa_forward_simt(msf_plan_t plan, const void* q, const void* k_w
  * K/V (window position 0, tokens [0, G)) into the ring slot
  * info.history_next_slot (the next free slot, else the oldest frame), and
  * pool it into that slot of every coarser pyramid level. Advances the
- * host-side count/slot state. Errors: STATE (not bound, capacity 0, or
- * s_1 != 1), INVALID_ARG, CUDA. */
+ * host-side count/slot state. Errors: STATE (not bound, capacity 0, s_1 != 1,
+ * or a fused_append plan), INVALID_ARG, CUDA. */
 msf_status msf_history_append(msf_plan_t plan, const void* k_win, const void* v_win,
                               void* stream);
+
+/* History-cache update of a fused_append plan (Algorithm 1's KV update): the
+ * head staged by the last msf_kv_resample becomes the newest history frame.
+ * While the ring holds fewer than `capacity` frames the next spare slot is the
+ * next free one; once it is full the oldest frame's slot becomes the spare
+ * (evicted). Host only: no launch, no device access; call it after the
+ * pass's msf_mssa_forward has been enqueued (the next resample overwrites the
+ * new spare slot, stream order keeps that after this pass's reads).
+ * Errors: INVALID_ARG, STATE (not bound, or not a fused_append plan). */
+msf_status msf_history_commit(msf_plan_t plan);
 
 /* Number of kernels this library has launched in this process (all plans,
  * all devices), for accounting in benchmarks. Host only. */

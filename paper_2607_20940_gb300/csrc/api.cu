@@ -30,48 +30,72 @@ void add_window_jobs(const Plan& p, const void* k_win, const void* v_win, bool w
                      msf::PoolBatch& jb) {
     const size_t row = row_bytes(p);
     const long long win_bs = (long long)p.N * row;
-    const long long hist_bs = (long long)p.d.history_capacity * p.G * row;
+    const long long hist_bs = (long long)p.ring_slots * p.G * row;
     const long long pyr_bs = (long long)p.pyr_tokens * row;
+    auto job = [&](const char* sk, const char* sv, long long sbs, char* dk, char* dv,
+                   int src_gw, int out_gw, int out_n, int sigma) -> msf::PoolJob& {
+        msf::PoolJob& j = jb.j[jb.n++];
+        j.src_k = sk;
+        j.src_v = sv;
+        j.dst_k = dk;
+        j.dst_v = dv;
+        j.src_bstride = sbs;
+        j.dst_bstride = pyr_bs;
+        j.src_gw = src_gw;
+        j.out_gw = out_gw;
+        j.out_n = out_n;
+        j.sigma = sigma;
+        return j;
+    };
+    // With fused_append the pyramid part of g is [finer states 2.. | ring slots]
+    // and the head (state 1) is staged in the ring's spare slot.
+    bool head_copied = false;
     for (int gi = 0; gi < p.n_groups; ++gi) {
         const msf::Group& g = p.groups[gi];
         if (g.scale == 1) continue;
+        const int ring0 = p.fused ? g.n_finer - 1 : 0;  // pyramid slot of ring slot 0
         if (with_history) {
-            for (int f = 0; f < p.hist_count; ++f) {
-                msf::PoolJob& j = jb.j[jb.n++];
+            for (int f = 0; f < (p.fused ? p.hist_count + 1 : p.hist_count); ++f) {
+                if (p.fused && f == p.hist_spare) continue;
                 size_t so = (size_t)f * p.G * row;
-                size_t dof = (size_t)(g.pyr_offset + f * g.pooled) * row;
-                j.src_k = (const char*)p.k_hist + so;
-                j.src_v = (const char*)p.v_hist + so;
-                j.dst_k = msf::pyr_k(p) + dof;
-                j.dst_v = msf::pyr_v(p) + dof;
-                j.src_bstride = hist_bs;
-                j.dst_bstride = pyr_bs;
-                j.src_gw = p.d.grid_w;
-                j.out_gw = p.d.grid_w / g.scale;
-                j.out_n = g.pooled;
-                j.sigma = g.scale;
+                size_t dof = (size_t)(g.pyr_offset + (ring0 + f) * g.pooled) * row;
+                job((const char*)p.k_hist + so, (const char*)p.v_hist + so, hist_bs,
+                    msf::pyr_k(p) + dof, msf::pyr_v(p) + dof, p.d.grid_w, p.d.grid_w / g.scale,
+                    g.pooled, g.scale);
             }
         }
         for (int l = 0; l < g.n_finer; ++l) {
-            msf::PoolJob& j = jb.j[jb.n++];
+            int slot;  // pyramid slot of this pooled state
+            if (!p.fused)
+                slot = p.hist_count + l;
+            else
+                slot = l == 0 ? ring0 + p.hist_spare : l - 1;
             size_t so = (size_t)p.st_off[l] * row;
-            size_t dof = (size_t)(g.pyr_offset + (p.hist_count + l) * g.pooled) * row;
-            j.src_k = (const char*)k_win + so;
-            j.src_v = (const char*)v_win + so;
-            j.dst_k = msf::pyr_k(p) + dof;
-            j.dst_v = msf::pyr_v(p) + dof;
-            j.src_bstride = win_bs;
-            j.dst_bstride = pyr_bs;
-            j.src_gw = p.st_gw[l];
-            j.out_gw = p.d.grid_w / g.scale;
-            j.out_n = g.pooled;
-            j.sigma = g.scale / p.d.scales[l];
+            size_t dof = (size_t)(g.pyr_offset + slot * g.pooled) * row;
+            msf::PoolJob& j = job((const char*)k_win + so, (const char*)v_win + so, win_bs,
+                                  msf::pyr_k(p) + dof, msf::pyr_v(p) + dof, p.st_gw[l],
+                                  p.d.grid_w / g.scale, g.pooled, g.scale / p.d.scales[l]);
+            if (p.fused && l == 0 && !head_copied && g.scale <= 4) {
+                // the same read also writes the fine head into the spare ring slot
+                const size_t ro = (size_t)p.hist_spare * p.G * row;
+                j.copy_k = (char*)p.k_hist + ro;
+                j.copy_v = (char*)p.v_hist + ro;
+                j.copy_bstride = hist_bs;
+                head_copied = true;
+            }
         }
+    }
+    if (p.fused && !head_copied) {
+        // no coarser level: a plain copy of the head into the spare slot
+        const size_t ro = (size_t)p.hist_spare * p.G * row;
+        msf::PoolJob& j = job((const char*)k_win, (const char*)v_win, win_bs, (char*)p.k_hist + ro,
+                              (char*)p.v_hist + ro, p.d.grid_w, p.d.grid_w, p.G, 1);
+        j.dst_bstride = hist_bs;
     }
 }
 
 int count_window_jobs(const Plan& p, bool with_history) {
-    int n = 0;
+    int n = p.fused ? 1 : 0;
     for (int gi = 0; gi < p.n_groups; ++gi) {
         const msf::Group& g = p.groups[gi];
         if (g.scale == 1) continue;
@@ -111,17 +135,23 @@ void build_attn_args(const Plan& p, const void* q, const void* k_win, const void
             s.rows_total = p.d.sink_tokens;
             s.map_id = msf::kMapSink;
         }
+        // fused_append: the head (state 1) is read from the ring's spare slot,
+        // which sits inside the used slots [0, count]; the window part starts
+        // after it.
+        const int ring_used = p.fused ? p.hist_count + 1 : p.hist_count;
+        int win0 = g.q_begin;
         if (g.scale == 1) {
-            if (p.hist_count > 0) {
+            if (ring_used > 0) {
                 msf::Segment& s = ag.seg[ns++];
                 s.k = (const char*)p.k_hist;
                 s.v = (const char*)p.v_hist;
-                s.bstride = (long long)p.d.history_capacity * p.G * row;
+                s.bstride = (long long)p.ring_slots * p.G * row;
                 s.row0 = 0;
-                s.len = p.hist_count * p.G;
-                s.rows_total = p.d.history_capacity * p.G;
+                s.len = ring_used * p.G;
+                s.rows_total = p.ring_slots * p.G;
                 s.map_id = msf::kMapHist;
             }
+            if (p.fused) win0 = p.st_n[0];
         } else {
             int n = msf::group_npyr(p, gi);
             if (n > 0) {
@@ -135,13 +165,13 @@ void build_attn_args(const Plan& p, const void* q, const void* k_win, const void
                 s.map_id = msf::kMapPyr;
             }
         }
-        {
+        if (win0 < p.N) {
             msf::Segment& s = ag.seg[ns++];
             s.k = (const char*)k_win;
             s.v = (const char*)v_win;
             s.bstride = (long long)p.N * row;
-            s.row0 = g.q_begin;
-            s.len = p.N - g.q_begin;
+            s.row0 = win0;
+            s.len = p.N - win0;
             s.rows_total = p.N;
             s.map_id = msf::kMapWin;
         }
@@ -173,6 +203,7 @@ extern "C" msf_status msf_plan_bind(msf_plan_t plan, void* workspace, size_t wor
     p.v_hist = v_hist;
     p.hist_count = p.d.history_frames;
     p.hist_oldest = 0;
+    p.hist_spare = p.d.history_frames;
     p.bound = true;
     msf::tc_cache_invalidate(plan);
     cudaError_t e = cudaMemset(msf::status_word(p), 0, msf::kStatusBytes);
@@ -203,7 +234,8 @@ extern "C" msf_status msf_history_append(msf_plan_t plan, const void* k_win, con
                                          void* stream) {
     if (!plan || !k_win || !v_win) return MSF_ERR_INVALID_ARG;
     Plan& p = *plan;
-    if (!p.bound || p.d.history_capacity == 0 || p.d.scales[0] != 1) return MSF_ERR_STATE;
+    if (!p.bound || p.d.history_capacity == 0 || p.d.scales[0] != 1 || p.fused)
+        return MSF_ERR_STATE;
     if (!aligned16(k_win) || !aligned16(v_win)) return MSF_ERR_INVALID_ARG;
     const int slot = p.hist_count < p.d.history_capacity ? p.hist_count : p.hist_oldest;
     const size_t row = row_bytes(p);
@@ -248,6 +280,23 @@ extern "C" msf_status msf_history_append(msf_plan_t plan, const void* k_win, con
         ++p.hist_count;
     } else {
         p.hist_oldest = (p.hist_oldest + 1) % p.d.history_capacity;
+    }
+    return MSF_OK;
+}
+
+extern "C" msf_status msf_history_commit(msf_plan_t plan) {
+    if (!plan) return MSF_ERR_INVALID_ARG;
+    Plan& p = *plan;
+    if (!p.bound || !p.fused) return MSF_ERR_STATE;
+    // The staged head joins the live frames (slot order: frames stay where
+    // they were written). Below capacity the next free slot becomes the spare;
+    // at capacity the oldest frame is evicted and its slot becomes the spare.
+    if (p.hist_count < p.d.history_capacity) {
+        ++p.hist_count;
+        p.hist_spare = p.hist_count;
+    } else {
+        p.hist_spare = p.hist_oldest;
+        p.hist_oldest = (p.hist_oldest + 1) % p.ring_slots;
     }
     return MSF_OK;
 }

@@ -23,6 +23,8 @@ struct Group {
 struct msf_plan {
     msf_plan_desc d;
     int T, G, N, H, D, B;
+    bool fused;      // fused_append: history update folded into the resample
+    int ring_slots;  // history ring slots: capacity (+1 spare with fused_append)
     int F;   // latent frames per state
     int gh;  // rows of a fine state's grid: F latent frames stacked (F * grid_h)
     int elem;  // bytes per element
@@ -40,6 +42,7 @@ struct msf_plan {
     // history ring state (host side)
     int hist_count;
     int hist_oldest;
+    int hist_spare;   // fused_append: ring slot the next resample stages the head in
 
     // bound buffers
     bool bound;

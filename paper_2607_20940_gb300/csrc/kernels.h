@@ -62,6 +62,12 @@ struct PoolJob {
     int out_gw;             // pooled grid width
     int out_n;              // pooled tokens
     int sigma;              // stride (1 = copy)
+    // Optional: also write every source token read to this block (same token
+    // index as in the source, so the whole source is copied when the pooled
+    // blocks tile it). NULL = no copy. Requires sigma <= 4.
+    char* copy_k;
+    char* copy_v;
+    long long copy_bstride;
 };
 constexpr int kMaxPoolJobs = 40;
 struct PoolBatch {

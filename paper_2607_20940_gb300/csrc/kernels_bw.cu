@@ -57,12 +57,15 @@ struct Vec<float> {
 
 // Two adjacent 16-byte vectors of one pooled token, K and V. With the stride
 // known at compile time every source load is issued before the first add, so
-// a thread keeps 4*S*S loads in flight.
+// a thread keeps 4*S*S loads in flight. ck/cv (NULL = none) receive a copy of
+// every source vector read, at its source token index (the staged history
+// head: one read serves the ring copy and the pooled level).
 template <typename T, int S>
-__device__ __forceinline__ void pool_pair(const char* sk, const char* sv, char* dk, char* dv, int src_gw,
-                                          int i, int jj, size_t row, int mode) {
+__device__ __forceinline__ void pool_pair(const char* sk, const char* sv, char* dk, char* dv,
+                                          char* ck, char* cv, int src_gw, int i, int jj,
+                                          size_t row, int mode) {
     uint4 xk[S * S][2], xv[S * S][2];
-    const int taps = mode == MSF_RESAMPLE_STRIDED ? 1 : S * S;
+    const int taps = (mode == MSF_RESAMPLE_STRIDED && !ck) ? 1 : S * S;
 #pragma unroll
     for (int t = 0; t < S * S; ++t) {
         if (t < taps) {
@@ -74,7 +77,18 @@ __device__ __forceinline__ void pool_pair(const char* sk, const char* sv, char* 
             xv[t][1] = __ldg(reinterpret_cast<const uint4*>(sv + src + 16));
         }
     }
-    if (taps == 1) {
+    if (ck) {
+#pragma unroll
+        for (int t = 0; t < S * S; ++t) {
+            const int dy = t / S, dx = t % S;
+            const size_t src = (size_t)((S * i + dy) * src_gw + S * jj + dx) * row;
+            *reinterpret_cast<uint4*>(ck + src) = xk[t][0];
+            *reinterpret_cast<uint4*>(ck + src + 16) = xk[t][1];
+            *reinterpret_cast<uint4*>(cv + src) = xv[t][0];
+            *reinterpret_cast<uint4*>(cv + src + 16) = xv[t][1];
+        }
+    }
+    if (S == 1 || mode == MSF_RESAMPLE_STRIDED) {
         *reinterpret_cast<uint4*>(dk) = xk[0][0];
         *reinterpret_cast<uint4*>(dk + 16) = xk[0][1];
         *reinterpret_cast<uint4*>(dv) = xv[0][0];
@@ -114,12 +128,18 @@ __global__ void __launch_bounds__(256) pool_kernel(const PoolBatch jobs) {
     const char* sv = jb.src_v + (size_t)b * jb.src_bstride + (size_t)vec * 16;
     char* dk = jb.dst_k + (size_t)b * jb.dst_bstride + (size_t)tok * row + (size_t)vec * 16;
     char* dv = jb.dst_v + (size_t)b * jb.dst_bstride + (size_t)tok * row + (size_t)vec * 16;
+    char* ck = nullptr;
+    char* cv = nullptr;
+    if (jb.copy_k) {
+        ck = jb.copy_k + (size_t)b * jb.copy_bstride + (size_t)vec * 16;
+        cv = jb.copy_v + (size_t)b * jb.copy_bstride + (size_t)vec * 16;
+    }
     switch (jb.sigma) {
-    case 1: pool_pair<T, 1>(sk, sv, dk, dv, jb.src_gw, i, jj, row, jobs.mode); break;
-    case 2: pool_pair<T, 2>(sk, sv, dk, dv, jb.src_gw, i, jj, row, jobs.mode); break;
-    case 4: pool_pair<T, 4>(sk, sv, dk, dv, jb.src_gw, i, jj, row, jobs.mode); break;
+    case 1: pool_pair<T, 1>(sk, sv, dk, dv, ck, cv, jb.src_gw, i, jj, row, jobs.mode); break;
+    case 2: pool_pair<T, 2>(sk, sv, dk, dv, ck, cv, jb.src_gw, i, jj, row, jobs.mode); break;
+    case 4: pool_pair<T, 4>(sk, sv, dk, dv, ck, cv, jb.src_gw, i, jj, row, jobs.mode); break;
     default: {
-        // Larger strides: same arithmetic, loads issued per tap.
+        // Larger strides (never with a copy): same arithmetic, loads issued per tap.
         const int s = jb.sigma;
         for (int h = 0; h < 2; ++h) {
             if (jobs.mode == MSF_RESAMPLE_STRIDED) {

@@ -65,6 +65,9 @@ extern "C" msf_status msf_plan_create(const msf_plan_desc* desc, msf_plan_t* out
         if (d.scales[l] > smax) smax = d.scales[l];
     }
     if (d.grid_h % smax || d.grid_w % smax) return MSF_ERR_UNSUPPORTED;
+    if (d.fused_append != 0 && d.fused_append != 1) return MSF_ERR_INVALID_ARG;
+    // The staged head is the fine state at position 1 and needs a spare slot.
+    if (d.fused_append && (d.scales[0] != 1 || d.history_capacity < 1)) return MSF_ERR_UNSUPPORTED;
     // Index arithmetic in the kernels is 32-bit per stream; keep every
     // per-stream element count well inside that range.
     long long G = (long long)F * d.grid_h * d.grid_w;
@@ -76,6 +79,8 @@ extern "C" msf_status msf_plan_create(const msf_plan_desc* desc, msf_plan_t* out
     if (!p) return MSF_ERR_INVALID_ARG;
     memset((void*)p, 0, sizeof(Plan));
     p->d = d;
+    p->fused = d.fused_append != 0;
+    p->ring_slots = d.history_capacity + (p->fused ? 1 : 0);
     p->F = F;
     p->gh = F * d.grid_h;
     p->T = d.T;
@@ -117,7 +122,9 @@ extern "C" msf_status msf_plan_create(const msf_plan_desc* desc, msf_plan_t* out
     p->n_groups = ng;
 
     // Pyramid: per group g > 1, room for every history slot and every finer
-    // window state, all pooled to G / g^2 tokens.
+    // window state, all pooled to G / g^2 tokens. With fused_append the part
+    // is [finer states 2..n_finer | ring slots 0..capacity] (the head's level
+    // lives in the ring's spare slot): the same size.
     int pyr = 0;
     for (int gi = 0; gi < ng; ++gi) {
         msf::Group& g = p->groups[gi];
@@ -140,7 +147,7 @@ extern "C" msf_status msf_plan_create(const msf_plan_desc* desc, msf_plan_t* out
             long long it = (long long)p->B * p->H * ((g.q_end - g.q_begin + 255) / 256);
             long long nt = (d.sink_tokens + 127) / 128 + (p->N - g.q_begin + 127) / 128;
             if (g.scale == 1)
-                nt += ((long long)d.history_capacity * p->G + 127) / 128;
+                nt += ((long long)p->ring_slots * p->G + 127) / 128;
             else
                 nt += ((long long)(d.history_capacity + g.n_finer) * g.pooled + 127) / 128;
             items += it;
@@ -156,6 +163,7 @@ extern "C" msf_status msf_plan_create(const msf_plan_desc* desc, msf_plan_t* out
     p->ws_bytes = msf::workspace_bytes(*p);
     p->hist_count = d.history_frames;
     p->hist_oldest = 0;
+    p->hist_spare = d.history_frames;
     *out = p;
     return MSF_OK;
 }
@@ -203,8 +211,9 @@ extern "C" msf_status msf_plan_query(msf_plan_t plan, msf_plan_info* info) {
         o.pyr_offset = g.pyr_offset;
     }
     info->history_count = p.hist_count;
-    info->history_next_slot =
-        p.hist_count < p.d.history_capacity ? p.hist_count : p.hist_oldest;
+    info->history_next_slot = p.fused ? p.hist_spare
+                                      : (p.hist_count < p.d.history_capacity ? p.hist_count
+                                                                             : p.hist_oldest);
     info->pyramid_tokens = p.pyr_tokens;
     info->frames_per_state = p.F;
     info->workspace_bytes = p.ws_bytes;
@@ -249,15 +258,34 @@ extern "C" msf_status msf_plan_index_map(msf_plan_t plan, int32_t group, int32_t
         ++n;
     };
     for (int t = 0; t < p.d.sink_tokens; ++t) put(0, 0, 1, t, 0);
-    for (int f = 0; f < p.hist_count; ++f)
-        for (int i = 0; i < p.gh / g; ++i)
-            for (int j = 0; j < p.d.grid_w / g; ++j) put(1, f, g, i, j);
-    for (int l = 0; l < p.T; ++l) {
-        int s = p.d.scales[l];
-        int st = s < g ? g / s : 1;
-        int gh = p.st_gh[l] / st, gw = p.st_gw[l] / st;
+    auto put_frame = [&](int kind, int frame, int st, int gh, int gw) {
         for (int i = 0; i < gh; ++i)
-            for (int j = 0; j < gw; ++j) put(2, l, st, i, j);
+            for (int j = 0; j < gw; ++j) put(kind, frame, st, i, j);
+    };
+    if (!p.fused) {
+        for (int f = 0; f < p.hist_count; ++f) put_frame(1, f, g, p.gh / g, p.d.grid_w / g);
+        for (int l = 0; l < p.T; ++l) {
+            int s = p.d.scales[l];
+            int st = s < g ? g / s : 1;
+            put_frame(2, l, st, p.st_gh[l] / st, p.st_gw[l] / st);
+        }
+    } else {
+        // Kernel order: [finer states 2.. pooled | ring slots 0..count | window from k_win].
+        const int first_win = g == 1 ? 1 : 0;
+        if (g > 1)
+            for (int l = 1; l < p.groups[group].n_finer; ++l)
+                put_frame(2, l, g / p.d.scales[l], p.gh / g, p.d.grid_w / g);
+        for (int slot = 0; slot <= p.hist_count; ++slot) {
+            if (slot == p.hist_spare)
+                put_frame(2, 0, g, p.gh / g, p.d.grid_w / g);
+            else
+                put_frame(1, slot, g, p.gh / g, p.d.grid_w / g);
+        }
+        for (int l = first_win; l < p.T; ++l) {
+            int s = p.d.scales[l];
+            if (s < g) continue;
+            put_frame(2, l, 1, p.st_gh[l], p.st_gw[l]);
+        }
     }
     *n_rows = n;
     return MSF_OK;

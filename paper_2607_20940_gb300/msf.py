@@ -35,7 +35,7 @@ EXPORTS = (
     "msf_plan_query", "msf_plan_index_map", "msf_plan_bind", "msf_patchify", "msf_unpatchify",
     "msf_kv_resample", "msf_mssa_forward", "msf_mssa_forward_simt", "msf_history_append",
     "msf_plan_device_status", "msf_kernel_launches", "msf_unpatchify_noalloc",
-    "msf_selftest_wait_timeout",
+    "msf_selftest_wait_timeout", "msf_history_commit",
 )
 
 
@@ -48,7 +48,7 @@ class msf_plan_desc(ctypes.Structure):
         ("batch", ctypes.c_int32), ("dtype", ctypes.c_int32), ("resample", ctypes.c_int32),
         ("softmax_scale", ctypes.c_float), ("latent_channels", ctypes.c_int32),
         ("patch", ctypes.c_int32), ("embed_dim", ctypes.c_int32),
-        ("frames_per_state", ctypes.c_int32),
+        ("frames_per_state", ctypes.c_int32), ("fused_append", ctypes.c_int32),
     ]
 
 
@@ -98,6 +98,7 @@ def _load():
         "msf_kernel_launches": (ctypes.c_uint64, []),
         "msf_unpatchify_noalloc": (ctypes.c_int, [P, I32, VP, VP, VP, VP]),
         "msf_selftest_wait_timeout": (ctypes.c_int, [P, ctypes.c_int64, VP]),
+        "msf_history_commit": (ctypes.c_int, [P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -208,6 +209,10 @@ def msf_history_append(plan: int, k_win, v_win, stream=None) -> None:
            "msf_history_append")
 
 
+def msf_history_commit(plan: int) -> None:
+    _check(_lib.msf_history_commit(plan), "msf_history_commit")
+
+
 def msf_plan_device_status(plan: int, stream=None) -> int:
     return _lib.msf_plan_device_status(plan, _stream(stream))
 
@@ -230,7 +235,7 @@ def msf_kernel_launches() -> int:
 def make_desc(scales, grid_h, grid_w, heads, head_dim, sink_tokens, history_frames,
               history_capacity=None, batch=1, dtype=MSF_DTYPE_BF16, resample=MSF_RESAMPLE_AVG,
               softmax_scale=0.0, latent_channels=0, patch=0, embed_dim=0,
-              frames_per_state=1) -> msf_plan_desc:
+              frames_per_state=1, fused_append=0) -> msf_plan_desc:
     d = msf_plan_desc()
     d.T = len(scales)
     for i, s in enumerate(scales):
@@ -241,6 +246,7 @@ def make_desc(scales, grid_h, grid_w, heads, head_dim, sink_tokens, history_fram
     d.batch, d.dtype, d.resample, d.softmax_scale = batch, dtype, resample, softmax_scale
     d.latent_channels, d.patch, d.embed_dim = latent_channels, patch, embed_dim
     d.frames_per_state = frames_per_state
+    d.fused_append = fused_append
     return d
 
 
@@ -297,6 +303,10 @@ class Plan:
 
     def history_append(self, k_win, v_win, stream=None):
         msf_history_append(self.handle, k_win, v_win, stream)
+        self.refresh()
+
+    def history_commit(self):
+        msf_history_commit(self.handle)
         self.refresh()
 
     def device_status(self, stream=None) -> int:

@@ -152,3 +152,64 @@ def test_calls_before_bind_and_bad_pointers_fail_without_cuda():
     assert lib.msf_plan_index_map(p.handle, 7, None, 0, ctypes.byref(ctypes.c_size_t())) == \
         msf.MSF_ERR_INVALID_ARG
     assert msf.msf_status_string(msf.MSF_ERR_TIMEOUT) == "device wait timed out"
+
+
+# ------------------------------------------------ fused history update --
+
+def _fused_plan(scales, gh, gw, ns, nh, cap, F=1):
+    msf = _msf()
+    return msf.Plan(msf.make_desc(scales, gh, gw, 2, 64, ns, nh, history_capacity=cap,
+                                  frames_per_state=F, fused_append=1))
+
+
+@pytest.mark.parametrize("scales,gh,gw,ns,nh,cap,F", [
+    ((1, 1, 2), 8, 8, 5, 1, 3, 1),
+    ((1, 2, 2, 4), 8, 8, 3, 2, 2, 1),   # at capacity: every ring slot in use
+    ((1, 1), 4, 6, 0, 0, 1, 1),         # no coarser level, empty history
+    ((1, 2), 4, 4, 2, 1, 2, 2),         # chunked
+])
+def test_fused_append_context_is_the_same_rows(scales, gh, gw, ns, nh, cap, F):
+    """With the head staged in the ring's spare slot the kernels read the
+    same Eq. 4 context in another order: sink; for g > 1 the pooled window
+    states 2..; ring slots 0..count (live frames, then the spare = the head);
+    the window states from k_win. Same rows, same lengths, same FLOPs."""
+    p = _fused_plan(scales, gh, gw, ns, nh, cap, F)
+    ref = _plan(scales, gh, gw, ns, nh, cap=cap, F=F)
+    assert p.info.attention_flops == ref.info.attention_flops
+    assert p.info.history_next_slot == nh          # spare = first free slot
+    for gi, g in enumerate(schedule.query_groups(scales, gh, gw, F)):
+        got = [tuple(r) for r in p.index_map(gi).tolist()]
+        want = schedule.context_rows(scales, gh, gw, ns, nh, g.scale, F)
+        assert sorted(got) == sorted(want)
+        assert p.info.groups[gi].n_kv == len(want)
+        # the kernel order, written out from the layout rule
+        sink = [r for r in want if r[0] == schedule.SINK]
+        hist = [r for r in want if r[0] == schedule.HIST]
+        win = [r for r in want if r[0] == schedule.WIN]
+        head = [r for r in win if r[1] == 0]
+        finer = [r for r in win if r[1] > 0 and scales[r[1]] < g.scale]
+        rest = [r for r in win if r[1] > 0 and scales[r[1]] >= g.scale]
+        if g.scale == 1:
+            order = sink + hist + head + rest
+        else:
+            order = sink + finer + hist + head + rest
+        assert got == order
+
+
+def test_fused_append_validation_and_state():
+    msf = _msf()
+    for kw, err in [(dict(scales=(2, 2)), msf.MSF_ERR_UNSUPPORTED),     # head not fine
+                    (dict(cap=0), msf.MSF_ERR_UNSUPPORTED),               # no ring
+                    (dict(fa=2), msf.MSF_ERR_INVALID_ARG)]:
+        a = dict(scales=(1, 2), cap=2, fa=1)
+        a.update(kw)
+        with pytest.raises(msf.MsfError) as ei:
+            msf.Plan(msf.make_desc(a["scales"], 8, 8, 2, 64, 4, 0, history_capacity=a["cap"],
+                                   fused_append=a["fa"]))
+        assert ei.value.status == err
+    p = _fused_plan((1, 2), 8, 8, 4, 1, 2)
+    lib = msf._lib
+    assert lib.msf_history_commit(p.handle) == msf.MSF_ERR_STATE      # not bound
+    q = _plan((1, 2), 8, 8, 4, 1, cap=2)
+    assert lib.msf_history_commit(q.handle) == msf.MSF_ERR_STATE      # not fused
+    assert lib.msf_history_commit(None) == msf.MSF_ERR_INVALID_ARG
