@@ -12,6 +12,8 @@ Everything is plain numpy in float64, written from the paper:
   msp.py       MSP patchify / unpatchify with optional tier projections
   stream.py    rolling-window history update (Sec. 3.1, Algorithm 1)
   brute.py     a second, per-query enumeration of Eq. 4 for tiny grids
+  mssa_bwd.py  the gradient of Eq. 4 (softmax Jacobian and the adjoint of
+               Subsample), for training through the window
 
 Readings of points the paper leaves open (all chosen once, used everywhere):
   * Subsample: AVG (s x s block mean, the default) or STRIDED (top-left pick).

@@ -111,3 +111,53 @@ def test_chunk_tokens_frame_minor(monkeypatch):
         return np.stack(per, axis=2).reshape(x.shape[0], -1, per[0].shape[2])
     monkeypatch.setattr(msp, "patchify_chunk", bad)
     _fails(pins.test_chunked_patch_embedding_equals_conv3d)
+
+
+# ----------------------------------------------------------- gradient --
+
+import test_oracle_bwd_pins as bpins  # noqa: E402
+from oracle import mssa_bwd  # noqa: E402
+
+
+def test_softmax_jacobian_without_row_term(monkeypatch):
+    def bad(q, k, v, dout, scale):
+        q, k, v, dout = (np.asarray(a, dtype=np.float64) for a in (q, k, v, dout))
+        B, Nq, H, D = q.shape
+        dq, dk, dv = np.zeros_like(q), np.zeros_like(k), np.zeros_like(v)
+        for b in range(B):
+            for h in range(H):
+                s = scale * (q[b, :, h] @ k[b, :, h].T)
+                p = np.exp(s - s.max(axis=1, keepdims=True))
+                p /= p.sum(axis=1, keepdims=True)
+                dv[b, :, h] = p.T @ dout[b, :, h]
+                ds = p * (dout[b, :, h] @ v[b, :, h].T)       # row term dropped
+                dq[b, :, h] = scale * (ds @ k[b, :, h])
+                dk[b, :, h] = scale * (ds.T @ q[b, :, h])
+        return dq, dk, dv
+    monkeypatch.setattr(mssa_bwd, "attention_backward", bad)
+    _fails(bpins.test_backward_equals_torch_autograd, mssa.AVG, (1, 2), 4, 4, 1, 3, 1)
+    _fails(bpins.test_backward_invariants, mssa.AVG)
+
+
+def test_pool_adjoint_without_normalisation(monkeypatch):
+    good = mssa_bwd.resample_adjoint
+
+    def bad(dy, gh, gw, sigma, mode=mssa.AVG):
+        y = good(dy, gh, gw, sigma, mode)
+        return y * (sigma * sigma) if mode == mssa.AVG else y
+    monkeypatch.setattr(mssa_bwd, "resample_adjoint", bad)
+    _fails(bpins.test_backward_equals_torch_autograd, mssa.AVG, (1, 2), 4, 4, 1, 3, 1)
+
+
+def test_strided_adjoint_to_the_wrong_token(monkeypatch):
+    good = mssa_bwd.resample_adjoint
+
+    def bad(dy, gh, gw, sigma, mode=mssa.AVG):
+        y = good(dy, gh, gw, sigma, mode)
+        if mode != mssa.STRIDED or sigma == 1:
+            return y
+        B = y.shape[0]
+        grid = y.reshape((B, gh, gw) + y.shape[2:])
+        return np.roll(grid, 1, axis=2).reshape(y.shape)   # one column to the right
+    monkeypatch.setattr(mssa_bwd, "resample_adjoint", bad)
+    _fails(bpins.test_backward_equals_torch_autograd, mssa.STRIDED, (1, 2), 4, 4, 1, 3, 1)
