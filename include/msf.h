@@ -131,6 +131,7 @@ typedef struct msf_plan_info {
     uint64_t pyramid_k_offset;        /* byte offset of the K pyramid [B, pyramid_tokens, H, D]
                                          inside the workspace */
     uint64_t pyramid_v_offset;        /* byte offset of the V pyramid */
+    uint64_t backward_workspace_bytes; /* scratch msf_mssa_backward needs */
 } msf_plan_info;
 
 typedef struct msf_plan* msf_plan_t;
@@ -233,6 +234,32 @@ msf_status msf_kv_resample(msf_plan_t plan, const void* k_win, const void* v_win
  * INVALID_ARG, STATE, CUDA. */
 msf_status msf_mssa_forward(msf_plan_t plan, const void* q, const void* k_win, const void* v_win,
                             void* out, void* stream);
+
+/* msf_mssa_forward that also writes, for every query row, the natural-log
+ * log-sum-exp of its scaled scores over its context,
+ *   lse[b, h, t] = ln sum_j exp(scale * q[b,t,h,:] . K_g[j]),
+ * fp32 [B, H, N] (16-byte aligned, or NULL for none): the statistic
+ * msf_mssa_backward needs to rebuild the softmax. Errors as msf_mssa_forward. */
+msf_status msf_mssa_forward_lse(msf_plan_t plan, const void* q, const void* k_win,
+                                const void* v_win, void* out, float* lse, void* stream);
+
+/* Gradient of MSSA (Eq. 4) for training through the window: given
+ * dout = dL/dout [B, N, H, D] and the forward's out and lse, writes
+ *   dq, dk_win, dv_win [B, N, H, D] (plan dtype) = dL/dq, dL/dk_win, dL/dv_win,
+ * with the softmax Jacobian per query group and the context gradients sent
+ * back through the adjoint of Subsample (AVG: 1/s^2 of a pooled row to each
+ * of its s x s source tokens; STRIDED: all of it to the top-left one); a
+ * token used by several groups sums their contributions. The sink and the
+ * history ring are a detached cache (Algorithm 1 updates it with a
+ * stop-gradient) and get no gradient. Needs the pyramid of the forward pass
+ * (the last msf_kv_resample on the stream) and the same history state (no
+ * commit or append in between). bwd_workspace: >= info.backward_workspace_bytes
+ * bytes, 16-byte aligned, overwritten. Output buffers may not alias inputs.
+ * Errors: INVALID_ARG, STATE (not bound), WORKSPACE, CUDA. */
+msf_status msf_mssa_backward(msf_plan_t plan, const void* q, const void* k_win, const void* v_win,
+                             const void* out, const void* dout, const float* lse, void* dq,
+                             void* dk_win, void* dv_win, void* bwd_workspace,
+                             size_t bwd_workspace_bytes, void* stream);
 
 /* Same computation always on the fp32 CUDA-core kernel (a cross-check of the
  * tensor-core kernel for bf16 plans). */

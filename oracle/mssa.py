@@ -136,3 +136,24 @@ def pyramid_segment(kv_win, kv_hist, scales, grid_h, grid_w, g, mode=AVG, frames
     if not parts:
         return np.zeros((kv_win.shape[0], 0) + tuple(kv_win.shape[2:]))
     return np.concatenate(parts, axis=1)
+
+
+def mssa_lse(q, k_win, k_sink, k_hist, scales, grid_h, grid_w, mode=AVG, softmax_scale=None,
+             heads=None, frames=1):
+    """Per query row, ln sum_j exp(scale q . k_j) over its Eq. 4 context (the
+    softmax normaliser the backward pass rebuilds P from). [B, H, N] float64;
+    heads outside ``heads`` are NaN."""
+    q = np.asarray(q, dtype=np.float64)
+    B, N, H, D = q.shape
+    scale = D ** -0.5 if not softmax_scale else softmax_scale
+    out = np.full((B, H, N), np.nan, dtype=np.float64)
+    hsel = list(range(H)) if heads is None else list(heads)
+    for grp in schedule.query_groups(scales, grid_h, grid_w, frames):
+        kc = group_context(k_win[:, :, hsel], k_sink[:, :, hsel], k_hist[:, :, :, hsel],
+                           scales, grid_h, grid_w, grp.scale, mode, frames)
+        for b in range(B):
+            for hi, h in enumerate(hsel):
+                s = scale * (q[b, grp.q_begin:grp.q_end, h] @ kc[b, :, hi].T)
+                m = s.max(axis=1)
+                out[b, h, grp.q_begin:grp.q_end] = m + np.log(np.exp(s - m[:, None]).sum(axis=1))
+    return out

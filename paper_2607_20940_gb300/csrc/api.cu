@@ -119,6 +119,7 @@ void build_attn_args(const Plan& p, const void* q, const void* k_win, const void
     a.scale_log2 = p.scale * 1.4426950408889634f;
     a.n_groups = p.n_groups;
     a.status = msf::status_word(p);
+    a.N = p.N;
     for (int gi = 0; gi < p.n_groups; ++gi) {
         const msf::Group& g = p.groups[gi];
         msf::AttnGroup& ag = a.g[gi];
@@ -322,6 +323,21 @@ extern "C" msf_status msf_mssa_forward_simt(msf_plan_t plan, const void* q, cons
     return cuda_status(msf::launch_attn_simt(a, p.elem == 2, (cudaStream_t)stream));
 }
 
+extern "C" msf_status msf_mssa_forward_lse(msf_plan_t plan, const void* q, const void* k_win,
+                                           const void* v_win, void* out, float* lse,
+                                           void* stream) {
+    if (!plan) return MSF_ERR_INVALID_ARG;
+    Plan& p = *plan;
+    msf_status st = check_attn_args(p, q, k_win, v_win, out);
+    if (st != MSF_OK) return st;
+    if (lse && !aligned16(lse)) return MSF_ERR_INVALID_ARG;
+    msf::AttnArgs a;
+    build_attn_args(p, q, k_win, v_win, out, a);
+    a.lse = lse;
+    if (p.elem == 2) return msf::launch_attn_tc(plan, a, (cudaStream_t)stream);
+    return cuda_status(msf::launch_attn_simt(a, false, (cudaStream_t)stream));
+}
+
 extern "C" msf_status msf_mssa_forward(msf_plan_t plan, const void* q, const void* k_win,
                                        const void* v_win, void* out, void* stream) {
     if (!plan) return MSF_ERR_INVALID_ARG;
@@ -332,6 +348,116 @@ extern "C" msf_status msf_mssa_forward(msf_plan_t plan, const void* q, const voi
     build_attn_args(p, q, k_win, v_win, out, a);
     if (p.elem == 2) return msf::launch_attn_tc(plan, a, (cudaStream_t)stream);
     return cuda_status(msf::launch_attn_simt(a, false, (cudaStream_t)stream));
+}
+
+// Gradient rows of group gi: the context rows that come from the window,
+// each run with the window token its rows map back to (Eq. 4's Subsample
+// undone by the adjoint). Mirrors the context layout of build_attn_args.
+static void build_bwd_group(const Plan& p, int gi, const void* k_win, const void* v_win,
+                            msf::BwdGroup& bg) {
+    memset(&bg, 0, sizeof(bg));
+    const msf::Group& g = p.groups[gi];
+    const size_t row = row_bytes(p);
+    bg.q_begin = g.q_begin;
+    bg.q_end = g.q_end;
+    auto add = [&](const char* k, const char* v, long long bs, int row0, int len, int rows_total,
+                   int map_id, int sigma, int dst0, int src_gw, int out_gw) {
+        if (len <= 0) return;
+        msf::GradSeg& s = bg.gseg[bg.n_gseg++];
+        s.k = k;
+        s.v = v;
+        s.bstride = bs;
+        s.row0 = row0;
+        s.len = len;
+        s.rows_total = rows_total;
+        s.map_id = map_id;
+        s.sigma = sigma;
+        s.dst0 = dst0;
+        s.src_gw = src_gw;
+        s.out_gw = out_gw;
+    };
+    const long long win_bs = (long long)p.N * row;
+    const long long pyr_bs = (long long)p.pyr_tokens * row;
+    const long long ring_bs = (long long)p.ring_slots * p.G * row;
+    if (g.scale == 1) {
+        if (p.fused) {
+            // the head is read from the ring's spare slot
+            add((const char*)p.k_hist, (const char*)p.v_hist, ring_bs, p.hist_spare * p.G, p.G,
+                p.ring_slots * p.G, msf::kMapHist, 1, 0, 0, 0);
+            add((const char*)k_win, (const char*)v_win, win_bs, p.st_n[0], p.N - p.st_n[0], p.N,
+                msf::kMapWin, 1, p.st_n[0], 0, 0);
+        } else {
+            add((const char*)k_win, (const char*)v_win, win_bs, 0, p.N, p.N, msf::kMapWin, 1, 0, 0,
+                0);
+        }
+        return;
+    }
+    const int out_gw = p.d.grid_w / g.scale;
+    for (int l = 0; l < g.n_finer; ++l) {
+        int slot;  // pyramid slot of pooled state l (same rule as the resample jobs)
+        if (!p.fused)
+            slot = p.hist_count + l;
+        else
+            slot = l == 0 ? g.n_finer - 1 + p.hist_spare : l - 1;
+        add(msf::pyr_k(p), msf::pyr_v(p), pyr_bs, g.pyr_offset + slot * g.pooled, g.pooled,
+            p.pyr_tokens, msf::kMapPyr, g.scale / p.d.scales[l], p.st_off[l], p.st_gw[l], out_gw);
+    }
+    add((const char*)k_win, (const char*)v_win, win_bs, g.q_begin, p.N - g.q_begin, p.N,
+        msf::kMapWin, 1, g.q_begin, 0, 0);
+}
+
+extern "C" msf_status msf_mssa_backward(msf_plan_t plan, const void* q, const void* k_win,
+                                        const void* v_win, const void* out, const void* dout,
+                                        const float* lse, void* dq, void* dk_win, void* dv_win,
+                                        void* bwd_ws, size_t bwd_ws_bytes, void* stream) {
+    if (!plan) return MSF_ERR_INVALID_ARG;
+    Plan& p = *plan;
+    if (!q || !k_win || !v_win || !out || !dout || !lse || !dq || !dk_win || !dv_win || !bwd_ws)
+        return MSF_ERR_INVALID_ARG;
+    if (!p.bound) return MSF_ERR_STATE;
+    const void* in[] = {q, k_win, v_win, out, dout, lse, dq, dk_win, dv_win, bwd_ws};
+    for (const void* x : in)
+        if (!aligned16(x)) return MSF_ERR_INVALID_ARG;
+    const void* outs[] = {dq, dk_win, dv_win};
+    const void* ins[] = {q, k_win, v_win, out, dout, lse};
+    for (const void* o : outs)
+        for (const void* i : ins)
+            if (o == i) return MSF_ERR_INVALID_ARG;
+    if (dq == dk_win || dq == dv_win || dk_win == dv_win) return MSF_ERR_INVALID_ARG;
+    if (bwd_ws_bytes < msf::bwd_workspace_bytes(p)) return MSF_ERR_WORKSPACE;
+    cudaStream_t s = (cudaStream_t)stream;
+    const bool bf16 = p.elem == 2;
+    msf::BwdCommon c;
+    memset(&c, 0, sizeof(c));
+    c.q = (const char*)q;
+    c.dout = (const char*)dout;
+    c.out = (const char*)out;
+    c.lse = lse;
+    c.delta = (float*)bwd_ws;
+    c.dk_acc = (float*)((char*)bwd_ws + msf::bwd_delta_bytes(p));
+    c.dv_acc = (float*)((char*)bwd_ws + msf::bwd_delta_bytes(p) + msf::bwd_acc_bytes(p));
+    c.bstride = (long long)p.N * row_bytes(p);
+    c.H = p.H;
+    c.D = p.D;
+    c.B = p.B;
+    c.N = p.N;
+    c.scale = p.scale;
+    c.scale_log2 = p.scale * 1.4426950408889634f;
+    c.mode = p.d.resample;
+    cudaError_t e = cudaMemsetAsync(c.dk_acc, 0, 2 * msf::bwd_acc_bytes(p), s);
+    if (e == cudaSuccess) e = msf::launch_bwd_delta(c, bf16, s);
+    if (e != cudaSuccess) return cuda_status(e);
+    msf::AttnArgs a;
+    build_attn_args(p, q, k_win, v_win, (void*)out, a);
+    e = msf::launch_bwd_dq_simt(c, a, dq, bf16, s);
+    if (e != cudaSuccess) return cuda_status(e);
+    for (int gi = 0; gi < p.n_groups; ++gi) {
+        msf::BwdGroup bg;
+        build_bwd_group(p, gi, k_win, v_win, bg);
+        e = msf::launch_bwd_dkdv_simt(c, bg, bf16, s);
+        if (e != cudaSuccess) return cuda_status(e);
+    }
+    return cuda_status(msf::launch_bwd_cast(c, dk_win, dv_win, bf16, s));
 }
 
 static msf::MspShape msp_shape(const Plan& p) {

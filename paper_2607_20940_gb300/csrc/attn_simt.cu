@@ -99,6 +99,8 @@ __global__ void __launch_bounds__(128) attn_simt_kernel(const AttnArgs a) {
     if (!valid) return;
     T* op = (T*)(a.out + (size_t)b * a.q_bstride + (size_t)t * row) + (size_t)h * D;
     const float inv = 1.0f / l;
+    // scores are in log2 units: ln sum_j exp(s_j) = (m + log2 l) * ln 2
+    if (a.lse && c == 0) a.lse[((size_t)b * a.H + h) * a.N + t] = (m + log2f(l)) * 0.6931471805599453f;
 #pragma unroll
     for (int i = 0; i < DP; ++i) op[4 * i + c] = tot<T>(o[i] * inv);
 }

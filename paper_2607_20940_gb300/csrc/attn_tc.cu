@@ -92,6 +92,8 @@ struct TcParams {
     unsigned int* counters;  // per item
     float* partials;         // 2 slots per CTA
     long long wait_limit;
+    float* lse;              // optional [B, H, N] row log-sum-exp (natural log)
+    int N;                   // query rows per stream
 };
 struct TcMaps {
     CUtensorMap q;
@@ -538,6 +540,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 p.out + (size_t)pc.b * p.out_bstride + ((size_t)qrow * p.H + pc.h) * D;
             if (pc.whole) {
                 const float inv = 1.0f / l;
+                // P, O and l share the scale 2^-m_used: ln sum exp = (m_used + log2 l) ln 2
+                if (store && p.lse)
+                    p.lse[((size_t)pc.b * p.H + pc.h) * p.N + qrow] =
+                        (m_used + log2f(l)) * 0.6931471805599453f;
 #pragma unroll
                 for (int c = 0; c < D / 32; ++c) {
                     uint32_t o[32];
@@ -616,6 +622,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                         L += ex2(__ldcg(q + C::kSlotML + rr) - M) * __ldcg(q + C::kSlotML + 2 * kBlockM + rr);
                     }
                     const float inv = 1.0f / L;
+                    if (store && p.lse)
+                        p.lse[((size_t)pc.b * p.H + pc.h) * p.N + qrow] =
+                            (M + log2f(L)) * 0.6931471805599453f;
 #pragma unroll 1
                     for (int ch = 0; ch < D / 32; ++ch) {
                         float acc[32];
@@ -765,6 +774,8 @@ msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st) {
     tp.counters = attn_counters(P);
     tp.partials = attn_partials(P);
     tp.wait_limit = kWaitLimit;
+    tp.lse = a.lse;
+    tp.N = P.N;
 
     if (!ensure(2 * kNumMaps, &cache.maps.q, a.q, P.N, a.q_bstride)) {
         set_cuda_error((int)cudaErrorInvalidValue);

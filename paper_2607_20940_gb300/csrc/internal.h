@@ -91,6 +91,11 @@ inline size_t msp_split_bytes(const Plan& p) {
     size_t per = (size_t)p.d.latent_channels * p.d.patch * p.gh * p.d.patch * p.d.grid_w;
     return round256((size_t)kMaxDeembedSplits * p.B * per * 4);
 }
+// Backward workspace (caller-provided per msf_mssa_backward call):
+// [delta fp32 [B, H, N] | dk_acc fp32 [B, N, H, D] | dv_acc fp32 [B, N, H, D]].
+inline size_t bwd_delta_bytes(const Plan& p) { return round256((size_t)p.B * p.H * p.N * 4); }
+inline size_t bwd_acc_bytes(const Plan& p) { return round256((size_t)p.B * p.N * p.H * p.D * 4); }
+inline size_t bwd_workspace_bytes(const Plan& p) { return bwd_delta_bytes(p) + 2 * bwd_acc_bytes(p); }
 inline size_t workspace_bytes(const Plan& p) {
     return kStatusBytes + 2 * pyramid_bytes(p) + msp_scratch_bytes(p) + attn_counter_bytes(p) +
            attn_partial_bytes(p) + msp_split_bytes(p);

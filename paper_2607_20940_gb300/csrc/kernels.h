@@ -131,7 +131,54 @@ struct AttnArgs {
     int n_groups;
     AttnGroup g[MSF_MAX_GROUPS];
     unsigned int* status;
+    float* lse;           // optional [B, H, N] row log-sum-exp (natural log); NULL = none
+    int N;                // query rows per stream
 };
 cudaError_t launch_attn_simt(const AttnArgs& a, bool bf16, cudaStream_t st);
+
+// ---------------------------------------------------------- MSSA backward
+//
+// Context rows whose key/value gradients flow back to window tokens: rows
+// [row0, row0 + len) of a [B, rows_total, H, D] tensor pair (k, v). sigma 1:
+// row row0 + r is window token dst0 + r. sigma > 1: row r is token
+// (r / out_gw, r % out_gw) of a pooled state whose fine grid (src_gw wide)
+// starts at window token dst0; the adjoint of Subsample spreads it back.
+struct GradSeg {
+    const char* k;
+    const char* v;
+    long long bstride;  // bytes between streams
+    int row0, len, rows_total, map_id;
+    int sigma, dst0, src_gw, out_gw;
+};
+constexpr int kMaxGradSeg = MSF_MAX_STATES + 1;
+struct BwdGroup {
+    int q_begin, q_end;
+    int n_gseg;
+    GradSeg gseg[kMaxGradSeg];
+};
+// Per-launch arguments shared by the backward kernels.
+struct BwdCommon {
+    const char* q;      // [B, N, H, D]
+    const char* dout;   // [B, N, H, D]
+    const char* out;    // [B, N, H, D]
+    const float* lse;   // [B, H, N], natural log
+    float* delta;       // [B, H, N]: rowsum(dout * out)
+    float* dk_acc;      // [B, N, H, D] fp32 accumulators (all groups)
+    float* dv_acc;
+    long long bstride;  // bytes between streams of q/dout/out/dq
+    int H, D, B, N;
+    float scale;        // softmax scale
+    float scale_log2;   // scale * log2(e)
+    int mode;           // msf_resample_mode (adjoint of Subsample)
+};
+cudaError_t launch_bwd_delta(const BwdCommon& c, bool bf16, cudaStream_t st);
+// dq for every query of every group (context of each group as in the forward).
+cudaError_t launch_bwd_dq_simt(const BwdCommon& c, const AttnArgs& a, void* dq, bool bf16,
+                               cudaStream_t st);
+// dK/dV of one group's gradient rows, accumulated into dk_acc/dv_acc.
+cudaError_t launch_bwd_dkdv_simt(const BwdCommon& c, const BwdGroup& g, bool bf16,
+                                 cudaStream_t st);
+// dk_win, dv_win = cast(dk_acc, dv_acc).
+cudaError_t launch_bwd_cast(const BwdCommon& c, void* dk, void* dv, bool bf16, cudaStream_t st);
 
 }  // namespace msf

@@ -217,6 +217,7 @@ extern "C" msf_status msf_plan_query(msf_plan_t plan, msf_plan_info* info) {
     info->pyramid_tokens = p.pyr_tokens;
     info->frames_per_state = p.F;
     info->workspace_bytes = p.ws_bytes;
+    info->backward_workspace_bytes = msf::bwd_workspace_bytes(p);
     info->attention_flops = flops_for(p);
     // Dense reference: every state fine, every query sees sink + history + T*G.
     uint64_t nd = (uint64_t)p.T * p.G;

@@ -35,7 +35,8 @@ EXPORTS = (
     "msf_plan_query", "msf_plan_index_map", "msf_plan_bind", "msf_patchify", "msf_unpatchify",
     "msf_kv_resample", "msf_mssa_forward", "msf_mssa_forward_simt", "msf_history_append",
     "msf_plan_device_status", "msf_kernel_launches", "msf_unpatchify_noalloc",
-    "msf_selftest_wait_timeout", "msf_history_commit",
+    "msf_selftest_wait_timeout", "msf_history_commit", "msf_mssa_forward_lse",
+    "msf_mssa_backward",
 )
 
 
@@ -71,6 +72,7 @@ class msf_plan_info(ctypes.Structure):
         ("workspace_bytes", ctypes.c_uint64), ("attention_flops", ctypes.c_uint64),
         ("dense_flops", ctypes.c_uint64), ("resample_bytes", ctypes.c_uint64),
         ("pyramid_k_offset", ctypes.c_uint64), ("pyramid_v_offset", ctypes.c_uint64),
+        ("backward_workspace_bytes", ctypes.c_uint64),
     ]
 
 
@@ -99,6 +101,8 @@ def _load():
         "msf_unpatchify_noalloc": (ctypes.c_int, [P, I32, VP, VP, VP, VP]),
         "msf_selftest_wait_timeout": (ctypes.c_int, [P, ctypes.c_int64, VP]),
         "msf_history_commit": (ctypes.c_int, [P]),
+        "msf_mssa_forward_lse": (ctypes.c_int, [P, VP, VP, VP, VP, VP, VP]),
+        "msf_mssa_backward": (ctypes.c_int, [P, VP, VP, VP, VP, VP, VP, VP, VP, VP, VP, SZ, VP]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -209,6 +213,19 @@ def msf_history_append(plan: int, k_win, v_win, stream=None) -> None:
            "msf_history_append")
 
 
+def msf_mssa_forward_lse(plan: int, q, k_win, v_win, out, lse, stream=None) -> None:
+    _check(_lib.msf_mssa_forward_lse(plan, _ptr(q), _ptr(k_win), _ptr(v_win), _ptr(out),
+                                     _ptr(lse), _stream(stream)), "msf_mssa_forward_lse")
+
+
+def msf_mssa_backward(plan: int, q, k_win, v_win, out, dout, lse, dq, dk_win, dv_win, bwd_ws,
+                      stream=None) -> None:
+    nbytes = bwd_ws.numel() * bwd_ws.element_size()
+    _check(_lib.msf_mssa_backward(plan, _ptr(q), _ptr(k_win), _ptr(v_win), _ptr(out), _ptr(dout),
+                                  _ptr(lse), _ptr(dq), _ptr(dk_win), _ptr(dv_win), _ptr(bwd_ws),
+                                  nbytes, _stream(stream)), "msf_mssa_backward")
+
+
 def msf_history_commit(plan: int) -> None:
     _check(_lib.msf_history_commit(plan), "msf_history_commit")
 
@@ -297,6 +314,19 @@ class Plan:
 
     def mssa_forward(self, q, k_win, v_win, out, stream=None):
         msf_mssa_forward(self.handle, q, k_win, v_win, out, stream)
+
+    def mssa_forward_lse(self, q, k_win, v_win, out, lse, stream=None):
+        msf_mssa_forward_lse(self.handle, q, k_win, v_win, out, lse, stream)
+
+    def mssa_backward(self, q, k_win, v_win, out, dout, lse, dq, dk_win, dv_win, bwd_ws,
+                      stream=None):
+        msf_mssa_backward(self.handle, q, k_win, v_win, out, dout, lse, dq, dk_win, dv_win, bwd_ws,
+                          stream)
+
+    def backward_workspace(self, device="cuda"):
+        import torch
+        return torch.empty(int(self.info.backward_workspace_bytes), dtype=torch.uint8,
+                           device=device)
 
     def mssa_forward_simt(self, q, k_win, v_win, out, stream=None):
         msf_mssa_forward_simt(self.handle, q, k_win, v_win, out, stream)

@@ -123,3 +123,16 @@ def test_backward_invariants(mode):
     np.testing.assert_allclose(ksum, 0.0, atol=1e-12)
     vsum = g["dv_win"].sum(1) + g["dv_sink"].sum(1) + g["dv_hist"].sum((1, 2))
     np.testing.assert_allclose(vsum, x["dout"].sum(1), atol=1e-12)
+
+
+def test_lse_equals_library_logsumexp():
+    """The row normaliser on the all-fine schedule is torch.logsumexp of the
+    scores against [sink || history || window]."""
+    rng = np.random.default_rng(31)
+    scales, gh, gw = (1, 1, 1), 4, 6
+    x = _inputs(rng, scales, gh, gw, 1, ns=5, nh=2, H=3, D=16, B=2)
+    got = mssa.mssa_lse(x["q"], x["k_win"], x["k_sink"], x["k_hist"], scales, gh, gw)
+    B, N, H, D = x["q"].shape
+    K = np.concatenate([x["k_sink"], x["k_hist"].reshape(B, -1, H, D), x["k_win"]], axis=1)
+    s = torch.einsum("bnhd,bmhd->bhnm", torch.from_numpy(x["q"]), torch.from_numpy(K)) / D ** 0.5
+    np.testing.assert_allclose(got, torch.logsumexp(s, dim=-1).numpy(), rtol=0, atol=1e-12)
