@@ -218,7 +218,8 @@ def _timed(fn, flush, reps=5, warm=2, sleep=True):
 
 def other_configs(msf, synth, dev, flush, peaks, rank):
     """The remaining configurations of the workload family, measured after the
-    timed region: the three-scale 48x80 window, the paper's chunked layout
+    timed region: the three-scale 48x80 window, the training direction (forward
+    with the row log-sum-exp and the MSSA gradient), the paper's chunked layout
     (3 latent frames per state) beside its all-fine window, the B=4 streaming rollout
     (120 steps, history 2 -> capacity 4), the 30-layer window pass, and the
     bandwidth of the pyramid and embedding kernels."""
@@ -265,6 +266,32 @@ def other_configs(msf, synth, dev, flush, peaks, rank):
         raise RuntimeError("device status error (three-scale)")
     plan.close()
     del t
+
+    # ---- training direction at the 480p layer: forward with the row
+    #      log-sum-exp, then the MSSA gradient (dq, dk_win, dv_win)
+    wl = synth.LAYER_480P
+    plan, t = setup(wl)
+    B, N, H = wl.batch, plan.info.n_tokens, wl.heads
+    lse = torch.empty((B, H, N), dtype=torch.float32, device=dev)
+    dout = rnd(t["q"].shape)
+    grads = [torch.empty_like(t["q"]) for _ in range(3)]
+    bws = plan.backward_workspace(dev)
+    plan.kv_resample(t["k_win"], t["v_win"], msf.MSF_RESAMPLE_FULL)
+    fwd_ms = _timed(lambda: plan.mssa_forward_lse(t["q"], t["k_win"], t["v_win"], t["out"], lse), flush)
+    bwd_ms = _timed(lambda: plan.mssa_backward(t["q"], t["k_win"], t["v_win"], t["out"], dout, lse,
+                                               *grads, bws), flush)
+    simt_ms = _timed(lambda: plan.mssa_backward_simt(t["q"], t["k_win"], t["v_win"], t["out"], dout,
+                                                     lse, *grads, bws), flush, reps=1, warm=1)
+    bfl = plan.info.backward_flops
+    if plan.device_status() != msf.MSF_OK:
+        raise RuntimeError("device status error (backward)")
+    out["backward_480p"] = {"workload": wl.name, "forward_lse_us": fwd_ms * 1e3,
+                            "backward_us": bwd_ms * 1e3, "backward_gflop": bfl / 1e9,
+                            "backward_tflops": bfl / (bwd_ms * 1e-3) / 1e12,
+                            "backward_frac": bfl / (bwd_ms * 1e-3) / 1e12 / bf16,
+                            "backward_cuda_core_us": simt_ms * 1e3}
+    plan.close()
+    del t, grads, bws
 
     # ---- the paper's chunked layout: 3 latent frames per state (12870 tokens),
     #      sink = one chunk, one history chunk; MSSA beside the all-fine window

@@ -132,6 +132,10 @@ typedef struct msf_plan_info {
                                          inside the workspace */
     uint64_t pyramid_v_offset;        /* byte offset of the V pyramid */
     uint64_t backward_workspace_bytes; /* scratch msf_mssa_backward needs */
+    uint64_t backward_flops;          /* algorithmic FLOPs of msf_mssa_backward: per group
+                                         Nq * (6*D*Nkv + 4*D*Nkv_window) * H * B (S, dP and
+                                         dQ over the whole context; dK and dV over the rows
+                                         that come from the window) */
 } msf_plan_info;
 
 typedef struct msf_plan* msf_plan_t;
@@ -255,11 +259,21 @@ msf_status msf_mssa_forward_lse(msf_plan_t plan, const void* q, const void* k_wi
  * (the last msf_kv_resample on the stream) and the same history state (no
  * commit or append in between). bwd_workspace: >= info.backward_workspace_bytes
  * bytes, 16-byte aligned, overwritten. Output buffers may not alias inputs.
+ * bf16 plans run tcgen05 tensor-core kernels (one for dq over each query
+ * tile's whole context, one per query group for the window rows' dk/dv);
+ * fp32 plans run CUDA-core kernels.
  * Errors: INVALID_ARG, STATE (not bound), WORKSPACE, CUDA. */
 msf_status msf_mssa_backward(msf_plan_t plan, const void* q, const void* k_win, const void* v_win,
                              const void* out, const void* dout, const float* lse, void* dq,
                              void* dk_win, void* dv_win, void* bwd_workspace,
                              size_t bwd_workspace_bytes, void* stream);
+
+/* Same gradient always on the fp32 CUDA-core kernels (a cross-check of the
+ * tensor-core backward for bf16 plans). */
+msf_status msf_mssa_backward_simt(msf_plan_t plan, const void* q, const void* k_win,
+                                  const void* v_win, const void* out, const void* dout,
+                                  const float* lse, void* dq, void* dk_win, void* dv_win,
+                                  void* bwd_workspace, size_t bwd_workspace_bytes, void* stream);
 
 /* Same computation always on the fp32 CUDA-core kernel (a cross-check of the
  * tensor-core kernel for bf16 plans). */

@@ -3,6 +3,7 @@
 #include <cuda_runtime.h>
 #include <string.h>
 
+#include "attn_bwd_tc.h"
 #include "attn_tc.h"
 #include "gemm_tc.h"
 #include "msp_tc.h"
@@ -406,10 +407,10 @@ static void build_bwd_group(const Plan& p, int gi, const void* k_win, const void
         msf::kMapWin, 1, g.q_begin, 0, 0);
 }
 
-extern "C" msf_status msf_mssa_backward(msf_plan_t plan, const void* q, const void* k_win,
-                                        const void* v_win, const void* out, const void* dout,
-                                        const float* lse, void* dq, void* dk_win, void* dv_win,
-                                        void* bwd_ws, size_t bwd_ws_bytes, void* stream) {
+static msf_status mssa_backward(msf_plan_t plan, const void* q, const void* k_win,
+                                const void* v_win, const void* out, const void* dout,
+                                const float* lse, void* dq, void* dk_win, void* dv_win,
+                                void* bwd_ws, size_t bwd_ws_bytes, void* stream, bool tc) {
     if (!plan) return MSF_ERR_INVALID_ARG;
     Plan& p = *plan;
     if (!q || !k_win || !v_win || !out || !dout || !lse || !dq || !dk_win || !dv_win || !bwd_ws)
@@ -449,15 +450,47 @@ extern "C" msf_status msf_mssa_backward(msf_plan_t plan, const void* q, const vo
     if (e != cudaSuccess) return cuda_status(e);
     msf::AttnArgs a;
     build_attn_args(p, q, k_win, v_win, (void*)out, a);
-    e = msf::launch_bwd_dq_simt(c, a, dq, bf16, s);
-    if (e != cudaSuccess) return cuda_status(e);
-    for (int gi = 0; gi < p.n_groups; ++gi) {
-        msf::BwdGroup bg;
-        build_bwd_group(p, gi, k_win, v_win, bg);
-        e = msf::launch_bwd_dkdv_simt(c, bg, bf16, s);
+    msf::BwdGroup bg[MSF_MAX_GROUPS];
+    for (int gi = 0; gi < p.n_groups; ++gi) build_bwd_group(p, gi, k_win, v_win, bg[gi]);
+    if (tc && bf16) {
+        msf::BwdTcInput in;
+        in.a = &a;
+        in.g = bg;
+        in.q = q;
+        in.dout = dout;
+        in.lse = lse;
+        in.delta = c.delta;
+        in.dq = dq;
+        in.dk_acc = c.dk_acc;
+        in.dv_acc = c.dv_acc;
+        msf_status st = msf::launch_bwd_tc(plan, in, s);
+        if (st != MSF_OK) return st;
+    } else {
+        e = msf::launch_bwd_dq_simt(c, a, dq, bf16, s);
         if (e != cudaSuccess) return cuda_status(e);
+        for (int gi = 0; gi < p.n_groups; ++gi) {
+            e = msf::launch_bwd_dkdv_simt(c, bg[gi], bf16, s);
+            if (e != cudaSuccess) return cuda_status(e);
+        }
     }
     return cuda_status(msf::launch_bwd_cast(c, dk_win, dv_win, bf16, s));
+}
+
+extern "C" msf_status msf_mssa_backward(msf_plan_t plan, const void* q, const void* k_win,
+                                        const void* v_win, const void* out, const void* dout,
+                                        const float* lse, void* dq, void* dk_win, void* dv_win,
+                                        void* bwd_ws, size_t bwd_ws_bytes, void* stream) {
+    return mssa_backward(plan, q, k_win, v_win, out, dout, lse, dq, dk_win, dv_win, bwd_ws,
+                         bwd_ws_bytes, stream, true);
+}
+
+extern "C" msf_status msf_mssa_backward_simt(msf_plan_t plan, const void* q, const void* k_win,
+                                             const void* v_win, const void* out, const void* dout,
+                                             const float* lse, void* dq, void* dk_win,
+                                             void* dv_win, void* bwd_ws, size_t bwd_ws_bytes,
+                                             void* stream) {
+    return mssa_backward(plan, q, k_win, v_win, out, dout, lse, dq, dk_win, dv_win, bwd_ws,
+                         bwd_ws_bytes, stream, false);
 }
 
 static msf::MspShape msp_shape(const Plan& p) {

@@ -218,6 +218,16 @@ extern "C" msf_status msf_plan_query(msf_plan_t plan, msf_plan_info* info) {
     info->frames_per_state = p.F;
     info->workspace_bytes = p.ws_bytes;
     info->backward_workspace_bytes = msf::bwd_workspace_bytes(p);
+    {
+        uint64_t f = 0;
+        for (int gi = 0; gi < p.n_groups; ++gi) {
+            const msf::Group& g = p.groups[gi];
+            const uint64_t nkv = (uint64_t)msf::group_nkv(p, gi);
+            const uint64_t cache = (uint64_t)p.d.sink_tokens + (uint64_t)p.hist_count * g.pooled;
+            f += (uint64_t)(g.q_end - g.q_begin) * (6ull * p.D * nkv + 4ull * p.D * (nkv - cache));
+        }
+        info->backward_flops = f * p.H * p.B;
+    }
     info->attention_flops = flops_for(p);
     // Dense reference: every state fine, every query sees sink + history + T*G.
     uint64_t nd = (uint64_t)p.T * p.G;

@@ -36,7 +36,7 @@ EXPORTS = (
     "msf_kv_resample", "msf_mssa_forward", "msf_mssa_forward_simt", "msf_history_append",
     "msf_plan_device_status", "msf_kernel_launches", "msf_unpatchify_noalloc",
     "msf_selftest_wait_timeout", "msf_history_commit", "msf_mssa_forward_lse",
-    "msf_mssa_backward",
+    "msf_mssa_backward", "msf_mssa_backward_simt",
 )
 
 
@@ -72,7 +72,7 @@ class msf_plan_info(ctypes.Structure):
         ("workspace_bytes", ctypes.c_uint64), ("attention_flops", ctypes.c_uint64),
         ("dense_flops", ctypes.c_uint64), ("resample_bytes", ctypes.c_uint64),
         ("pyramid_k_offset", ctypes.c_uint64), ("pyramid_v_offset", ctypes.c_uint64),
-        ("backward_workspace_bytes", ctypes.c_uint64),
+        ("backward_workspace_bytes", ctypes.c_uint64), ("backward_flops", ctypes.c_uint64),
     ]
 
 
@@ -103,6 +103,7 @@ def _load():
         "msf_history_commit": (ctypes.c_int, [P]),
         "msf_mssa_forward_lse": (ctypes.c_int, [P, VP, VP, VP, VP, VP, VP]),
         "msf_mssa_backward": (ctypes.c_int, [P, VP, VP, VP, VP, VP, VP, VP, VP, VP, VP, SZ, VP]),
+        "msf_mssa_backward_simt": (ctypes.c_int, [P, VP, VP, VP, VP, VP, VP, VP, VP, VP, VP, SZ, VP]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -226,6 +227,15 @@ def msf_mssa_backward(plan: int, q, k_win, v_win, out, dout, lse, dq, dk_win, dv
                                   nbytes, _stream(stream)), "msf_mssa_backward")
 
 
+def msf_mssa_backward_simt(plan: int, q, k_win, v_win, out, dout, lse, dq, dk_win, dv_win, bwd_ws,
+                           stream=None) -> None:
+    nbytes = bwd_ws.numel() * bwd_ws.element_size()
+    _check(_lib.msf_mssa_backward_simt(plan, _ptr(q), _ptr(k_win), _ptr(v_win), _ptr(out),
+                                       _ptr(dout), _ptr(lse), _ptr(dq), _ptr(dk_win), _ptr(dv_win),
+                                       _ptr(bwd_ws), nbytes, _stream(stream)),
+           "msf_mssa_backward_simt")
+
+
 def msf_history_commit(plan: int) -> None:
     _check(_lib.msf_history_commit(plan), "msf_history_commit")
 
@@ -322,6 +332,11 @@ class Plan:
                       stream=None):
         msf_mssa_backward(self.handle, q, k_win, v_win, out, dout, lse, dq, dk_win, dv_win, bwd_ws,
                           stream)
+
+    def mssa_backward_simt(self, q, k_win, v_win, out, dout, lse, dq, dk_win, dv_win, bwd_ws,
+                           stream=None):
+        msf_mssa_backward_simt(self.handle, q, k_win, v_win, out, dout, lse, dq, dk_win, dv_win,
+                               bwd_ws, stream)
 
     def backward_workspace(self, device="cuda"):
         import torch

@@ -213,3 +213,13 @@ def test_fused_append_validation_and_state():
     q = _plan((1, 2), 8, 8, 4, 1, cap=2)
     assert lib.msf_history_commit(q.handle) == msf.MSF_ERR_STATE      # not fused
     assert lib.msf_history_commit(None) == msf.MSF_ERR_INVALID_ARG
+
+
+def test_backward_flops_480p():
+    """S, dP and dQ over every query-key pair (6 D flops each), dK and dV over
+    the pairs whose key comes from the window (4 D more); the sink and the
+    history are a detached cache."""
+    info = _plan(synth.LAYER_480P.scales, 30, 52, 1560, 2, H=12, D=128).info
+    g1 = 3120 * (6 * 128 * 8970 + 4 * 128 * (8970 - 1560 - 2 * 1560))
+    g2 = 1170 * (6 * 128 * 4290 + 4 * 128 * (4290 - 1560 - 2 * 390))
+    assert info.backward_flops == 12 * (g1 + g2)

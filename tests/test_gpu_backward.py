@@ -110,3 +110,21 @@ def test_backward_480p_sampled_heads():
     w = synth.LAYER_480P
     x, dout, out, lse, g, _ = _run(w, BF16, 0)
     _check(x, dout, lse, g, w, BF16, 0, heads=[0, 7])
+
+
+@pytest.mark.parametrize("w", [RAGGED, RAGGED64], ids=lambda w: w.name)
+def test_backward_tensor_core_matches_cuda_core(w):
+    """bf16 plans: the tcgen05 backward against the fp32 CUDA-core backward on
+    the same inputs (both checked against the oracle above)."""
+    x, dout, out, lse, g, plan = _run(w, BF16, 0)
+    dx = device_inputs(x, w.history_capacity)
+    bind(plan, dx)
+    plan.kv_resample(dx["k_win"], dx["v_win"])
+    h = {k: torch.full_like(g["dq"], float("nan")) for k in ("dq", "dk", "dv")}
+    plan.mssa_backward_simt(dx["q"], dx["k_win"], dx["v_win"], out, dout.cuda(), lse, h["dq"], h["dk"],
+                            h["dv"], plan.backward_workspace())
+    torch.cuda.synchronize()
+    for k in ("dq", "dk", "dv"):
+        a, b = g[k].float(), h[k].float()
+        scale = b.abs().max().item()
+        assert (a - b).abs().max().item() <= 1e-2 * scale, k
