@@ -355,7 +355,7 @@ extern "C" msf_status msf_mssa_forward(msf_plan_t plan, const void* q, const voi
 // each run with the window token its rows map back to (Eq. 4's Subsample
 // undone by the adjoint). Mirrors the context layout of build_attn_args.
 static void build_bwd_group(const Plan& p, int gi, const void* k_win, const void* v_win,
-                            msf::BwdGroup& bg) {
+                            msf::BwdGroup& bg, int& crow) {
     memset(&bg, 0, sizeof(bg));
     const msf::Group& g = p.groups[gi];
     const size_t row = row_bytes(p);
@@ -376,6 +376,8 @@ static void build_bwd_group(const Plan& p, int gi, const void* k_win, const void
         s.dst0 = dst0;
         s.src_gw = src_gw;
         s.out_gw = out_gw;
+        s.crow0 = crow;
+        crow += len;
     };
     const long long win_bs = (long long)p.N * row;
     const long long pyr_bs = (long long)p.pyr_tokens * row;
@@ -435,8 +437,9 @@ static msf_status mssa_backward(msf_plan_t plan, const void* q, const void* k_wi
     c.out = (const char*)out;
     c.lse = lse;
     c.delta = (float*)bwd_ws;
-    c.dk_acc = (float*)((char*)bwd_ws + msf::bwd_delta_bytes(p));
-    c.dv_acc = (float*)((char*)bwd_ws + msf::bwd_delta_bytes(p) + msf::bwd_acc_bytes(p));
+    c.dk_ctx = (float*)((char*)bwd_ws + msf::bwd_delta_bytes(p));
+    c.dv_ctx = (float*)((char*)bwd_ws + msf::bwd_delta_bytes(p) + msf::bwd_ctx_bytes(p));
+    c.R = msf::bwd_ctx_rows(p);
     c.bstride = (long long)p.N * row_bytes(p);
     c.H = p.H;
     c.D = p.D;
@@ -444,14 +447,39 @@ static msf_status mssa_backward(msf_plan_t plan, const void* q, const void* k_wi
     c.N = p.N;
     c.scale = p.scale;
     c.scale_log2 = p.scale * 1.4426950408889634f;
-    c.mode = p.d.resample;
-    cudaError_t e = cudaMemsetAsync(c.dk_acc, 0, 2 * msf::bwd_acc_bytes(p), s);
-    if (e == cudaSuccess) e = msf::launch_bwd_delta(c, bf16, s);
+    cudaError_t e = msf::launch_bwd_delta(c, bf16, s);
     if (e != cudaSuccess) return cuda_status(e);
     msf::AttnArgs a;
     build_attn_args(p, q, k_win, v_win, (void*)out, a);
     msf::BwdGroup bg[MSF_MAX_GROUPS];
-    for (int gi = 0; gi < p.n_groups; ++gi) build_bwd_group(p, gi, k_win, v_win, bg[gi]);
+    int crow = 0;
+    for (int gi = 0; gi < p.n_groups; ++gi) build_bwd_group(p, gi, k_win, v_win, bg[gi], crow);
+    if (crow != c.R) return MSF_ERR_STATE;
+    // The adjoint of Subsample per window state: the runs of every group
+    // that hold the state, as is (sigma 1) or pooled.
+    msf::GatherArgs ga;
+    memset(&ga, 0, sizeof(ga));
+    ga.T = p.T;
+    ga.mode = p.d.resample;
+    for (int l = 0; l < p.T; ++l) ga.st_off[l] = p.st_off[l];
+    ga.st_off[p.T] = p.N;
+    for (int gi = 0; gi < p.n_groups; ++gi)
+        for (int si = 0; si < bg[gi].n_gseg; ++si) {
+            const msf::GradSeg& gs = bg[gi].gseg[si];
+            for (int l = 0; l < p.T; ++l) {
+                const int lo = p.st_off[l], hi = p.st_off[l] + p.st_n[l];
+                const bool holds = gs.sigma == 1 ? (gs.dst0 <= lo && hi <= gs.dst0 + gs.len)
+                                                 : gs.dst0 == lo;
+                if (!holds) continue;
+                if (ga.n_ent[l] == MSF_MAX_GROUPS) return MSF_ERR_STATE;
+                msf::GatherEntry& en = ga.e[l][ga.n_ent[l]++];
+                en.crow0 = gs.crow0;
+                en.dst0 = gs.dst0;
+                en.sigma = gs.sigma;
+                en.src_gw = gs.src_gw;
+                en.out_gw = gs.out_gw;
+            }
+        }
     if (tc && bf16) {
         msf::BwdTcInput in;
         in.a = &a;
@@ -461,8 +489,9 @@ static msf_status mssa_backward(msf_plan_t plan, const void* q, const void* k_wi
         in.lse = lse;
         in.delta = c.delta;
         in.dq = dq;
-        in.dk_acc = c.dk_acc;
-        in.dv_acc = c.dv_acc;
+        in.dk_ctx = c.dk_ctx;
+        in.dv_ctx = c.dv_ctx;
+        in.R = c.R;
         msf_status st = msf::launch_bwd_tc(plan, in, s);
         if (st != MSF_OK) return st;
     } else {
@@ -473,7 +502,7 @@ static msf_status mssa_backward(msf_plan_t plan, const void* q, const void* k_wi
             if (e != cudaSuccess) return cuda_status(e);
         }
     }
-    return cuda_status(msf::launch_bwd_cast(c, dk_win, dv_win, bf16, s));
+    return cuda_status(msf::launch_bwd_gather(c, ga, dk_win, dv_win, bf16, s));
 }
 
 extern "C" msf_status msf_mssa_backward(msf_plan_t plan, const void* q, const void* k_win,

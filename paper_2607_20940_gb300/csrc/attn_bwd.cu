@@ -8,12 +8,11 @@
 //   dq_i = c sum_j dS_ij k_j,  dk_j = c sum_i dS_ij q_i,  dv_j = sum_i P_ij dO_i
 // dq is computed query by query over the whole context. dk, dv are needed
 // only for context rows that come from the window (the sink and the history
-// are a detached cache in Algorithm 1); they are computed key by key and sent
-// back through the adjoint of Subsample into fp32 accumulators: a row kept as
-// is adds to its window token, a pooled row adds 1/s^2 of itself to each of
-// its s x s source tokens (AVG) or all of itself to the top-left one
-// (STRIDED). Within one group every window token has a single writer; groups
-// run one after another, so the sums are deterministic.
+// are a detached cache in Algorithm 1); they are computed key by key into a
+// buffer of context-row gradients, and a gather kernel applies the adjoint
+// of Subsample: a window token sums the rows that hold it as is and 1/s^2 of
+// each pooled row that covers it (AVG; STRIDED: the pooled row whose
+// top-left it is), over every group, in a fixed order, and rounds once.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <math.h>
@@ -39,26 +38,32 @@ __device__ __forceinline__ __nv_bfloat16 st1(float x) { return __float2bfloat16_
 
 constexpr float kLog2e = 1.4426950408889634f;
 
-// delta[b, h, t] = sum_d dout * out; one warp per (b, t, h) row.
+// delta[b, h, t] = sum_d dout * out: a row of D elements is shared by D/8
+// consecutive threads, each loading 8 elements of both tensors.
 template <typename T, int D>
 __global__ void __launch_bounds__(256) bwd_delta_kernel(const BwdCommon c) {
     ptx::grid_dep_wait();
     ptx::grid_dep_launch();
-    const long long w = (long long)blockIdx.x * 8 + threadIdx.x / 32;
-    const int lane = threadIdx.x % 32;
-    if (w >= (long long)c.B * c.N * c.H) return;
-    const int h = (int)(w % c.H);
-    const int t = (int)((w / c.H) % c.N);
-    const int b = (int)(w / ((long long)c.H * c.N));
-    const size_t off = (size_t)b * c.bstride + ((size_t)t * c.H + h) * D * sizeof(T);
-    const T* go = (const T*)(c.dout + off);
-    const T* o = (const T*)(c.out + off);
+    constexpr int kTpr = D / 8;
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    const long long w = idx / kTpr;
+    const int part = (int)(idx % kTpr);
+    const bool live = w < (long long)c.B * c.N * c.H;
     float acc = 0.f;
+    int b = 0, t = 0, h = 0;
+    if (live) {
+        h = (int)(w % c.H);
+        t = (int)((w / c.H) % c.N);
+        b = (int)(w / ((long long)c.H * c.N));
+        const size_t off = (size_t)b * c.bstride + (((size_t)t * c.H + h) * D + 8 * part) * sizeof(T);
+        const T* go = (const T*)(c.dout + off);
+        const T* o = (const T*)(c.out + off);
 #pragma unroll
-    for (int i = 0; i < D / 32; ++i) acc = fmaf(ld1<T>(go + 32 * i + lane), ld1<T>(o + 32 * i + lane), acc);
+        for (int i = 0; i < 8; ++i) acc = fmaf(ld1<T>(go + i), ld1<T>(o + i), acc);
+    }
 #pragma unroll
-    for (int s = 16; s > 0; s >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, s);
-    if (lane == 0) c.delta[((size_t)b * c.H + h) * c.N + t] = acc;
+    for (int s = kTpr / 2; s > 0; s >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, s);
+    if (live && part == 0) c.delta[((size_t)b * c.H + h) * c.N + t] = acc;
 }
 
 // dq: a block owns 32 queries of one (stream, head, group); four threads share
@@ -136,36 +141,9 @@ __global__ void __launch_bounds__(128) bwd_dq_kernel(const BwdCommon c, const At
     for (int i = 0; i < DP; ++i) o[4 * i + cc] = st1<T>(acc[i] * c.scale);
 }
 
-// Add one context row's fp32 gradient (this thread's DP elements) to the
-// window accumulator through the adjoint of Subsample.
-template <int D>
-__device__ __forceinline__ void scatter_row(float* accb, const GradSeg& gs, int r, int h, int H,
-                                            int cc, const float* val, int mode) {
-    constexpr int DP = D / 4;
-    auto add = [&](int token, float w) {
-        float* dst = accb + ((size_t)token * H + h) * D;
-#pragma unroll
-        for (int i = 0; i < DP; ++i) dst[4 * i + cc] += w * val[i];
-    };
-    if (gs.sigma == 1) {
-        add(gs.dst0 + r, 1.f);
-        return;
-    }
-    const int s = gs.sigma;
-    const int i = r / gs.out_gw, j = r - (r / gs.out_gw) * gs.out_gw;
-    const int base = gs.dst0 + (s * i) * gs.src_gw + s * j;
-    if (mode == MSF_RESAMPLE_STRIDED) {
-        add(base, 1.f);
-        return;
-    }
-    const float w = 1.0f / (float)(s * s);
-    for (int dy = 0; dy < s; ++dy)
-        for (int dx = 0; dx < s; ++dx) add(base + dy * gs.src_gw + dx, w);
-}
-
 // dk, dv of one group's gradient rows: a block owns 32 rows of one segment of
 // one (stream, head); four threads share a row. The group's queries stream
-// through shared memory 32 at a time.
+// through shared memory 32 at a time. Rows go to the context-gradient buffer.
 template <typename T, int D>
 __global__ void __launch_bounds__(128) bwd_dkdv_kernel(const BwdCommon c, const BwdGroup G) {
     ptx::grid_dep_wait();
@@ -236,39 +214,69 @@ __global__ void __launch_bounds__(128) bwd_dkdv_kernel(const BwdCommon c, const 
         }
     }
     if (!valid) return;
+    const size_t o = (((size_t)b * c.R + gs.crow0 + r) * c.H + h) * D;
 #pragma unroll
-    for (int e = 0; e < DP; ++e) dk[e] *= c.scale;
-    const size_t accb = (size_t)b * c.N * c.H * D;
-    scatter_row<D>(c.dk_acc + accb, gs, r, h, c.H, cc, dk, c.mode);
-    scatter_row<D>(c.dv_acc + accb, gs, r, h, c.H, cc, dv, c.mode);
+    for (int e = 0; e < DP; ++e) {
+        c.dk_ctx[o + 4 * e + cc] = dk[e] * c.scale;
+        c.dv_ctx[o + 4 * e + cc] = dv[e];
+    }
 }
 
-template <typename T>
-__global__ void __launch_bounds__(256) bwd_cast_kernel(const float* __restrict__ a,
-                                                        const float* __restrict__ bsrc,
-                                                        T* __restrict__ oa, T* __restrict__ ob,
-                                                        long long n4) {
+// dk_win, dv_win: one warp per (stream, token, head) row; a lane holds D/32
+// consecutive elements. Entries of the token's state come in a fixed order.
+template <typename T, int D>
+__global__ void __launch_bounds__(256) bwd_gather_kernel(const BwdCommon c, const GatherArgs g,
+                                                         T* __restrict__ dk, T* __restrict__ dv) {
     ptx::grid_dep_wait();
     ptx::grid_dep_launch();
-    const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-    if (i >= n4) return;
-    const float4 x = reinterpret_cast<const float4*>(a)[i];
-    const float4 y = reinterpret_cast<const float4*>(bsrc)[i];
-    oa[4 * i] = st1<T>(x.x);
-    oa[4 * i + 1] = st1<T>(x.y);
-    oa[4 * i + 2] = st1<T>(x.z);
-    oa[4 * i + 3] = st1<T>(x.w);
-    ob[4 * i] = st1<T>(y.x);
-    ob[4 * i + 1] = st1<T>(y.y);
-    ob[4 * i + 2] = st1<T>(y.z);
-    ob[4 * i + 3] = st1<T>(y.w);
+    constexpr int E = D / 32;
+    const long long w = (long long)blockIdx.x * 8 + threadIdx.x / 32;
+    const int lane = threadIdx.x % 32;
+    if (w >= (long long)c.B * c.N * c.H) return;
+    const int h = (int)(w % c.H);
+    const int t = (int)((w / c.H) % c.N);
+    const int b = (int)(w / ((long long)c.H * c.N));
+    int l = 0;
+    while (l + 1 < g.T && t >= g.st_off[l + 1]) ++l;
+    float ak[E], av[E];
+#pragma unroll
+    for (int e = 0; e < E; ++e) ak[e] = av[e] = 0.f;
+    for (int k = 0; k < g.n_ent[l]; ++k) {
+        const GatherEntry& en = g.e[l][k];
+        int row;
+        float wgt = 1.f;
+        if (en.sigma == 1) {
+            row = en.crow0 + (t - en.dst0);
+        } else {
+            const int s = en.sigma, loc = t - en.dst0;
+            const int i = loc / en.src_gw, j = loc - (loc / en.src_gw) * en.src_gw;
+            if (g.mode == MSF_RESAMPLE_STRIDED) {
+                if (i % s || j % s) continue;
+            } else {
+                wgt = 1.0f / (float)(s * s);
+            }
+            row = en.crow0 + (i / s) * en.out_gw + j / s;
+        }
+        const size_t o = (((size_t)b * c.R + row) * c.H + h) * D + E * lane;
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+            ak[e] = fmaf(wgt, c.dk_ctx[o + e], ak[e]);
+            av[e] = fmaf(wgt, c.dv_ctx[o + e], av[e]);
+        }
+    }
+    const size_t o = (((size_t)b * c.N + t) * c.H + h) * D + E * lane;
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+        dk[o + e] = st1<T>(ak[e]);
+        dv[o + e] = st1<T>(av[e]);
+    }
 }
 
 }  // namespace
 
 cudaError_t launch_bwd_delta(const BwdCommon& c, bool bf16, cudaStream_t st) {
-    const long long rows = (long long)c.B * c.N * c.H;
-    dim3 grid((unsigned)((rows + 7) / 8));
+    const long long threads = (long long)c.B * c.N * c.H * (c.D / 8);
+    dim3 grid((unsigned)((threads + 255) / 256));
     if (c.D == 128)
         return bf16 ? launch_pdl(bwd_delta_kernel<__nv_bfloat16, 128>, grid, dim3(256), 0, st, c)
                     : launch_pdl(bwd_delta_kernel<float, 128>, grid, dim3(256), 0, st, c);
@@ -304,14 +312,19 @@ cudaError_t launch_bwd_dkdv_simt(const BwdCommon& c, const BwdGroup& g, bool bf1
                 : launch_pdl(bwd_dkdv_kernel<float, 64>, grid, dim3(128), 0, st, c, g);
 }
 
-cudaError_t launch_bwd_cast(const BwdCommon& c, void* dk, void* dv, bool bf16, cudaStream_t st) {
-    const long long n4 = (long long)c.B * c.N * c.H * c.D / 4;
-    dim3 grid((unsigned)((n4 + 255) / 256));
-    if (bf16)
-        return launch_pdl(bwd_cast_kernel<__nv_bfloat16>, grid, dim3(256), 0, st, (const float*)c.dk_acc,
-                          (const float*)c.dv_acc, (__nv_bfloat16*)dk, (__nv_bfloat16*)dv, n4);
-    return launch_pdl(bwd_cast_kernel<float>, grid, dim3(256), 0, st, (const float*)c.dk_acc,
-                      (const float*)c.dv_acc, (float*)dk, (float*)dv, n4);
+cudaError_t launch_bwd_gather(const BwdCommon& c, const GatherArgs& g, void* dk, void* dv,
+                              bool bf16, cudaStream_t st) {
+    const long long rows = (long long)c.B * c.N * c.H;
+    dim3 grid((unsigned)((rows + 7) / 8));
+    if (c.D == 128)
+        return bf16 ? launch_pdl(bwd_gather_kernel<__nv_bfloat16, 128>, grid, dim3(256), 0, st, c, g,
+                                 (__nv_bfloat16*)dk, (__nv_bfloat16*)dv)
+                    : launch_pdl(bwd_gather_kernel<float, 128>, grid, dim3(256), 0, st, c, g, (float*)dk,
+                                 (float*)dv);
+    return bf16 ? launch_pdl(bwd_gather_kernel<__nv_bfloat16, 64>, grid, dim3(256), 0, st, c, g,
+                             (__nv_bfloat16*)dk, (__nv_bfloat16*)dv)
+                : launch_pdl(bwd_gather_kernel<float, 64>, grid, dim3(256), 0, st, c, g, (float*)dk,
+                             (float*)dv);
 }
 
 }  // namespace msf

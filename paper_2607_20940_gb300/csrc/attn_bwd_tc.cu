@@ -9,23 +9,29 @@
 // bwd_dq_tc_kernel: one CTA per 128-row query tile of one (stream, head,
 //   group). It walks the group's whole context (sink, history or pyramid
 //   part, window suffix) in 128-row K/V tiles:
-//     S = Q K^T (SS), dP = dO V^T (SS)              -> TMEM
-//     softmax warps: P, dS (bf16, over S's columns)  -> TMEM
-//     dQ += dS K (TS, K read MN-major)              -> TMEM
+//     S = Q K^T (SS, two buffers), dP = dO V^T (SS)  -> TMEM
+//     softmax warps: P, dS (bf16, over S's columns)   -> TMEM
+//     dQ += dS K (TS, K read MN-major)               -> TMEM
 //   then scales dQ by c and stores it.
 // bwd_dkdv_tc_kernel: one CTA per 128-row tile of context rows that come
-//   from the window (one group per launch). It walks the group's queries in
-//   128-row tiles:
+//   from the window, every group in one launch. It walks its group's
+//   queries in 128-row tiles:
 //     S^T = K Q^T (SS), dP^T = V dO^T (SS)            -> TMEM (lanes = keys)
 //     softmax warps: P^T, dS^T (bf16, over S^T/dP^T)  -> TMEM
 //     dV += P^T dO (TS), dK += dS^T Q (TS)           -> TMEM
-//   then sends c dK and dV through the adjoint of Subsample into the fp32
-//   window accumulators; each window token has one writer per launch.
+//   then writes c dK and dV (fp32) to its rows of the context-gradient
+//   buffers, staged through shared memory so that every warp stores whole
+//   rows. A gather kernel applies the adjoint of Subsample afterwards.
 //
-// Roles (256 threads): warp 0 TMA producer, warp 1 MMA issuer (warp-wide
-// loop, one elected lane issues), warp 2 TMEM allocation, warps 4-7 one
-// thread per TMEM lane (query row or key row). TMEM columns: S [0,128),
-// dP [128,256), then dQ (or dV, dK) from 256. The tensor pipe executes MMAs
+// Roles (384 threads): warp 0 TMA producer, warp 1 MMA issuer (warp-wide
+// loop, one elected lane issues), warp 2 TMEM allocation, warps 4-11 the
+// softmax: a thread per TMEM lane (query row or key row) and column half,
+// warps 4-7 columns 0-63, warps 8-11 columns 64-127. Each half writes its
+// bf16 P / dS into its own columns (the MMA that reads them takes its A
+// operand per 16-column step), so the halves never wait for each other.
+// TMEM columns of the dK/dV
+// kernel: S^T [0,128), dP^T [128,256), dV, dK from 256 (the dQ kernel's
+// layout is given with it). The tensor pipe executes MMAs
 // in issue order, so an MMA that overwrites S or dP never overtakes the MMA
 // that reads the bf16 P or dS stored there. Every wait is bounded.
 #include <cuda.h>
@@ -42,7 +48,7 @@ namespace msf {
 namespace {
 
 constexpr int kBM = 128;       // rows of every Q / dO / K / V tile
-constexpr int kThreads = 256;  // 8 warps
+constexpr int kThreads = 384;  // 12 warps
 constexpr long long kWaitLimit = 2000000000LL;  // ~1 s of SM clock
 constexpr float kLog2e = 1.4426950408889634f;
 
@@ -58,7 +64,14 @@ struct BGroupQ {
 };
 struct BGrad {
     int map, row0, len, kt0;  // row0 relative to the map; kt0 = first key tile of the run
-    int sigma, dst0, src_gw, out_gw;
+    int crow0;                // first row of the run in the context-gradient buffers
+};
+struct BGroupK {
+    int q_begin, q_end, n_qt;
+    int item_base;  // first item of this group
+    int n_kt;       // key tiles of this group (all runs)
+    int n_grad;
+    BGrad gr[kMaxGradSeg];
 };
 struct BwdTcParams {
     int H, B, N;
@@ -66,17 +79,17 @@ struct BwdTcParams {
     const float* lse;
     const float* delta;
     __nv_bfloat16* dq;
-    float* dk_acc;
-    float* dv_acc;
-    int mode;
+    float* dk_ctx;
+    float* dv_ctx;
+    int R;  // rows per stream of the context-gradient buffers
     unsigned int* status;
     long long wait_limit;
     // bwd_dq_tc_kernel
     int n_groups;
     BGroupQ g[MSF_MAX_GROUPS];
-    // bwd_dkdv_tc_kernel (one group)
-    int q_begin, q_end, n_qt, n_grad;
-    BGrad gr[kMaxGradSeg];
+    // bwd_dkdv_tc_kernel
+    int n_kgroups;
+    BGroupK kg[MSF_MAX_GROUPS];
 };
 struct BwdMaps {
     CUtensorMap q, dout;
@@ -114,19 +127,33 @@ __device__ __forceinline__ void load_tile(unsigned char* dst, const CUtensorMap*
 }
 
 // ============================================================== dQ kernel
+//
+// TMEM: S for even tiles [0,128), S for odd tiles [128,256), dP [256,384),
+// dQ from 384. Smem: Q, dO, a 3-deep K ring, a 2-deep V ring. The softmax
+// warps first copy dP_j into registers and release it, so dP_{j+1} (and
+// S_{j+1}, issued a tile ahead into the other S buffer) run on the tensor
+// pipe while they compute dS_j; dQ_j and S_{j+2} then run while the softmax
+// works on tile j+1.
+
+template <int D>
+struct QCfg {
+    static constexpr int kTile = kBM * D * 2;
+    static constexpr int kSmem = 7 * kTile + 1024 > 120 * 1024 ? 7 * kTile + 1024 : 120 * 1024;
+};
 
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     bwd_dq_tc_kernel(const __grid_constant__ BwdMaps maps, const __grid_constant__ BwdTcParams p) {
-    using C = BCfg<D>;
+    using C = QCfg<D>;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     unsigned char* sQ = smem;
     unsigned char* sG = smem + C::kTile;       // dO
-    unsigned char* sK = smem + 2 * C::kTile;   // [2]
-    unsigned char* sV = smem + 4 * C::kTile;   // [2]
+    unsigned char* sK = smem + 2 * C::kTile;   // [3]
+    unsigned char* sV = smem + 5 * C::kTile;   // [2]
 
-    __shared__ uint64_t qg_full, kv_full[2], kv_empty[2], st_full, ds_full, dq_full, drain_bar;
+    __shared__ uint64_t qg_full, k_full[3], k_empty[3], v_full[2], v_empty[2];
+    __shared__ uint64_t sdp_full, dp_free, ds_full, dq_full, drain_bar;
     __shared__ uint32_t tmem_base_sh;
     __shared__ int abort_flag;
 
@@ -144,12 +171,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         abort_flag = 0;
         ptx::mbar_init(&qg_full, 1);
-        for (int s = 0; s < 2; ++s) {
-            ptx::mbar_init(&kv_full[s], 1);
-            ptx::mbar_init(&kv_empty[s], 1);
+        for (int s = 0; s < 3; ++s) {
+            ptx::mbar_init(&k_full[s], 1);
+            ptx::mbar_init(&k_empty[s], 1);
         }
-        ptx::mbar_init(&st_full, 1);
-        ptx::mbar_init(&ds_full, 4);
+        for (int s = 0; s < 2; ++s) {
+            ptx::mbar_init(&v_full[s], 1);
+            ptx::mbar_init(&v_empty[s], 1);
+        }
+        ptx::mbar_init(&sdp_full, 1);
+        ptx::mbar_init(&dp_free, 8);
+        ptx::mbar_init(&ds_full, 8);
         ptx::mbar_init(&dq_full, 1);
         ptx::mbar_init(&drain_bar, 1);
         ptx::fence_mbar_init();
@@ -183,24 +215,35 @@ __global__ void __launch_bounds__(kThreads, 1)
             ptx::mbar_arrive_expect_tx(&qg_full, 2 * C::kTile);
             load_tile<D>(sQ, &maps.q, &qg_full, h, q_row0, b);
             load_tile<D>(sG, &maps.dout, &qg_full, h, q_row0, b);
-            int j = 0;
+            int j = 0, nk = 0, nv = 0;
             for (; j < n; ++j) {
                 int seg, row, valid;
                 tile_of(j, seg, row, valid);
-                const int st = j & 1;
-                if (!ptx::mbar_wait_bounded(&kv_empty[st], (uint32_t)(((j >> 1) & 1) ^ 1), abort_p,
+                const int ks = j % 3, vs = j & 1;
+                if (!ptx::mbar_wait_bounded(&k_empty[ks], (uint32_t)(((j / 3) & 1) ^ 1), abort_p,
                                             p.wait_limit)) {
                     ok = false;
                     break;
                 }
-                ptx::mbar_arrive_expect_tx(&kv_full[st], 2 * C::kTile);
-                load_tile<D>(sK + st * C::kTile, &maps.k[G.seg[seg].map], &kv_full[st], h, row, b);
-                load_tile<D>(sV + st * C::kTile, &maps.v[G.seg[seg].map], &kv_full[st], h, row, b);
+                ptx::mbar_arrive_expect_tx(&k_full[ks], C::kTile);
+                load_tile<D>(sK + ks * C::kTile, &maps.k[G.seg[seg].map], &k_full[ks], h, row, b);
+                ++nk;
+                if (!ptx::mbar_wait_bounded(&v_empty[vs], (uint32_t)(((j >> 1) & 1) ^ 1), abort_p,
+                                            p.wait_limit)) {
+                    ok = false;
+                    break;
+                }
+                ptx::mbar_arrive_expect_tx(&v_full[vs], C::kTile);
+                load_tile<D>(sV + vs * C::kTile, &maps.v[G.seg[seg].map], &v_full[vs], h, row, b);
+                ++nv;
             }
             if (!ok) {
+                // every copy issued lands before the CTA exits
                 ptx::mbar_wait_bounded(&qg_full, 0, &never, kWaitLimit);
-                for (int jj = (j > 2 ? j - 2 : 0); jj < j; ++jj)
-                    ptx::mbar_wait_bounded(&kv_full[jj & 1], (uint32_t)((jj >> 1) & 1), &never, kWaitLimit);
+                for (int jj = (nk > 3 ? nk - 3 : 0); jj < nk; ++jj)
+                    ptx::mbar_wait_bounded(&k_full[jj % 3], (uint32_t)((jj / 3) & 1), &never, kWaitLimit);
+                for (int jj = (nv > 2 ? nv - 2 : 0); jj < nv; ++jj)
+                    ptx::mbar_wait_bounded(&v_full[jj & 1], (uint32_t)((jj >> 1) & 1), &never, kWaitLimit);
                 atomicOr(p.status, kDevTimeout);
             }
         }
@@ -218,38 +261,69 @@ __global__ void __launch_bounds__(kThreads, 1)
             const bool r = ptx::mbar_wait_bounded(bar, parity, abort_p, p.wait_limit);
             return __all_sync(0xffffffffu, r);
         };
-        bool ok = wait_all(&qg_full, 0);
-        for (int j = 0; j < n && ok; ++j) {
-            const int st = j & 1;
-            ok = wait_all(&kv_full[st], (uint32_t)((j >> 1) & 1));
-            if (!ok) break;
+        auto issue_s = [&](int j) {  // S_j = Q K_j^T into the S buffer of j's parity
+            const uint64_t kd = k_desc + (uint64_t)(j % 3) * kTileDesc;
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk)
+                ptx::mma_ss(tbase + (j & 1) * 128, q_desc + kmajor_step(kk), kd + kmajor_step(kk), idS,
+                            kk > 0 ? 1u : 0u);
+        };
+        auto issue_dp = [&](int j) {  // dP_j = dO V_j^T
+            const uint64_t vd = v_desc + (uint64_t)(j & 1) * kTileDesc;
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk)
+                ptx::mma_ss(tbase + 256, g_desc + kmajor_step(kk), vd + kmajor_step(kk), idS,
+                            kk > 0 ? 1u : 0u);
+            ptx::mma_commit(&v_empty[j & 1]);
+            ptx::mma_commit(&sdp_full);
+        };
+        bool ok = wait_all(&qg_full, 0) && wait_all(&k_full[0], 0) && wait_all(&v_full[0], 0);
+        if (ok) {
             ptx::tc_fence_after();
             if (ptx::elect_one_sync()) {
-                const uint64_t kd = k_desc + (uint64_t)st * kTileDesc;
-                const uint64_t vd = v_desc + (uint64_t)st * kTileDesc;
-#pragma unroll
-                for (int kk = 0; kk < D / 16; ++kk)
-                    ptx::mma_ss(tbase, q_desc + kmajor_step(kk), kd + kmajor_step(kk), idS, kk > 0 ? 1u : 0u);
-#pragma unroll
-                for (int kk = 0; kk < D / 16; ++kk)
-                    ptx::mma_ss(tbase + 128, g_desc + kmajor_step(kk), vd + kmajor_step(kk), idS,
-                                kk > 0 ? 1u : 0u);
-                ptx::mma_commit(&st_full);
+                issue_s(0);
+                issue_dp(0);
             }
             __syncwarp();
+            if (n > 1) {
+                ok = wait_all(&k_full[1], 0);
+                if (ok) {
+                    ptx::tc_fence_after();
+                    if (ptx::elect_one_sync()) issue_s(1);
+                    __syncwarp();
+                }
+            }
+        }
+        for (int j = 0; j < n && ok; ++j) {
+            ok = wait_all(&dp_free, (uint32_t)(j & 1));
+            if (!ok) break;
+            if (j + 1 < n) {
+                ok = wait_all(&v_full[(j + 1) & 1], (uint32_t)(((j + 1) >> 1) & 1));
+                if (!ok) break;
+                ptx::tc_fence_after();
+                if (ptx::elect_one_sync()) issue_dp(j + 1);
+                __syncwarp();
+            }
             ok = wait_all(&ds_full, (uint32_t)(j & 1));
             if (!ok) break;
             ptx::tc_fence_after();
             if (ptx::elect_one_sync()) {
-                const uint64_t kd = kmn_desc + (uint64_t)st * kTileDesc;
+                const uint64_t kd = kmn_desc + (uint64_t)(j % 3) * kTileDesc;
 #pragma unroll
                 for (int kk = 0; kk < kBM / 16; ++kk)
-                    ptx::mma_ts(tbase + 256, tbase + kk * 8, kd + (uint64_t)(kk * (2048 >> 4)), idQ,
-                                (j > 0 || kk > 0) ? 1u : 0u);
-                ptx::mma_commit(&kv_empty[st]);
+                    ptx::mma_ts(tbase + 384, tbase + (j & 1) * 128 + 64 * (kk / 4) + (kk % 4) * 8,
+                                kd + (uint64_t)(kk * (2048 >> 4)), idQ, (j > 0 || kk > 0) ? 1u : 0u);
+                ptx::mma_commit(&k_empty[j % 3]);
                 if (j + 1 == n) ptx::mma_commit(&dq_full);
             }
             __syncwarp();
+            if (j + 2 < n) {
+                ok = wait_all(&k_full[(j + 2) % 3], (uint32_t)(((j + 2) / 3) & 1));
+                if (!ok) break;
+                ptx::tc_fence_after();
+                if (ptx::elect_one_sync()) issue_s(j + 2);
+                __syncwarp();
+            }
         }
         if (!ok) {
             if (ptx::elect_one_sync()) ptx::mma_commit(&drain_bar);
@@ -258,43 +332,64 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (lane == 0) atomicOr(p.status, kDevTimeout);
         }
     } else if (warp >= 4) {
-        // ===================== softmax: one thread per query row =====================
+        // ============ softmax: one thread per query row and column half ============
+        const int half = (warp - 4) / 4;
         const int wq = warp % 4;
         const int r = wq * 32 + lane;
         const uint32_t lane_off = (uint32_t)(wq * 32) << 16;
-        const uint32_t tS = tbase + lane_off, tP = tbase + 128 + lane_off, tQ = tbase + 256 + lane_off;
+        const uint32_t tP = tbase + 256 + 64 * half + lane_off;
         const int q = q_row0 + r;
         const bool qv = q < G.q_end;
         const size_t rix = ((size_t)b * p.H + h) * p.N + (qv ? q : 0);
         const float nl = qv ? -p.lse[rix] * kLog2e : -INFINITY;  // -lse in log2 units
         const float dl = qv ? p.delta[rix] : 0.f;
-        const float sl2 = p.scale_log2;
+        const uint64_t sl2x2 = ptx::f2_pack(p.scale_log2, p.scale_log2), nlx2 = ptx::f2_pack(nl, nl);
+        const uint64_t ndlx2 = ptx::f2_pack(-dl, -dl);
         bool ok = true;
         for (int j = 0; j < n && ok; ++j) {
             int seg, row, valid;
             tile_of(j, seg, row, valid);
-            ok = __all_sync(0xffffffffu, ptx::mbar_wait_bounded(&st_full, (uint32_t)(j & 1), abort_p,
+            ok = __all_sync(0xffffffffu, ptx::mbar_wait_bounded(&sdp_full, (uint32_t)(j & 1), abort_p,
                                                                 p.wait_limit));
             if (!ok) break;
             ptx::tc_fence_after();
+            // this half's dP_j into registers, then release its columns
+            uint32_t dp[2][32];
+            ptx::tmem_ld32(tP, dp[0]);
+            ptx::tmem_ld32(tP + 32, dp[1]);
+            ptx::tmem_wait_ld();
+            ptx::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&dp_free);
+            const uint32_t tS = tbase + (j & 1) * 128 + 64 * half + lane_off;
 #pragma unroll
-            for (int c4 = 0; c4 < 4; ++c4) {
-                uint32_t s[32], dp[32];
-                ptx::tmem_ld32(tS + 32 * c4, s);
-                ptx::tmem_ld32(tP + 32 * c4, dp);
+            for (int c2 = 0; c2 < 2; ++c2) {
+                uint32_t s[32];
+                ptx::tmem_ld32(tS + 32 * c2, s);
                 ptx::tmem_wait_ld();
+                const int lim = valid - (64 * half + 32 * c2);
+                if (lim < 32) {
+                    // keys past the segment's end: score -inf, probability 0
+#pragma unroll
+                    for (int e = 0; e < 32; ++e)
+                        if (e >= lim) s[e] = 0xff800000u;
+                }
                 uint32_t pk[16];
 #pragma unroll
                 for (int e = 0; e < 16; ++e) {
-                    const int c0 = 32 * c4 + 2 * e;
-                    float p0 = ex2(fmaf(__uint_as_float(s[2 * e]), sl2, nl));
-                    float p1 = ex2(fmaf(__uint_as_float(s[2 * e + 1]), sl2, nl));
-                    if (c0 >= valid) p0 = 0.f;
-                    if (c0 + 1 >= valid) p1 = 0.f;
-                    pk[e] = ptx::pack_bf16(p0 * (__uint_as_float(dp[2 * e]) - dl),
-                                           p1 * (__uint_as_float(dp[2 * e + 1]) - dl));
+                    const uint64_t arg = ptx::f2_fma(
+                        ptx::f2_pack(__uint_as_float(s[2 * e]), __uint_as_float(s[2 * e + 1])), sl2x2, nlx2);
+                    float a0, a1;
+                    ptx::f2_unpack(arg, a0, a1);
+                    const uint64_t pp = ptx::f2_pack(ex2(a0), ex2(a1));
+                    const uint64_t dd = ptx::f2_add(
+                        ptx::f2_pack(__uint_as_float(dp[c2][2 * e]), __uint_as_float(dp[c2][2 * e + 1])), ndlx2);
+                    const uint64_t ds = ptx::f2_mul(pp, dd);
+                    float d0, d1;
+                    ptx::f2_unpack(ds, d0, d1);
+                    pk[e] = ptx::pack_bf16(d0, d1);
                 }
-                ptx::tmem_st16(tS + 16 * c4, pk);
+                ptx::tmem_st16(tS + 16 * c2, pk);
             }
             ptx::tmem_wait_st();
             ptx::tc_fence_before();
@@ -303,10 +398,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (ok) ok = __all_sync(0xffffffffu, ptx::mbar_wait_bounded(&dq_full, 0, abort_p, p.wait_limit));
         if (ok) {
+            // each half stores D/2 columns of its row
             ptx::tc_fence_after();
-            __nv_bfloat16* dst = p.dq + (((size_t)b * p.N + (qv ? q : 0)) * p.H + h) * D;
+            constexpr int DH = D / 2;
+            const uint32_t tQ = tbase + 384 + DH * half + lane_off;
+            __nv_bfloat16* dst = p.dq + (((size_t)b * p.N + (qv ? q : 0)) * p.H + h) * D + DH * half;
 #pragma unroll
-            for (int c = 0; c < D / 32; ++c) {
+            for (int c = 0; c < DH / 32; ++c) {
                 uint32_t o[32];
                 ptx::tmem_ld32(tQ + 32 * c, o);
                 ptx::tmem_wait_ld();
@@ -336,39 +434,6 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // ============================================================ dK/dV kernel
 
-// Add one key row's gradient (D fp32 values) to the window accumulator
-// through the adjoint of Subsample.
-template <int D>
-__device__ __forceinline__ void scatter_row_tc(float* accb, const BGrad& gr, int rr, int h, int H,
-                                               const float* val, int mode) {
-    auto add = [&](int token, float w) {
-        float4* dst = reinterpret_cast<float4*>(accb + ((size_t)token * H + h) * D);
-#pragma unroll
-        for (int i = 0; i < D / 4; ++i) {
-            float4 x = dst[i];
-            x.x = fmaf(w, val[4 * i], x.x);
-            x.y = fmaf(w, val[4 * i + 1], x.y);
-            x.z = fmaf(w, val[4 * i + 2], x.z);
-            x.w = fmaf(w, val[4 * i + 3], x.w);
-            dst[i] = x;
-        }
-    };
-    if (gr.sigma == 1) {
-        add(gr.dst0 + rr, 1.f);
-        return;
-    }
-    const int s = gr.sigma;
-    const int i = rr / gr.out_gw, j = rr - (rr / gr.out_gw) * gr.out_gw;
-    const int base = gr.dst0 + (s * i) * gr.src_gw + s * j;
-    if (mode == MSF_RESAMPLE_STRIDED) {
-        add(base, 1.f);
-        return;
-    }
-    const float w = 1.0f / (float)(s * s);
-    for (int dy = 0; dy < s; ++dy)
-        for (int dx = 0; dx < s; ++dx) add(base + dy * gr.src_gw + dx, w);
-}
-
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     bwd_dkdv_tc_kernel(const __grid_constant__ BwdMaps maps, const __grid_constant__ BwdTcParams p) {
@@ -386,17 +451,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     __shared__ float sL[2][kBM], sD[2][kBM];
 
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-    const int n_kt_items = p.gr[p.n_grad - 1].kt0 + (p.gr[p.n_grad - 1].len + kBM - 1) / kBM;
-    const int kt_all = (int)blockIdx.x % n_kt_items;
-    const int h = ((int)blockIdx.x / n_kt_items) % p.H;
-    const int b = (int)blockIdx.x / (n_kt_items * p.H);
+    int kgi = 0;
+    while (kgi + 1 < p.n_kgroups && (int)blockIdx.x >= p.kg[kgi + 1].item_base) ++kgi;
+    const BGroupK& KG = p.kg[kgi];
+    const int local = (int)blockIdx.x - KG.item_base;
+    const int kt_all = local % KG.n_kt;
+    const int h = (local / KG.n_kt) % p.H;
+    const int b = local / (KG.n_kt * p.H);
     int gsi = 0;
-    while (gsi + 1 < p.n_grad && kt_all >= p.gr[gsi + 1].kt0) ++gsi;
-    const BGrad& gr = p.gr[gsi];
+    while (gsi + 1 < KG.n_grad && kt_all >= KG.gr[gsi + 1].kt0) ++gsi;
+    const BGrad& gr = KG.gr[gsi];
     const int kt = kt_all - gr.kt0;
     const int key_row = gr.row0 + kt * kBM;
     const int valid_keys = min(kBM, gr.len - kt * kBM);
-    const int nq = p.n_qt;
+    const int nq = KG.n_qt;
 
     if (threadIdx.x == 0) {
         abort_flag = 0;
@@ -406,7 +474,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             ptx::mbar_init(&qg_empty[s], 1);
         }
         ptx::mbar_init(&st_full, 1);
-        ptx::mbar_init(&pds_full, 4);
+        ptx::mbar_init(&pds_full, 8);
         ptx::mbar_init(&kv_done, 1);
         ptx::mbar_init(&drain_bar, 1);
         ptx::fence_mbar_init();
@@ -440,8 +508,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     break;
                 }
                 ptx::mbar_arrive_expect_tx(&qg_full[st], 2 * C::kTile);
-                load_tile<D>(sQ + st * C::kTile, &maps.q, &qg_full[st], h, p.q_begin + i * kBM, b);
-                load_tile<D>(sG + st * C::kTile, &maps.dout, &qg_full[st], h, p.q_begin + i * kBM, b);
+                load_tile<D>(sQ + st * C::kTile, &maps.q, &qg_full[st], h, KG.q_begin + i * kBM, b);
+                load_tile<D>(sG + st * C::kTile, &maps.dout, &qg_full[st], h, KG.q_begin + i * kBM, b);
             }
             if (!ok) {
                 ptx::mbar_wait_bounded(&kv_full, 0, &never, kWaitLimit);
@@ -492,12 +560,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint64_t qd = qmn_desc + (uint64_t)st * kTileDesc;
 #pragma unroll
                 for (int kk = 0; kk < kBM / 16; ++kk)
-                    ptx::mma_ts(tbase + 256, tbase + kk * 8, gd + (uint64_t)(kk * (2048 >> 4)), idO,
-                                (i > 0 || kk > 0) ? 1u : 0u);
+                    ptx::mma_ts(tbase + 256, tbase + 64 * (kk / 4) + (kk % 4) * 8,
+                                gd + (uint64_t)(kk * (2048 >> 4)), idO, (i > 0 || kk > 0) ? 1u : 0u);
 #pragma unroll
                 for (int kk = 0; kk < kBM / 16; ++kk)
-                    ptx::mma_ts(tbase + 256 + D, tbase + 128 + kk * 8, qd + (uint64_t)(kk * (2048 >> 4)),
-                                idO, (i > 0 || kk > 0) ? 1u : 0u);
+                    ptx::mma_ts(tbase + 256 + D, tbase + 128 + 64 * (kk / 4) + (kk % 4) * 8,
+                                qd + (uint64_t)(kk * (2048 >> 4)), idO, (i > 0 || kk > 0) ? 1u : 0u);
                 ptx::mma_commit(&qg_empty[st]);
                 if (i + 1 == nq) ptx::mma_commit(&kv_done);
             }
@@ -510,47 +578,61 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (lane == 0) atomicOr(p.status, kDevTimeout);
         }
     } else if (warp >= 4) {
-        // ====================== softmax: one thread per key row ======================
+        // ============= softmax: one thread per key row and column half =============
+        const int half = (warp - 4) / 4;
         const int wq = warp % 4;
         const int r = wq * 32 + lane;
+        const int tix = (warp - 4) * 32 + lane;  // 0..255
         const uint32_t lane_off = (uint32_t)(wq * 32) << 16;
-        const uint32_t tS = tbase + lane_off, tP = tbase + 128 + lane_off;
-        const float sl2 = p.scale_log2;
+        const uint32_t tS = tbase + 64 * half + lane_off, tP = tbase + 128 + 64 * half + lane_off;
+        const uint64_t sl2x2 = ptx::f2_pack(p.scale_log2, p.scale_log2);
         bool ok = true;
         for (int i = 0; i < nq && ok; ++i) {
-            // this tile's per-query statistics, shared by the 128 key rows
+            // this tile's per-query statistics, shared by the 128 key rows:
+            // threads 0-127 load -lse (log2 units), 128-255 delta
             {
-                const int q = p.q_begin + i * kBM + r;
-                const bool qv = q < p.q_end;
+                const int qq = tix & 127;
+                const int q = KG.q_begin + i * kBM + qq;
+                const bool qv = q < KG.q_end;
                 const size_t rix = ((size_t)b * p.H + h) * p.N + (qv ? q : 0);
-                sL[i & 1][r] = qv ? -p.lse[rix] * kLog2e : -INFINITY;
-                sD[i & 1][r] = qv ? p.delta[rix] : 0.f;
+                if (tix < 128)
+                    sL[i & 1][qq] = qv ? -p.lse[rix] * kLog2e : -INFINITY;
+                else
+                    sD[i & 1][qq] = qv ? -p.delta[rix] : 0.f;
             }
-            ptx::named_bar_sync(1, 128);
-            const float* L = sL[i & 1];
-            const float* Dl = sD[i & 1];
+            ptx::named_bar_sync(1, 256);
+            const float* L = sL[i & 1] + 64 * half;
+            const float* ND = sD[i & 1] + 64 * half;
             ok = __all_sync(0xffffffffu, ptx::mbar_wait_bounded(&st_full, (uint32_t)(i & 1), abort_p,
                                                                 p.wait_limit));
             if (!ok) break;
             ptx::tc_fence_after();
 #pragma unroll
-            for (int c4 = 0; c4 < 4; ++c4) {
+            for (int c2 = 0; c2 < 2; ++c2) {
                 uint32_t s[32], dp[32];
-                ptx::tmem_ld32(tS + 32 * c4, s);
-                ptx::tmem_ld32(tP + 32 * c4, dp);
+                ptx::tmem_ld32(tS + 32 * c2, s);
+                ptx::tmem_ld32(tP + 32 * c2, dp);
                 ptx::tmem_wait_ld();
                 uint32_t pp[16], pd[16];
 #pragma unroll
                 for (int e = 0; e < 16; ++e) {
-                    const int c0 = 32 * c4 + 2 * e;
-                    const float p0 = ex2(fmaf(__uint_as_float(s[2 * e]), sl2, L[c0]));
-                    const float p1 = ex2(fmaf(__uint_as_float(s[2 * e + 1]), sl2, L[c0 + 1]));
+                    const int c0 = 32 * c2 + 2 * e;
+                    const uint64_t arg = ptx::f2_fma(
+                        ptx::f2_pack(__uint_as_float(s[2 * e]), __uint_as_float(s[2 * e + 1])), sl2x2,
+                        ptx::f2_pack(L[c0], L[c0 + 1]));
+                    float a0, a1;
+                    ptx::f2_unpack(arg, a0, a1);
+                    const float p0 = ex2(a0), p1 = ex2(a1);
                     pp[e] = ptx::pack_bf16(p0, p1);
-                    pd[e] = ptx::pack_bf16(p0 * (__uint_as_float(dp[2 * e]) - Dl[c0]),
-                                           p1 * (__uint_as_float(dp[2 * e + 1]) - Dl[c0 + 1]));
+                    const uint64_t dd = ptx::f2_add(
+                        ptx::f2_pack(__uint_as_float(dp[2 * e]), __uint_as_float(dp[2 * e + 1])),
+                        ptx::f2_pack(ND[c0], ND[c0 + 1]));
+                    float d0, d1;
+                    ptx::f2_unpack(ptx::f2_mul(ptx::f2_pack(p0, p1), dd), d0, d1);
+                    pd[e] = ptx::pack_bf16(d0, d1);
                 }
-                ptx::tmem_st16(tS + 16 * c4, pp);
-                ptx::tmem_st16(tP + 16 * c4, pd);
+                ptx::tmem_st16(tS + 16 * c2, pp);
+                ptx::tmem_st16(tP + 16 * c2, pd);
             }
             ptx::tmem_wait_st();
             ptx::tc_fence_before();
@@ -559,23 +641,39 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (ok) ok = __all_sync(0xffffffffu, ptx::mbar_wait_bounded(&kv_done, 0, abort_p, p.wait_limit));
         if (ok) {
+            // Every MMA has completed: the Q/dO ring is free and stages one
+            // fp32 [128][D + 4] tile (dK, then dV); each half fills D/2
+            // columns of its rows, then every warp stores whole rows.
             ptx::tc_fence_after();
-            const bool kv = r < valid_keys;
-            const size_t accb = (size_t)b * p.N * p.H * D;
-            const int rr = kt * kBM + r;  // row inside the gradient run
+            float* stage = reinterpret_cast<float*>(sQ);
+            constexpr int kStride = D + 4;
+            constexpr int E = D / 32;
+            constexpr int DH = D / 2;
             for (int which = 0; which < 2; ++which) {
-                float val[D];
+                const float mul = which == 0 ? p.scale : 1.f;
 #pragma unroll
-                for (int c = 0; c < D / 32; ++c) {
+                for (int c = 0; c < DH / 32; ++c) {
                     uint32_t o[32];
-                    ptx::tmem_ld32(tbase + 256 + (which == 0 ? D : 0) + 32 * c + lane_off, o);
+                    ptx::tmem_ld32(tbase + 256 + (which == 0 ? D : 0) + DH * half + 32 * c + lane_off, o);
                     ptx::tmem_wait_ld();
+                    float4* dst = reinterpret_cast<float4*>(stage + r * kStride + DH * half + 32 * c);
 #pragma unroll
-                    for (int e = 0; e < 32; ++e)
-                        val[32 * c + e] = __uint_as_float(o[e]) * (which == 0 ? p.scale : 1.f);
+                    for (int e = 0; e < 8; ++e)
+                        dst[e] = make_float4(__uint_as_float(o[4 * e]) * mul, __uint_as_float(o[4 * e + 1]) * mul,
+                                             __uint_as_float(o[4 * e + 2]) * mul,
+                                             __uint_as_float(o[4 * e + 3]) * mul);
                 }
-                if (kv)
-                    scatter_row_tc<D>((which == 0 ? p.dk_acc : p.dv_acc) + accb, gr, rr, h, p.H, val, p.mode);
+                ptx::named_bar_sync(1, 256);
+                float* base = (which == 0 ? p.dk_ctx : p.dv_ctx);
+                for (int rr = warp - 4; rr < valid_keys; rr += 8) {
+                    const size_t o = (((size_t)b * p.R + gr.crow0 + kt * kBM + rr) * p.H + h) * D + E * lane;
+                    const float* src = stage + rr * kStride + E * lane;
+                    if (E == 4)
+                        *reinterpret_cast<float4*>(base + o) = *reinterpret_cast<const float4*>(src);
+                    else
+                        *reinterpret_cast<float2*>(base + o) = *reinterpret_cast<const float2*>(src);
+                }
+                ptx::named_bar_sync(1, 256);
             }
         }
         if (!ok && lane == 0) atomicOr(p.status, kDevTimeout);
@@ -640,9 +738,9 @@ msf_status launch_bwd_tc(msf_plan_t plan, const BwdTcInput& in, cudaStream_t st)
     tp.lse = in.lse;
     tp.delta = in.delta;
     tp.dq = (__nv_bfloat16*)in.dq;
-    tp.dk_acc = in.dk_acc;
-    tp.dv_acc = in.dv_acc;
-    tp.mode = P.d.resample;
+    tp.dk_ctx = in.dk_ctx;
+    tp.dv_ctx = in.dv_ctx;
+    tp.R = in.R;
     tp.status = a.status;
     tp.wait_limit = kWaitLimit;
     // dQ: every query tile of every group, longest contexts first.
@@ -685,13 +783,14 @@ msf_status launch_bwd_tc(msf_plan_t plan, const BwdTcInput& in, cudaStream_t st)
     tp.n_groups = a.n_groups;
     const bool d128 = P.D == 128;
     const int smem = d128 ? BCfg<128>::kSmem : BCfg<64>::kSmem;
+    const int qsmem = d128 ? QCfg<128>::kSmem : QCfg<64>::kSmem;
     static bool attr_set = false;
     if (!attr_set) {
         cudaError_t e = cudaFuncSetAttribute(bwd_dq_tc_kernel<128>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, BCfg<128>::kSmem);
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, QCfg<128>::kSmem);
         if (e == cudaSuccess)
             e = cudaFuncSetAttribute(bwd_dq_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     BCfg<64>::kSmem);
+                                     QCfg<64>::kSmem);
         if (e == cudaSuccess)
             e = cudaFuncSetAttribute(bwd_dkdv_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      BCfg<128>::kSmem);
@@ -706,40 +805,56 @@ msf_status launch_bwd_tc(msf_plan_t plan, const BwdTcInput& in, cudaStream_t st)
     }
     cudaError_t e = cudaSuccess;
     if (items > 0)
-        e = d128 ? launch_pdl(bwd_dq_tc_kernel<128>, dim3((unsigned)items), dim3(kThreads), smem, st, maps, tp)
-                 : launch_pdl(bwd_dq_tc_kernel<64>, dim3((unsigned)items), dim3(kThreads), smem, st, maps, tp);
+        e = d128 ? launch_pdl(bwd_dq_tc_kernel<128>, dim3((unsigned)items), dim3(kThreads), qsmem, st, maps, tp)
+                 : launch_pdl(bwd_dq_tc_kernel<64>, dim3((unsigned)items), dim3(kThreads), qsmem, st, maps, tp);
     if (e != cudaSuccess) {
         set_cuda_error((int)e);
         return MSF_ERR_CUDA;
     }
-    // dK/dV: one launch per group, so that every accumulator row has one
-    // writer per launch and the sums over groups come in a fixed order.
-    for (int gi = 0; gi < a.n_groups; ++gi) {
+    // dK/dV: every group's window-derived rows in one launch, groups with
+    // the most query tiles first.
+    int korder[MSF_MAX_GROUPS];
+    int nk = 0;
+    for (int gi = 0; gi < a.n_groups; ++gi)
+        if (in.g[gi].n_gseg > 0 && in.g[gi].q_end > in.g[gi].q_begin) korder[nk++] = gi;
+    for (int i = 0; i < nk; ++i)
+        for (int k = i + 1; k < nk; ++k)
+            if (in.g[korder[k]].q_end - in.g[korder[k]].q_begin >
+                in.g[korder[i]].q_end - in.g[korder[i]].q_begin) {
+                const int t = korder[i];
+                korder[i] = korder[k];
+                korder[k] = t;
+            }
+    int kitems = 0;
+    for (int oi = 0; oi < nk; ++oi) {
+        const int gi = korder[oi];
         const BwdGroup& bg = in.g[gi];
-        if (bg.n_gseg == 0 || bg.q_end <= bg.q_begin) continue;
-        tp.q_begin = bg.q_begin;
-        tp.q_end = bg.q_end;
-        tp.n_qt = (bg.q_end - bg.q_begin + kBM - 1) / kBM;
-        tp.n_grad = bg.n_gseg;
+        BGroupK& kg = tp.kg[oi];
+        kg.q_begin = bg.q_begin;
+        kg.q_end = bg.q_end;
+        kg.n_qt = (bg.q_end - bg.q_begin + kBM - 1) / kBM;
+        kg.item_base = kitems;
+        kg.n_grad = bg.n_gseg;
         int kt0 = 0;
         for (int s = 0; s < bg.n_gseg; ++s) {
             const GradSeg& gs = bg.gseg[s];
-            BGrad& g = tp.gr[s];
+            BGrad& g = kg.gr[s];
             g.map = gs.map_id == kMapPyr ? kMapPyr0 + gi : gs.map_id;
             // pyramid rows are addressed from the group's pyramid part, the
             // ring from its first slot, the window from token 0
             g.row0 = gs.map_id == kMapPyr ? gs.row0 - P.groups[gi].pyr_offset : gs.row0;
             g.len = gs.len;
             g.kt0 = kt0;
-            g.sigma = gs.sigma;
-            g.dst0 = gs.dst0;
-            g.src_gw = gs.src_gw;
-            g.out_gw = gs.out_gw;
+            g.crow0 = gs.crow0;
             kt0 += (gs.len + kBM - 1) / kBM;
         }
-        const unsigned grid = (unsigned)(kt0 * P.H * P.B);
-        e = d128 ? launch_pdl(bwd_dkdv_tc_kernel<128>, dim3(grid), dim3(kThreads), smem, st, maps, tp)
-                 : launch_pdl(bwd_dkdv_tc_kernel<64>, dim3(grid), dim3(kThreads), smem, st, maps, tp);
+        kg.n_kt = kt0;
+        kitems += kt0 * P.H * P.B;
+    }
+    tp.n_kgroups = nk;
+    if (kitems > 0) {
+        e = d128 ? launch_pdl(bwd_dkdv_tc_kernel<128>, dim3((unsigned)kitems), dim3(kThreads), smem, st, maps, tp)
+                 : launch_pdl(bwd_dkdv_tc_kernel<64>, dim3((unsigned)kitems), dim3(kThreads), smem, st, maps, tp);
         if (e != cudaSuccess) {
             set_cuda_error((int)e);
             return MSF_ERR_CUDA;

@@ -16,12 +16,13 @@ struct BwdTcInput {
     const float* lse;     // [B, H, N]
     const float* delta;   // [B, H, N]
     void* dq;             // [B, N, H, D] bf16, written
-    float* dk_acc;        // [B, N, H, D] fp32, accumulated into
-    float* dv_acc;
+    float* dk_ctx;        // [B, R, H, D] fp32 context-row gradients, written
+    float* dv_ctx;
+    int R;
 };
 
-// dq (bf16) for every query, and the window key/value gradients added into
-// dk_acc/dv_acc: one launch for dq, one per query group for dk/dv.
+// dq (bf16) for every query (one launch), and the key/value gradients of
+// every group's window-derived context rows (one launch).
 msf_status launch_bwd_tc(msf_plan_t plan, const BwdTcInput& in, cudaStream_t st);
 
 }  // namespace msf

@@ -92,10 +92,23 @@ inline size_t msp_split_bytes(const Plan& p) {
     return round256((size_t)kMaxDeembedSplits * p.B * per * 4);
 }
 // Backward workspace (caller-provided per msf_mssa_backward call):
-// [delta fp32 [B, H, N] | dk_acc fp32 [B, N, H, D] | dv_acc fp32 [B, N, H, D]].
+// [delta fp32 [B, H, N] | dk_ctx fp32 [B, R, H, D] | dv_ctx fp32 [B, R, H, D]],
+// R = rows of every group's context that come from the window (the rows
+// that receive key/value gradients): N for g = 1, n_finer * G/g^2 + the
+// window suffix for g > 1.
+inline int bwd_ctx_rows(const Plan& p) {
+    int r = 0;
+    for (int gi = 0; gi < p.n_groups; ++gi) {
+        const Group& g = p.groups[gi];
+        r += g.scale == 1 ? p.N : g.n_finer * g.pooled + (p.N - g.q_begin);
+    }
+    return r;
+}
 inline size_t bwd_delta_bytes(const Plan& p) { return round256((size_t)p.B * p.H * p.N * 4); }
-inline size_t bwd_acc_bytes(const Plan& p) { return round256((size_t)p.B * p.N * p.H * p.D * 4); }
-inline size_t bwd_workspace_bytes(const Plan& p) { return bwd_delta_bytes(p) + 2 * bwd_acc_bytes(p); }
+inline size_t bwd_ctx_bytes(const Plan& p) {
+    return round256((size_t)p.B * bwd_ctx_rows(p) * p.H * p.D * 4);
+}
+inline size_t bwd_workspace_bytes(const Plan& p) { return bwd_delta_bytes(p) + 2 * bwd_ctx_bytes(p); }
 inline size_t workspace_bytes(const Plan& p) {
     return kStatusBytes + 2 * pyramid_bytes(p) + msp_scratch_bytes(p) + attn_counter_bytes(p) +
            attn_partial_bytes(p) + msp_split_bytes(p);

@@ -139,16 +139,18 @@ cudaError_t launch_attn_simt(const AttnArgs& a, bool bf16, cudaStream_t st);
 // ---------------------------------------------------------- MSSA backward
 //
 // Context rows whose key/value gradients flow back to window tokens: rows
-// [row0, row0 + len) of a [B, rows_total, H, D] tensor pair (k, v). sigma 1:
-// row row0 + r is window token dst0 + r. sigma > 1: row r is token
-// (r / out_gw, r % out_gw) of a pooled state whose fine grid (src_gw wide)
-// starts at window token dst0; the adjoint of Subsample spreads it back.
+// [row0, row0 + len) of a [B, rows_total, H, D] tensor pair (k, v). Their
+// gradients go to rows [crow0, crow0 + len) of the context-gradient buffers
+// (one run after another, all groups). sigma 1: row row0 + r is window token
+// dst0 + r. sigma > 1: row r is token (r / out_gw, r % out_gw) of a pooled
+// state whose fine grid (src_gw wide) starts at window token dst0.
 struct GradSeg {
     const char* k;
     const char* v;
     long long bstride;  // bytes between streams
     int row0, len, rows_total, map_id;
     int sigma, dst0, src_gw, out_gw;
+    int crow0;
 };
 constexpr int kMaxGradSeg = MSF_MAX_STATES + 1;
 struct BwdGroup {
@@ -163,22 +165,40 @@ struct BwdCommon {
     const char* out;    // [B, N, H, D]
     const float* lse;   // [B, H, N], natural log
     float* delta;       // [B, H, N]: rowsum(dout * out)
-    float* dk_acc;      // [B, N, H, D] fp32 accumulators (all groups)
-    float* dv_acc;
+    float* dk_ctx;      // [B, R, H, D] fp32 gradients of the window-derived context
+    float* dv_ctx;      //   rows of every group (GradSeg.crow0 places each run)
+    int R;
     long long bstride;  // bytes between streams of q/dout/out/dq
     int H, D, B, N;
     float scale;        // softmax scale
     float scale_log2;   // scale * log2(e)
-    int mode;           // msf_resample_mode (adjoint of Subsample)
+};
+// The adjoint of Subsample, summed over groups: window token t of state l
+// receives, from each entry of state l, context-gradient row
+//   sigma 1:  crow0 + (t - dst0)
+//   sigma > 1: crow0 + (i / sigma) * out_gw + j / sigma, weight 1/sigma^2 (AVG),
+//              or only when sigma divides i and j, weight 1 (STRIDED),
+// where (i, j) is t's position on the state's grid (src_gw wide).
+struct GatherEntry {
+    int crow0, dst0, sigma, src_gw, out_gw;
+};
+struct GatherArgs {
+    int T;
+    int st_off[MSF_MAX_STATES + 1];
+    int n_ent[MSF_MAX_STATES];
+    GatherEntry e[MSF_MAX_STATES][MSF_MAX_GROUPS];
+    int mode;  // msf_resample_mode
 };
 cudaError_t launch_bwd_delta(const BwdCommon& c, bool bf16, cudaStream_t st);
 // dq for every query of every group (context of each group as in the forward).
 cudaError_t launch_bwd_dq_simt(const BwdCommon& c, const AttnArgs& a, void* dq, bool bf16,
                                cudaStream_t st);
-// dK/dV of one group's gradient rows, accumulated into dk_acc/dv_acc.
+// Context-row gradients of one group's window-derived rows.
 cudaError_t launch_bwd_dkdv_simt(const BwdCommon& c, const BwdGroup& g, bool bf16,
                                  cudaStream_t st);
-// dk_win, dv_win = cast(dk_acc, dv_acc).
-cudaError_t launch_bwd_cast(const BwdCommon& c, void* dk, void* dv, bool bf16, cudaStream_t st);
+// dk_win, dv_win from the context-row gradients (adjoint of Subsample, sum
+// over groups, one rounding to the dtype).
+cudaError_t launch_bwd_gather(const BwdCommon& c, const GatherArgs& g, void* dk, void* dv,
+                              bool bf16, cudaStream_t st);
 
 }  // namespace msf

@@ -4,6 +4,7 @@ synthetic inputs so that `ncu -k <kernel>` can capture it in isolation.
     python -m paper_2607_20940_gb300.profile_cases pool     # K/V pyramid at three sizes
     python -m paper_2607_20940_gb300.profile_cases embed    # MSP patchify + tier embedding
     python -m paper_2607_20940_gb300.profile_cases deembed  # de-embedding + unpatchify
+    python -m paper_2607_20940_gb300.profile_cases backward # forward with lse + MSSA gradient
 
 Each case runs twice after an L2 flush (a 256 MiB write) and checks the
 device status word. Nothing here is timed; the numbers come from the
@@ -70,8 +71,25 @@ def run(case: str) -> None:
             torch.cuda.synchronize()
             assert plan.device_status() == msf.MSF_OK
             plan.close()
+    elif case == "backward":
+        w = synth.LAYER_480P
+        plan, d, _ = _setup(w)
+        B, N, H = w.batch, plan.info.n_tokens, w.heads
+        lse = torch.empty((B, H, N), dtype=torch.float32, device=dev)
+        out = torch.empty_like(d["q"])
+        dout = torch.randn(d["q"].shape, device=dev).to(torch.bfloat16)
+        grads = [torch.empty_like(d["q"]) for _ in range(3)]
+        bws = plan.backward_workspace(dev)
+        plan.kv_resample(d["k_win"], d["v_win"])
+        for _ in range(2):
+            flush.fill_(1)
+            plan.mssa_forward_lse(d["q"], d["k_win"], d["v_win"], out, lse)
+            plan.mssa_backward(d["q"], d["k_win"], d["v_win"], out, dout, lse, *grads, bws)
+        torch.cuda.synchronize()
+        assert plan.device_status() == msf.MSF_OK
+        plan.close()
     else:
-        raise SystemExit(f"unknown case {case!r}: pool, embed or deembed")
+        raise SystemExit(f"unknown case {case!r}: pool, embed, deembed or backward")
 
 
 if __name__ == "__main__":
