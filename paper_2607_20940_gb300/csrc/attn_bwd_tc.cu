@@ -87,9 +87,15 @@ struct BwdTcParams {
     // bwd_dq_tc_kernel
     int n_groups;
     BGroupQ g[MSF_MAX_GROUPS];
-    // bwd_dkdv_tc_kernel
+    // dK/dV work
     int n_kgroups;
     BGroupK kg[MSF_MAX_GROUPS];
+    // Block ranges of the one launch, most expensive items first: kind 0 =
+    // dq items of group g[group], kind 1 = dK/dV items of kg[group].
+    int n_ranges;
+    struct Range {
+        int kind, group, base, count;
+    } range[2 * MSF_MAX_GROUPS];
 };
 struct BwdMaps {
     CUtensorMap q, dout;
@@ -97,13 +103,13 @@ struct BwdMaps {
     CUtensorMap v[kNumMaps];
 };
 
+// Dynamic shared memory of the launch: seven 128 x D bf16 tiles (dq items:
+// Q, dO, a 3-deep K ring and a 2-deep V ring; dK/dV items: K, V, a 2-deep
+// Q/dO ring and the per-query statistics), at least 120 KB so that one CTA
+// (and one 512-column TMEM allocation) sits on an SM.
 template <int D>
 struct BCfg {
     static constexpr int kTile = kBM * D * 2;
-    // Q, dO and two K/V stages (dQ kernel) or K, V and two Q/dO stages (dK/dV
-    // kernel); at least 120 KB so that one CTA (and one 512-column TMEM
-    // allocation) sits on an SM.
-    static constexpr int kSmem = 6 * kTile + 1024 > 120 * 1024 ? 6 * kTile + 1024 : 120 * 1024;
 };
 
 __device__ __forceinline__ float ex2(float x) {
@@ -140,10 +146,10 @@ struct QCfg {
     static constexpr int kTile = kBM * D * 2;
     static constexpr int kSmem = 7 * kTile + 1024 > 120 * 1024 ? 7 * kTile + 1024 : 120 * 1024;
 };
+static_assert(7 * QCfg<128>::kTile + 1024 + 2048 <= 227 * 1024, "shared memory of the launch");
 
 template <int D>
-__global__ void __launch_bounds__(kThreads, 1)
-    bwd_dq_tc_kernel(const __grid_constant__ BwdMaps maps, const __grid_constant__ BwdTcParams p) {
+__device__ __forceinline__ void dq_item(const BwdMaps& maps, const BwdTcParams& p, int gi, int local) {
     using C = QCfg<D>;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -158,10 +164,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __shared__ int abort_flag;
 
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-    int gi = 0;
-    while (gi + 1 < p.n_groups && (int)blockIdx.x >= p.g[gi + 1].item_base) ++gi;
     const BGroupQ& G = p.g[gi];
-    const int local = (int)blockIdx.x - G.item_base;
     const int qt = local % G.n_qt;
     const int h = (local / G.n_qt) % p.H;
     const int b = local / (G.n_qt * p.H);
@@ -435,8 +438,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 // ============================================================ dK/dV kernel
 
 template <int D>
-__global__ void __launch_bounds__(kThreads, 1)
-    bwd_dkdv_tc_kernel(const __grid_constant__ BwdMaps maps, const __grid_constant__ BwdTcParams p) {
+__device__ __forceinline__ void dkdv_item(const BwdMaps& maps, const BwdTcParams& p, int kgi,
+                                          int local) {
     using C = BCfg<D>;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -445,16 +448,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     unsigned char* sQ = smem + 2 * C::kTile;   // [2]
     unsigned char* sG = smem + 4 * C::kTile;   // [2] dO
 
-    __shared__ uint64_t kv_full, qg_full[2], qg_empty[2], st_full, pds_full, kv_done, drain_bar;
+    __shared__ uint64_t kv_full, qg_full[2], qg_empty[2], st_full[2], pds_full[2], kv_done, drain_bar;
     __shared__ uint32_t tmem_base_sh;
     __shared__ int abort_flag;
-    __shared__ float sL[2][kBM], sD[2][kBM];
+    // per-query statistics of the current and the previous query tile, in
+    // the seventh tile of the dynamic shared memory
+    float(*sL)[kBM] = reinterpret_cast<float(*)[kBM]>(smem + 6 * C::kTile);
+    float(*sD)[kBM] = reinterpret_cast<float(*)[kBM]>(smem + 6 * C::kTile + 2 * kBM * 4);
 
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-    int kgi = 0;
-    while (kgi + 1 < p.n_kgroups && (int)blockIdx.x >= p.kg[kgi + 1].item_base) ++kgi;
     const BGroupK& KG = p.kg[kgi];
-    const int local = (int)blockIdx.x - KG.item_base;
     const int kt_all = local % KG.n_kt;
     const int h = (local / KG.n_kt) % p.H;
     const int b = local / (KG.n_kt * p.H);
@@ -473,8 +476,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             ptx::mbar_init(&qg_full[s], 1);
             ptx::mbar_init(&qg_empty[s], 1);
         }
-        ptx::mbar_init(&st_full, 1);
-        ptx::mbar_init(&pds_full, 8);
+        for (int s = 0; s < 2; ++s) {
+            ptx::mbar_init(&st_full[s], 1);
+            ptx::mbar_init(&pds_full[s], 4);  // one arrival per warp of the column half
+        }
         ptx::mbar_init(&kv_done, 1);
         ptx::mbar_init(&drain_bar, 1);
         ptx::fence_mbar_init();
@@ -520,7 +525,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else if (warp == 1) {
         // ============================= MMA issuer =============================
-        constexpr uint32_t idS = ptx::idesc_bf16(kBM, kBM, false, false);
         constexpr uint32_t idO = ptx::idesc_bf16(kBM, D, false, true);
         constexpr uint64_t kTileDesc = (uint64_t)(C::kTile >> 4);
         const uint64_t k_desc = ptx::sdesc_sw128(ptx::smem_u32(sK), 16, 1024);
@@ -533,41 +537,71 @@ __global__ void __launch_bounds__(kThreads, 1)
             const bool r = ptx::mbar_wait_bounded(bar, parity, abort_p, p.wait_limit);
             return __all_sync(0xffffffffu, r);
         };
-        bool ok = wait_all(&kv_full, 0);
-        for (int i = 0; i < nq && ok; ++i) {
+        // Query tile i is done in two halves of 64 queries: half A's
+        // dV/dK MMAs and the next tile's S^T/dP^T of half A run while the
+        // softmax works on half B, and the other way round.
+        constexpr uint32_t idS64 = ptx::idesc_bf16(kBM, 64, false, false);
+        auto issue_st = [&](int i, int hf) {  // S^T, dP^T of half hf of query tile i
             const int st = i & 1;
-            ok = wait_all(&qg_full[st], (uint32_t)((i >> 1) & 1));
-            if (!ok) break;
+            const uint64_t qd = q_desc + (uint64_t)st * kTileDesc + (uint64_t)((64 * 128 * hf) >> 4);
+            const uint64_t gd = g_desc + (uint64_t)st * kTileDesc + (uint64_t)((64 * 128 * hf) >> 4);
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk)
+                ptx::mma_ss(tbase + 64 * hf, k_desc + kmajor_step(kk), qd + kmajor_step(kk), idS64,
+                            kk > 0 ? 1u : 0u);
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk)
+                ptx::mma_ss(tbase + 128 + 64 * hf, v_desc + kmajor_step(kk), gd + kmajor_step(kk), idS64,
+                            kk > 0 ? 1u : 0u);
+            ptx::mma_commit(&st_full[hf]);
+        };
+        auto issue_kv = [&](int i, int hf) {  // dV += P^T dO, dK += dS^T Q over half hf
+            const int st = i & 1;
+            const uint64_t gd = gmn_desc + (uint64_t)st * kTileDesc;
+            const uint64_t qd = qmn_desc + (uint64_t)st * kTileDesc;
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk) {
+                const uint64_t roff = (uint64_t)((4 * hf + kk) * (2048 >> 4));
+                ptx::mma_ts(tbase + 256, tbase + 64 * hf + kk * 8, gd + roff, idO,
+                            (i > 0 || hf > 0 || kk > 0) ? 1u : 0u);
+                ptx::mma_ts(tbase + 256 + D, tbase + 128 + 64 * hf + kk * 8, qd + roff, idO,
+                            (i > 0 || hf > 0 || kk > 0) ? 1u : 0u);
+            }
+        };
+        bool ok = wait_all(&kv_full, 0) && wait_all(&qg_full[0], 0);
+        if (ok) {
             ptx::tc_fence_after();
             if (ptx::elect_one_sync()) {
-                const uint64_t qd = q_desc + (uint64_t)st * kTileDesc;
-                const uint64_t gd = g_desc + (uint64_t)st * kTileDesc;
-#pragma unroll
-                for (int kk = 0; kk < D / 16; ++kk)
-                    ptx::mma_ss(tbase, k_desc + kmajor_step(kk), qd + kmajor_step(kk), idS, kk > 0 ? 1u : 0u);
-#pragma unroll
-                for (int kk = 0; kk < D / 16; ++kk)
-                    ptx::mma_ss(tbase + 128, v_desc + kmajor_step(kk), gd + kmajor_step(kk), idS,
-                                kk > 0 ? 1u : 0u);
-                ptx::mma_commit(&st_full);
+                issue_st(0, 0);
+                issue_st(0, 1);
             }
             __syncwarp();
-            ok = wait_all(&pds_full, (uint32_t)(i & 1));
+        }
+        for (int i = 0; i < nq && ok; ++i) {
+            const int st = i & 1;
+            const bool more = i + 1 < nq;
+            ok = wait_all(&pds_full[0], (uint32_t)(i & 1));
+            if (!ok) break;
+            ptx::tc_fence_after();
+            if (ptx::elect_one_sync()) issue_kv(i, 0);
+            __syncwarp();
+            if (more) {
+                ok = wait_all(&qg_full[st ^ 1], (uint32_t)(((i + 1) >> 1) & 1));
+                if (!ok) break;
+                ptx::tc_fence_after();
+                if (ptx::elect_one_sync()) issue_st(i + 1, 0);
+                __syncwarp();
+            }
+            ok = wait_all(&pds_full[1], (uint32_t)(i & 1));
             if (!ok) break;
             ptx::tc_fence_after();
             if (ptx::elect_one_sync()) {
-                const uint64_t gd = gmn_desc + (uint64_t)st * kTileDesc;
-                const uint64_t qd = qmn_desc + (uint64_t)st * kTileDesc;
-#pragma unroll
-                for (int kk = 0; kk < kBM / 16; ++kk)
-                    ptx::mma_ts(tbase + 256, tbase + 64 * (kk / 4) + (kk % 4) * 8,
-                                gd + (uint64_t)(kk * (2048 >> 4)), idO, (i > 0 || kk > 0) ? 1u : 0u);
-#pragma unroll
-                for (int kk = 0; kk < kBM / 16; ++kk)
-                    ptx::mma_ts(tbase + 256 + D, tbase + 128 + 64 * (kk / 4) + (kk % 4) * 8,
-                                qd + (uint64_t)(kk * (2048 >> 4)), idO, (i > 0 || kk > 0) ? 1u : 0u);
+                issue_kv(i, 1);
                 ptx::mma_commit(&qg_empty[st]);
-                if (i + 1 == nq) ptx::mma_commit(&kv_done);
+                if (more)
+                    issue_st(i + 1, 1);
+                else
+                    ptx::mma_commit(&kv_done);
             }
             __syncwarp();
         }
@@ -588,22 +622,23 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint64_t sl2x2 = ptx::f2_pack(p.scale_log2, p.scale_log2);
         bool ok = true;
         for (int i = 0; i < nq && ok; ++i) {
-            // this tile's per-query statistics, shared by the 128 key rows:
-            // threads 0-127 load -lse (log2 units), 128-255 delta
+            // this half's 64 per-query statistics, shared by its 128 key rows:
+            // threads 0-63 of the half load -lse (log2 units), 64-127 -delta
             {
-                const int qq = tix & 127;
+                const int hix = tix & 127;
+                const int qq = 64 * half + (hix & 63);
                 const int q = KG.q_begin + i * kBM + qq;
                 const bool qv = q < KG.q_end;
                 const size_t rix = ((size_t)b * p.H + h) * p.N + (qv ? q : 0);
-                if (tix < 128)
+                if (hix < 64)
                     sL[i & 1][qq] = qv ? -p.lse[rix] * kLog2e : -INFINITY;
                 else
                     sD[i & 1][qq] = qv ? -p.delta[rix] : 0.f;
             }
-            ptx::named_bar_sync(1, 256);
+            ptx::named_bar_sync(1 + half, 128);
             const float* L = sL[i & 1] + 64 * half;
             const float* ND = sD[i & 1] + 64 * half;
-            ok = __all_sync(0xffffffffu, ptx::mbar_wait_bounded(&st_full, (uint32_t)(i & 1), abort_p,
+            ok = __all_sync(0xffffffffu, ptx::mbar_wait_bounded(&st_full[half], (uint32_t)(i & 1), abort_p,
                                                                 p.wait_limit));
             if (!ok) break;
             ptx::tc_fence_after();
@@ -637,7 +672,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             ptx::tmem_wait_st();
             ptx::tc_fence_before();
             __syncwarp();
-            if (lane == 0) ptx::mbar_arrive(&pds_full);
+            if (lane == 0) ptx::mbar_arrive(&pds_full[half]);
         }
         if (ok) ok = __all_sync(0xffffffffu, ptx::mbar_wait_bounded(&kv_done, 0, abort_p, p.wait_limit));
         if (ok) {
@@ -663,7 +698,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                              __uint_as_float(o[4 * e + 2]) * mul,
                                              __uint_as_float(o[4 * e + 3]) * mul);
                 }
-                ptx::named_bar_sync(1, 256);
+                ptx::named_bar_sync(3, 256);
                 float* base = (which == 0 ? p.dk_ctx : p.dv_ctx);
                 for (int rr = warp - 4; rr < valid_keys; rr += 8) {
                     const size_t o = (((size_t)b * p.R + gr.crow0 + kt * kBM + rr) * p.H + h) * D + E * lane;
@@ -673,7 +708,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     else
                         *reinterpret_cast<float2*>(base + o) = *reinterpret_cast<const float2*>(src);
                 }
-                ptx::named_bar_sync(1, 256);
+                ptx::named_bar_sync(3, 256);
             }
         }
         if (!ok && lane == 0) atomicOr(p.status, kDevTimeout);
@@ -685,6 +720,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::tc_fence_after();
         ptx::tmem_dealloc(tbase, 512);
     }
+}
+
+// One launch for both kinds of work, so that short dK/dV items fill the
+// SMs that long dq items leave idle at the end.
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    bwd_tc_kernel(const __grid_constant__ BwdMaps maps, const __grid_constant__ BwdTcParams p) {
+    int r = 0;
+    while (r + 1 < p.n_ranges && (int)blockIdx.x >= p.range[r + 1].base) ++r;
+    const int local = (int)blockIdx.x - p.range[r].base;
+    if (p.range[r].kind == 0)
+        dq_item<D>(maps, p, p.range[r].group, local);
+    else
+        dkdv_item<D>(maps, p, p.range[r].group, local);
 }
 
 bool encode_all(BwdMaps& m, const Plan& P, const BwdTcInput& in) {
@@ -781,36 +830,7 @@ msf_status launch_bwd_tc(msf_plan_t plan, const BwdTcInput& in, cudaStream_t st)
         items += g.n_qt * P.H * P.B;
     }
     tp.n_groups = a.n_groups;
-    const bool d128 = P.D == 128;
-    const int smem = d128 ? BCfg<128>::kSmem : BCfg<64>::kSmem;
-    const int qsmem = d128 ? QCfg<128>::kSmem : QCfg<64>::kSmem;
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(bwd_dq_tc_kernel<128>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, QCfg<128>::kSmem);
-        if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(bwd_dq_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     QCfg<64>::kSmem);
-        if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(bwd_dkdv_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     BCfg<128>::kSmem);
-        if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(bwd_dkdv_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     BCfg<64>::kSmem);
-        if (e != cudaSuccess) {
-            set_cuda_error((int)e);
-            return MSF_ERR_CUDA;
-        }
-        attr_set = true;
-    }
-    cudaError_t e = cudaSuccess;
-    if (items > 0)
-        e = d128 ? launch_pdl(bwd_dq_tc_kernel<128>, dim3((unsigned)items), dim3(kThreads), qsmem, st, maps, tp)
-                 : launch_pdl(bwd_dq_tc_kernel<64>, dim3((unsigned)items), dim3(kThreads), qsmem, st, maps, tp);
-    if (e != cudaSuccess) {
-        set_cuda_error((int)e);
-        return MSF_ERR_CUDA;
-    }
+    tp.n_groups = a.n_groups;
     // dK/dV: every group's window-derived rows in one launch, groups with
     // the most query tiles first.
     int korder[MSF_MAX_GROUPS];
@@ -852,13 +872,58 @@ msf_status launch_bwd_tc(msf_plan_t plan, const BwdTcInput& in, cudaStream_t st)
         kitems += kt0 * P.H * P.B;
     }
     tp.n_kgroups = nk;
-    if (kitems > 0) {
-        e = d128 ? launch_pdl(bwd_dkdv_tc_kernel<128>, dim3((unsigned)kitems), dim3(kThreads), smem, st, maps, tp)
-                 : launch_pdl(bwd_dkdv_tc_kernel<64>, dim3((unsigned)kitems), dim3(kThreads), smem, st, maps, tp);
+    // Ranges in decreasing cost per item (MMA blocks of 128x128xD: 3 per
+    // K/V tile of a dq item, 4 per query tile of a dK/dV item).
+    struct R {
+        int kind, group, count;
+        long long cost;
+    } rs[2 * MSF_MAX_GROUPS];
+    int nr = 0;
+    for (int oi = 0; oi < a.n_groups; ++oi)
+        if (tp.g[oi].n_qt > 0)
+            rs[nr++] = {0, oi, tp.g[oi].n_qt * P.H * P.B, 3LL * tp.g[oi].n_tiles};
+    for (int oi = 0; oi < nk; ++oi)
+        if (tp.kg[oi].n_kt > 0)
+            rs[nr++] = {1, oi, tp.kg[oi].n_kt * P.H * P.B, 4LL * tp.kg[oi].n_qt};
+    for (int i = 0; i < nr; ++i)
+        for (int k = i + 1; k < nr; ++k)
+            if (rs[k].cost > rs[i].cost) {
+                const R t = rs[i];
+                rs[i] = rs[k];
+                rs[k] = t;
+            }
+    int total = 0;
+    for (int i = 0; i < nr; ++i) {
+        tp.range[i].kind = rs[i].kind;
+        tp.range[i].group = rs[i].group;
+        tp.range[i].base = total;
+        tp.range[i].count = rs[i].count;
+        total += rs[i].count;
+    }
+    tp.n_ranges = nr;
+    (void)items;
+    (void)kitems;
+    if (total == 0) return MSF_OK;
+    const bool d128 = P.D == 128;
+    const int smem = d128 ? QCfg<128>::kSmem : QCfg<64>::kSmem;
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(bwd_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             QCfg<128>::kSmem);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(bwd_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     QCfg<64>::kSmem);
         if (e != cudaSuccess) {
             set_cuda_error((int)e);
             return MSF_ERR_CUDA;
         }
+        attr_set = true;
+    }
+    cudaError_t e = d128 ? launch_pdl(bwd_tc_kernel<128>, dim3((unsigned)total), dim3(kThreads), smem, st, maps, tp)
+                         : launch_pdl(bwd_tc_kernel<64>, dim3((unsigned)total), dim3(kThreads), smem, st, maps, tp);
+    if (e != cudaSuccess) {
+        set_cuda_error((int)e);
+        return MSF_ERR_CUDA;
     }
     return MSF_OK;
 }
