@@ -398,6 +398,26 @@ def other_configs(msf, synth, dev, flush, peaks, rank):
     fl = plan.info.attention_flops * wp.layers
     out["window_pass_30"] = {"workload": wp.name, "layers": wp.layers, "pass_ms": pass_ms,
                              "us_per_layer": pass_ms * 1e3 / wp.layers, "tflops": fl / (pass_ms * 1e-3) / 1e12}
+    # The same pass replayed from a CUDA graph (120 launches, no host work per
+    # launch): the pass holds no history update, so it is a static sequence.
+    try:
+        graph = torch.cuda.CUDAGraph()
+        cap = torch.cuda.Stream(device=dev)
+        cap.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(cap):
+            one_pass()
+        torch.cuda.current_stream().wait_stream(cap)
+        torch.cuda.synchronize()
+        with torch.cuda.graph(graph):
+            one_pass()
+        g_ms = _timed(graph.replay, flush, reps=3, warm=1)
+        out["window_pass_30"].update({"graph_pass_ms": g_ms, "graph_us_per_layer": g_ms * 1e3 / wp.layers,
+                                      "graph_tflops": fl / (g_ms * 1e-3) / 1e12})
+        del graph
+    except Exception as e:  # report the eager pass alone
+        out["window_pass_30"]["graph_error"] = str(e)[:200]
+    if plan.device_status() != msf.MSF_OK:
+        raise RuntimeError("device status error (window pass)")
 
     # ---- bandwidth of the pyramid and embedding kernels (480p layer, B=1 and the B=4 streams)
     bw = {}

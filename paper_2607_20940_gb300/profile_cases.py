@@ -5,6 +5,7 @@ synthetic inputs so that `ncu -k <kernel>` can capture it in isolation.
     python -m paper_2607_20940_gb300.profile_cases embed    # MSP patchify + tier embedding
     python -m paper_2607_20940_gb300.profile_cases deembed  # de-embedding + unpatchify
     python -m paper_2607_20940_gb300.profile_cases backward # forward with lse + MSSA gradient
+    python -m paper_2607_20940_gb300.profile_cases attention # MSSA forward, 480p layer
 
 Each case runs twice after an L2 flush (a 256 MiB write) and checks the
 device status word. Nothing here is timed; the numbers come from the
@@ -71,6 +72,17 @@ def run(case: str) -> None:
             torch.cuda.synchronize()
             assert plan.device_status() == msf.MSF_OK
             plan.close()
+    elif case == "attention":
+        w = synth.LAYER_480P
+        plan, d, _ = _setup(w)
+        out = torch.empty_like(d["q"])
+        plan.kv_resample(d["k_win"], d["v_win"])
+        for _ in range(2):
+            flush.fill_(1)
+            plan.mssa_forward(d["q"], d["k_win"], d["v_win"], out)
+        torch.cuda.synchronize()
+        assert plan.device_status() == msf.MSF_OK
+        plan.close()
     elif case == "backward":
         w = synth.LAYER_480P
         plan, d, _ = _setup(w)
@@ -89,7 +101,7 @@ def run(case: str) -> None:
         assert plan.device_status() == msf.MSF_OK
         plan.close()
     else:
-        raise SystemExit(f"unknown case {case!r}: pool, embed, deembed or backward")
+        raise SystemExit(f"unknown case {case!r}: pool, embed, deembed, backward or attention")
 
 
 if __name__ == "__main__":
