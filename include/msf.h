@@ -299,6 +299,29 @@ msf_status msf_history_append(msf_plan_t plan, const void* k_win, const void* v_
  * Errors: INVALID_ARG, STATE (not bound, or not a fused_append plan). */
 msf_status msf_history_commit(msf_plan_t plan);
 
+/* Host-side state of the history ring, for checkpointing a streaming
+ * rollout. Everything else the rollout needs lives in the caller's buffers:
+ * the ring itself (k_hist, v_hist) and, for a plan that keeps its pyramid
+ * incrementally, the workspace's pyramid (or rebuild it after a restore with
+ * msf_kv_resample(..., MSF_RESAMPLE_FULL)). */
+typedef struct msf_history_state {
+    int32_t count;   /* live frames in the ring */
+    int32_t oldest;  /* slot of the oldest live frame (meaningful once full) */
+    int32_t spare;   /* fused_append: the slot the next head is staged in */
+    int32_t _pad;
+} msf_history_state;
+
+/* Read the ring state. Host only. Errors: INVALID_ARG. */
+msf_status msf_history_get(msf_plan_t plan, msf_history_state* out);
+
+/* Restore a ring state read from a plan with the same description (for
+ * example after msf_plan_bind of a new plan on restored ring buffers).
+ * Checks count <= capacity, slots inside the ring, and the slot rules of the
+ * plan's mode (the next free slot or the oldest frame; with fused_append the
+ * spare is the free slot below capacity, else not a live one). Host only.
+ * Errors: INVALID_ARG (inconsistent state), STATE (not bound). */
+msf_status msf_history_set(msf_plan_t plan, const msf_history_state* st);
+
 /* Number of kernels this library has launched in this process (all plans,
  * all devices), for accounting in benchmarks. Host only. */
 uint64_t msf_kernel_launches(void);

@@ -303,6 +303,37 @@ extern "C" msf_status msf_history_commit(msf_plan_t plan) {
     return MSF_OK;
 }
 
+extern "C" msf_status msf_history_get(msf_plan_t plan, msf_history_state* out) {
+    if (!plan || !out) return MSF_ERR_INVALID_ARG;
+    out->count = plan->hist_count;
+    out->oldest = plan->hist_oldest;
+    out->spare = plan->fused ? plan->hist_spare : -1;
+    out->_pad = 0;
+    return MSF_OK;
+}
+
+extern "C" msf_status msf_history_set(msf_plan_t plan, const msf_history_state* st) {
+    if (!plan || !st) return MSF_ERR_INVALID_ARG;
+    Plan& p = *plan;
+    if (!p.bound) return MSF_ERR_STATE;
+    const int cap = p.d.history_capacity;
+    if (st->count < 0 || st->count > cap) return MSF_ERR_INVALID_ARG;
+    if (st->oldest < 0 || st->oldest >= (p.fused ? cap + 1 : (cap > 0 ? cap : 1)))
+        return MSF_ERR_INVALID_ARG;
+    if (st->count < cap && st->oldest != 0) return MSF_ERR_INVALID_ARG;
+    if (p.fused) {
+        // below capacity the live frames are slots [0, count) and the spare
+        // is slot count; at capacity the spare is the slot just before the
+        // oldest frame (the one evicted last)
+        const int want = st->count < cap ? st->count : (st->oldest + cap) % (cap + 1);
+        if (st->spare != want) return MSF_ERR_INVALID_ARG;
+        p.hist_spare = st->spare;
+    }
+    p.hist_count = st->count;
+    p.hist_oldest = st->oldest;
+    return MSF_OK;
+}
+
 static msf_status check_attn_args(const Plan& p, const void* q, const void* k_win,
                                   const void* v_win, void* out) {
     if (!q || !k_win || !v_win || !out) return MSF_ERR_INVALID_ARG;

@@ -36,7 +36,7 @@ EXPORTS = (
     "msf_kv_resample", "msf_mssa_forward", "msf_mssa_forward_simt", "msf_history_append",
     "msf_plan_device_status", "msf_kernel_launches", "msf_unpatchify_noalloc",
     "msf_selftest_wait_timeout", "msf_history_commit", "msf_mssa_forward_lse",
-    "msf_mssa_backward", "msf_mssa_backward_simt",
+    "msf_mssa_backward", "msf_mssa_backward_simt", "msf_history_get", "msf_history_set",
 )
 
 
@@ -51,6 +51,10 @@ class msf_plan_desc(ctypes.Structure):
         ("patch", ctypes.c_int32), ("embed_dim", ctypes.c_int32),
         ("frames_per_state", ctypes.c_int32), ("fused_append", ctypes.c_int32),
     ]
+
+
+class msf_history_state(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in ("count", "oldest", "spare", "_pad")]
 
 
 class msf_group_info(ctypes.Structure):
@@ -101,6 +105,8 @@ def _load():
         "msf_unpatchify_noalloc": (ctypes.c_int, [P, I32, VP, VP, VP, VP]),
         "msf_selftest_wait_timeout": (ctypes.c_int, [P, ctypes.c_int64, VP]),
         "msf_history_commit": (ctypes.c_int, [P]),
+        "msf_history_get": (ctypes.c_int, [P, ctypes.POINTER(msf_history_state)]),
+        "msf_history_set": (ctypes.c_int, [P, ctypes.POINTER(msf_history_state)]),
         "msf_mssa_forward_lse": (ctypes.c_int, [P, VP, VP, VP, VP, VP, VP]),
         "msf_mssa_backward": (ctypes.c_int, [P, VP, VP, VP, VP, VP, VP, VP, VP, VP, VP, SZ, VP]),
         "msf_mssa_backward_simt": (ctypes.c_int, [P, VP, VP, VP, VP, VP, VP, VP, VP, VP, VP, SZ, VP]),
@@ -236,6 +242,16 @@ def msf_mssa_backward_simt(plan: int, q, k_win, v_win, out, dout, lse, dq, dk_wi
            "msf_mssa_backward_simt")
 
 
+def msf_history_get(plan: int) -> msf_history_state:
+    st = msf_history_state()
+    _check(_lib.msf_history_get(plan, ctypes.byref(st)), "msf_history_get")
+    return st
+
+
+def msf_history_set(plan: int, st: msf_history_state) -> None:
+    _check(_lib.msf_history_set(plan, ctypes.byref(st)), "msf_history_set")
+
+
 def msf_history_commit(plan: int) -> None:
     _check(_lib.msf_history_commit(plan), "msf_history_commit")
 
@@ -348,6 +364,13 @@ class Plan:
 
     def history_append(self, k_win, v_win, stream=None):
         msf_history_append(self.handle, k_win, v_win, stream)
+        self.refresh()
+
+    def history_state(self) -> msf_history_state:
+        return msf_history_get(self.handle)
+
+    def set_history_state(self, st: msf_history_state):
+        msf_history_set(self.handle, st)
         self.refresh()
 
     def history_commit(self):

@@ -223,3 +223,16 @@ def test_backward_flops_480p():
     g1 = 3120 * (6 * 128 * 8970 + 4 * 128 * (8970 - 1560 - 2 * 1560))
     g2 = 1170 * (6 * 128 * 4290 + 4 * 128 * (4290 - 1560 - 2 * 390))
     assert info.backward_flops == 12 * (g1 + g2)
+
+
+def test_history_state_host_checks():
+    msf = _msf()
+    p = _plan((1, 2), 8, 8, 4, 1, cap=3)
+    st = p.history_state()
+    assert (st.count, st.oldest, st.spare) == (1, 0, -1)
+    with pytest.raises(msf.MsfError) as ei:
+        p.set_history_state(st)                      # not bound
+    assert ei.value.status == msf.MSF_ERR_STATE
+    q = _fused_plan((1, 2), 8, 8, 4, 2, 3)
+    st = q.history_state()
+    assert (st.count, st.oldest, st.spare) == (2, 0, 2)

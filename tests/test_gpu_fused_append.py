@@ -116,3 +116,60 @@ def test_fused_append_streaming_480p_b4():
     """The streaming rollout's shapes (B = 4, history 2 -> capacity 4,
     sink fixed) with the fused update; one sampled head per step."""
     _rollout(synth.STREAM_480P, BF16, 0, steps=5, heads=[0, 5, 10, 3, 8])
+
+
+@pytest.mark.parametrize("fused", [False, True], ids=["append", "fused"])
+def test_checkpoint_resume_rollout(fused):
+    """A rollout checkpointed after three steps (ring tensors + the ring's
+    host state) and resumed in a fresh plan gives the same outputs, bit for
+    bit, as the uninterrupted rollout (the restored plan rebuilds its pyramid
+    with a full resample)."""
+    m = msf()
+    w = dataclasses.replace(BASE, history_frames=1, history_capacity=2, batch=2, seed=51)
+    x = synth.attention_inputs(w, BF16)
+    B, G, H, D = w.batch, w.fine_tokens, w.heads, w.head_dim
+    slots = w.history_capacity + (1 if fused else 0)
+
+    def new_plan():
+        return m.Plan(m.make_desc(w.scales, w.grid_h, w.grid_w, w.heads, w.head_dim, w.sink_tokens,
+                                  w.history_frames, history_capacity=w.history_capacity,
+                                  batch=w.batch, fused_append=int(fused)))
+
+    def ring_from(src):
+        r = torch.zeros((B, slots, G, H, D), dtype=BF16, device="cuda")
+        r[:, :src.shape[1]] = src
+        return r
+
+    sink = {k: x[k].cuda() for k in ("k_sink", "v_sink")}
+    ring = {k: ring_from(x[k].cuda()) for k in ("k_hist", "v_hist")}
+    a = new_plan()
+    a.bind(a.workspace(), sink["k_sink"], sink["v_sink"], ring["k_hist"], ring["v_hist"])
+
+    def step(plan, kv, first):
+        plan.kv_resample(kv["k_win"], kv["v_win"], m.MSF_RESAMPLE_FULL if first else m.MSF_RESAMPLE_WINDOW_ONLY)
+        out = torch.empty_like(kv["q"])
+        plan.mssa_forward(kv["q"], kv["k_win"], kv["v_win"], out)
+        if fused:
+            plan.history_commit()
+        else:
+            plan.history_append(kv["k_win"], kv["v_win"])
+        return out
+
+    kvs = [{k: v.cuda() for k, v in synth.step_kv(w, 8000 + i, BF16).items()} for i in range(6)]
+    for i in range(3):
+        step(a, kvs[i], i == 0)
+    torch.cuda.synchronize()
+    # checkpoint: the ring buffers and the ring's host state
+    saved = {k: v.clone() for k, v in ring.items()}
+    st = a.history_state()
+    b = new_plan()
+    b.bind(b.workspace(), sink["k_sink"], sink["v_sink"], saved["k_hist"], saved["v_hist"])
+    b.set_history_state(st)
+    assert b.info.history_count == a.info.history_count
+    for i in range(3, 6):
+        oa = step(a, kvs[i], False)
+        ob = step(b, kvs[i], i == 3)
+        torch.cuda.synchronize()
+        assert torch.equal(oa, ob), i
+    assert torch.equal(ring["k_hist"], saved["k_hist"]) and torch.equal(ring["v_hist"], saved["v_hist"])
+    assert a.device_status() == m.MSF_OK and b.device_status() == m.MSF_OK
