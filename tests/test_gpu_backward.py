@@ -128,3 +128,11 @@ def test_backward_tensor_core_matches_cuda_core(w):
         a, b = g[k].float(), h[k].float()
         scale = b.abs().max().item()
         assert (a - b).abs().max().item() <= 1e-2 * scale, k
+
+
+def test_backward_three_scale_sampled_head():
+    """Three query groups (g = 1, 2, 4) at the 48x80 shapes: every pooled
+    level's adjoint at full size; the oracle checks one head."""
+    w = synth.THREE_SCALE
+    x, dout, out, lse, g, _ = _run(w, BF16, 0)
+    _check(x, dout, lse, g, w, BF16, 0, heads=[5])
