@@ -60,7 +60,10 @@ static_assert(4 * kCtrlRegs + 8 * kSoftmaxRegs == 12 * kLaunchRegs, "register sp
 constexpr long long kWaitLimit = 2000000000LL;  // ~1 s of SM clock
 // Lead tiles per item in the stream-K sequence: the fixed cost of a piece
 // (Q load and pipeline fill, epilogue or partial write) measured as ~5 K/V
-// tiles, so CTAs whose ranges hold many short items get fewer tiles.
+// tiles, so CTAs whose ranges hold many short items get fewer tiles. Where
+// the resulting range boundaries fall also decides how many items are split
+// (partial writes, merges), so msf_plan_tune_attention can pick another
+// count per plan by timing a few.
 constexpr int kItemLeadTiles = 5;
 
 struct TcSeg {
@@ -840,7 +843,7 @@ msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st) {
             ts.tile0 = tg.n_tiles;
             tg.n_tiles += (sg.len + kBlockN - 1) / kBlockN;
         }
-        tg.n_virt = tg.n_tiles + kItemLeadTiles;
+        tg.n_virt = tg.n_tiles + (P.attn_lead >= 0 ? P.attn_lead : kItemLeadTiles);
         tg.tile_base = total_tiles;
         tg.item_base = item_base;
         total_tiles += (long long)tg.n_items * tg.n_virt;
