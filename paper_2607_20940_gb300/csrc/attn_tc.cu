@@ -95,6 +95,9 @@ struct TcParams {
     unsigned int* counters;  // per item
     float* partials;         // 2 slots per CTA
     long long wait_limit;
+    int dp_rounds;           // whole items of group 0 per CTA before the stream-K range
+    long long dp_stride;     // group 0's tiles per item in the sequence (n_virt)
+    long long t_sk;          // first sequence position of the stream-K part
     float* lse;              // optional [B, H, N] row log-sum-exp (natural log)
     int N;                   // query rows per stream
 };
@@ -202,8 +205,21 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const long long T = p.total_tiles;
     const long long ncta = gridDim.x;
-    const long long r0 = cta_begin(blockIdx.x, T, ncta);
-    const long long r1 = cta_begin(blockIdx.x + 1, T, ncta);
+    // Work of this CTA: dp_rounds whole items of the first group (items
+    // blockIdx.x, blockIdx.x + ncta, ...), then its equal share of the rest of
+    // the sequence (stream-K), which starts at t_sk.
+    const long long Tsk = T - p.t_sk;
+    const long long r0 = p.t_sk + cta_begin(blockIdx.x, Tsk, ncta);
+    const long long r1 = p.t_sk + cta_begin(blockIdx.x + 1, Tsk, ncta);
+    auto phase_range = [&](int ph, long long& a0, long long& a1) {
+        if (ph < p.dp_rounds) {
+            a0 = ((long long)blockIdx.x + (long long)ph * ncta) * p.dp_stride;
+            a1 = a0 + p.dp_stride;
+        } else {
+            a0 = r0;
+            a1 = r1;
+        }
+    };
 
     if (threadIdx.x == 0) {
         abort_flag = 0;
@@ -251,8 +267,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             // K(j) and V(j) wait for one release: the commit that follows S1 of
             // tile j-2. It covers the last reader of K(j)'s slot (S of tile
             // j-2) and of V(j)'s slot in the 3-deep V ring (PV1 of tile j-3).
-            for (long long t = r0; t < r1 && ok;) {
-                const Piece pc = locate(p, t, r1);
+            for (int ph = 0; ph <= p.dp_rounds && ok; ++ph) {
+            long long a0, a1;
+            phase_range(ph, a0, a1);
+            for (long long t = a0; t < a1 && ok;) {
+                const Piece pc = locate(p, t, a1);
                 t = pc.t_next;
                 if (pc.u0 == pc.u1) continue;  // lead tiles only
                 const TcGroup& G = p.g[pc.gi];
@@ -288,6 +307,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                          &maps.v[G.seg[seg].map], &v_full[sv], c * 64, pc.h, row, pc.b);
                 }
                 ++piece;
+            }
             }
             if (!ok) {
                 // Drain: every copy issued must land before the CTA exits.
@@ -351,8 +371,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             int ks = 0, vs = 0;
             uint32_t kph = 0, vph = 0, pph = 0;
             int piece = 0;
-            for (long long t = r0; t < r1 && ok;) {
-                const Piece pc = locate(p, t, r1);
+            for (int ph = 0; ph <= p.dp_rounds && ok; ++ph) {
+            long long a0, a1;
+            phase_range(ph, a0, a1);
+            for (long long t = a0; t < a1 && ok;) {
+                const Piece pc = locate(p, t, a1);
                 t = pc.t_next;
                 const int n = pc.u1 - pc.u0;
                 if (n == 0) continue;  // lead tiles only
@@ -413,6 +436,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 __syncwarp();
                 ++piece;
             }
+            }
             if (!ok) {
                 // drain_bar covers every MMA issued: TMEM is never released under one.
                 if (ptx::elect_one_sync()) ptx::mma_commit(&drain_bar);
@@ -435,8 +459,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool ok = true;
         long long js = 0;
         int piece = 0, nsplit = 0;
-        for (long long tt = r0; tt < r1 && ok;) {
-            const Piece pc = locate(p, tt, r1);
+        for (int ph = 0; ph <= p.dp_rounds && ok; ++ph) {
+        long long a0, a1;
+        phase_range(ph, a0, a1);
+        for (long long tt = a0; tt < a1 && ok;) {
+            const Piece pc = locate(p, tt, a1);
             tt = pc.t_next;
             if (pc.u0 == pc.u1) continue;  // lead tiles only
             const TcGroup& G = p.g[pc.gi];
@@ -566,9 +593,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             } else {
                 // ---- split item: write this piece's partial result
-                const long long c1 = cta_of(pc.item_start, T, ncta);
-                const long long c2 = cta_of(pc.item_start + G.n_tiles - 1, T, ncta);
-                const int slot = slot_of(blockIdx.x, c1, pc.item_start, T, ncta);
+                // (only stream-K pieces are split: positions relative to t_sk)
+                const long long c1 = cta_of(pc.item_start - p.t_sk, Tsk, ncta);
+                const long long c2 = cta_of(pc.item_start + G.n_tiles - 1 - p.t_sk, Tsk, ncta);
+                const int slot = slot_of(blockIdx.x, c1, pc.item_start - p.t_sk, Tsk, ncta);
                 const int rr = t * kBlockM + r;
                 float* ps = p.partials + (size_t)slot * C::kSlotFloats;
                 float4* po = reinterpret_cast<float4*>(ps) + rr;
@@ -615,13 +643,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                     float M = -INFINITY;
                     for (long long c = c1; c <= c2; ++c) {
                         const float* q = p.partials +
-                                         (size_t)slot_of(c, c1, pc.item_start, T, ncta) * C::kSlotFloats;
+                                         (size_t)slot_of(c, c1, pc.item_start - p.t_sk, Tsk, ncta) * C::kSlotFloats;
                         M = fmaxf(M, __ldcg(q + C::kSlotML + rr));
                     }
                     float L = 0.f;
                     for (long long c = c1; c <= c2; ++c) {
                         const float* q = p.partials +
-                                         (size_t)slot_of(c, c1, pc.item_start, T, ncta) * C::kSlotFloats;
+                                         (size_t)slot_of(c, c1, pc.item_start - p.t_sk, Tsk, ncta) * C::kSlotFloats;
                         L += ex2(__ldcg(q + C::kSlotML + rr) - M) * __ldcg(q + C::kSlotML + 2 * kBlockM + rr);
                     }
                     const float inv = 1.0f / L;
@@ -635,7 +663,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         for (int e = 0; e < 32; ++e) acc[e] = 0.f;
                         for (long long c = c1; c <= c2; ++c) {
                             const float* base =
-                                p.partials + (size_t)slot_of(c, c1, pc.item_start, T, ncta) * C::kSlotFloats;
+                                p.partials + (size_t)slot_of(c, c1, pc.item_start - p.t_sk, Tsk, ncta) * C::kSlotFloats;
                             const float w = ex2(__ldcg(base + C::kSlotML + rr) - M);
                             const float4* src = reinterpret_cast<const float4*>(base) + rr;
 #pragma unroll
@@ -660,6 +688,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
             ++piece;
+        }
         }
         if (!ok && lane == 0) atomicOr(p.status, kDevTimeout);
     }
@@ -857,6 +886,13 @@ msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st) {
     if (ncta > P.attn_max_ctas) ncta = P.attn_max_ctas;
     if (ncta > total_tiles) ncta = total_tiles;
     if (ncta < 1) ncta = 1;
+    // Data-parallel rounds: while the longest group has at least one item per
+    // CTA, each CTA first takes whole items of it (no partial results), and
+    // only the rest of the sequence is split evenly (stream-K).
+    tp.dp_rounds = 0;
+    tp.dp_stride = tp.g[0].n_virt;
+    if (P.attn_dp != 0 && tp.n_groups > 0) tp.dp_rounds = (int)(tp.g[0].n_items / ncta);
+    tp.t_sk = (long long)tp.dp_rounds * ncta * tp.dp_stride;
 
     if (P.D == 128) {
         if (!cache.attr_set[1]) {
