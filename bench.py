@@ -257,7 +257,6 @@ def other_configs(msf, synth, dev, flush, peaks, rank):
     w3 = synth.THREE_SCALE
     plan, t = setup(w3)
     pyr_ms = _timed(lambda: plan.kv_resample(t["k_win"], t["v_win"], msf.MSF_RESAMPLE_FULL), flush)
-    plan.tune_attention(t["q"], t["k_win"], t["v_win"], t["out"])
     attn_ms = _timed(lambda: plan.mssa_forward(t["q"], t["k_win"], t["v_win"], t["out"]), flush)
     fl = plan.info.attention_flops
     out["three_scale"] = {"workload": w3.name, "attention_us": attn_ms * 1e3, "gflop": fl / 1e9,
@@ -299,7 +298,6 @@ def other_configs(msf, synth, dev, flush, peaks, rank):
     wc = synth.CHUNKED_480P
     plan, t = setup(wc)
     pyr_ms = _timed(lambda: plan.kv_resample(t["k_win"], t["v_win"], msf.MSF_RESAMPLE_FULL), flush)
-    plan.tune_attention(t["q"], t["k_win"], t["v_win"], t["out"])
     attn_ms = _timed(lambda: plan.mssa_forward(t["q"], t["k_win"], t["v_win"], t["out"]), flush)
     fl = plan.info.attention_flops
     if plan.device_status() != msf.MSF_OK:
@@ -309,7 +307,6 @@ def other_configs(msf, synth, dev, flush, peaks, rank):
     wcf = wc.with_scales((1,) * wc.T)
     plan, t = setup(wcf)
     plan.kv_resample(t["k_win"], t["v_win"], msf.MSF_RESAMPLE_FULL)
-    plan.tune_attention(t["q"], t["k_win"], t["v_win"], t["out"])
     fine_ms = _timed(lambda: plan.mssa_forward(t["q"], t["k_win"], t["v_win"], t["out"]), flush,
                      warm=2, reps=5)
     fl_fine = plan.info.attention_flops
@@ -389,7 +386,6 @@ def other_configs(msf, synth, dev, flush, peaks, rank):
     lat_out = torch.empty((wp.batch, wp.latent_channels, wp.grid_h * wp.patch, wp.grid_w * wp.patch),
                           dtype=torch.bfloat16, device=dev)
     plan.kv_resample(t["k_win"], t["v_win"], msf.MSF_RESAMPLE_FULL)
-    plan.tune_attention(t["q"], t["k_win"], t["v_win"], t["out"])
 
     def one_pass():
         for _ in range(wp.layers):
@@ -541,8 +537,6 @@ def main():
         plan.unpatchify(0, out.view(w.batch, N, E), w_out, lat_dst, stream=stream)
 
     plan.kv_resample(d["k_win"], d["v_win"], msf.MSF_RESAMPLE_FULL)
-    # one-time choice of the attention's stream-K split for this plan
-    plan.tune_attention(d["q"], d["k_win"], d["v_win"], out)
     for _ in range(args.warmup):
         step(d["q"], d["k_win"], d["v_win"], lat)
     torch.cuda.synchronize()
@@ -665,7 +659,6 @@ def main():
     plan_f.bind(wsf, df["k_sink"], df["v_sink"], df["k_hist"], df["v_hist"])
     outf = torch.empty_like(df["q"])
     plan_f.kv_resample(df["k_win"], df["v_win"])
-    plan_f.tune_attention(df["q"], df["k_win"], df["v_win"], outf)
     fine_ms = []
     for i in range(args.warmup + max(5, args.steps // 2)):
         flush.fill_(1)

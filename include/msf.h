@@ -275,16 +275,6 @@ msf_status msf_mssa_backward_simt(msf_plan_t plan, const void* q, const void* k_
                                   const float* lse, void* dq, void* dk_win, void* dv_win,
                                   void* bwd_workspace, size_t bwd_workspace_bytes, void* stream);
 
-/* Tune the tensor-core attention's work split for this plan: times the
- * kernel (a warm-up and three runs each, CUDA events on `stream`) with a few
- * stream-K lead-tile counts and keeps the fastest for later msf_mssa_forward
- * calls. The result does not depend on the values of q/k/v, only on the
- * plan's shapes and history count. Synchronises the stream; call it once
- * after bind and a resample, not during stream capture. fp32 plans: no-op.
- * Writes `out`. Errors: as msf_mssa_forward. */
-msf_status msf_plan_tune_attention(msf_plan_t plan, const void* q, const void* k_win,
-                                   const void* v_win, void* out, void* stream);
-
 /* Same computation always on the fp32 CUDA-core kernel (a cross-check of the
  * tensor-core kernel for bf16 plans). */
 msf_status msf_mssa_forward_simt(msf_plan_t plan, const void* q, const void* k_win,

@@ -370,63 +370,6 @@ extern "C" msf_status msf_mssa_forward_lse(msf_plan_t plan, const void* q, const
     return cuda_status(msf::launch_attn_simt(a, false, (cudaStream_t)stream));
 }
 
-extern "C" msf_status msf_plan_tune_attention(msf_plan_t plan, const void* q, const void* k_win,
-                                              const void* v_win, void* out, void* stream) {
-    if (!plan) return MSF_ERR_INVALID_ARG;
-    Plan& p = *plan;
-    msf_status st = check_attn_args(p, q, k_win, v_win, out);
-    if (st != MSF_OK) return st;
-    if (p.elem != 2) return MSF_OK;
-    cudaStream_t s = (cudaStream_t)stream;
-    msf::AttnArgs a;
-    build_attn_args(p, q, k_win, v_win, out, a);
-    // (lead tiles, data-parallel rounds on/off)
-    static const int kCand[][2] = {{5, 1}, {0, 1}, {2, 1}, {3, 1}, {8, 1}, {12, 1}, {16, 1},
-                                   {5, 0}, {0, 0}, {2, 0}, {3, 0}, {8, 0}, {12, 0}, {16, 0}};
-    cudaEvent_t e0, e1;
-    if (cudaEventCreate(&e0) != cudaSuccess) return cuda_status(cudaGetLastError());
-    if (cudaEventCreate(&e1) != cudaSuccess) {
-        cudaEventDestroy(e0);
-        return cuda_status(cudaGetLastError());
-    }
-    const int keep = p.attn_lead, keep_dp = p.attn_dp;
-    int best = -1, best_dp = 1;
-    float best_ms = 0.f;
-    cudaError_t e = cudaSuccess;
-    for (int ci = 0; ci < (int)(sizeof(kCand) / sizeof(kCand[0])) && e == cudaSuccess; ++ci) {
-        p.attn_lead = kCand[ci][0];
-        p.attn_dp = kCand[ci][1];
-        float ms[3];
-        st = msf::launch_attn_tc(plan, a, s);  // warm-up
-        for (int r = 0; r < 3 && st == MSF_OK; ++r) {
-            e = cudaEventRecord(e0, s);
-            if (e == cudaSuccess) st = msf::launch_attn_tc(plan, a, s);
-            if (st == MSF_OK && e == cudaSuccess) e = cudaEventRecord(e1, s);
-            if (st == MSF_OK && e == cudaSuccess) e = cudaEventSynchronize(e1);
-            if (st == MSF_OK && e == cudaSuccess) e = cudaEventElapsedTime(&ms[r], e0, e1);
-        }
-        if (st != MSF_OK || e != cudaSuccess) break;
-        // median of three
-        const float lo = fminf(ms[0], fminf(ms[1], ms[2])), hi = fmaxf(ms[0], fmaxf(ms[1], ms[2]));
-        const float med = ms[0] + ms[1] + ms[2] - lo - hi;
-        if (best < 0 || med < best_ms) {
-            best = kCand[ci][0];
-            best_dp = kCand[ci][1];
-            best_ms = med;
-        }
-    }
-    cudaEventDestroy(e0);
-    cudaEventDestroy(e1);
-    if (st != MSF_OK || e != cudaSuccess || best < 0) {
-        p.attn_lead = keep;
-        p.attn_dp = keep_dp;
-        return st != MSF_OK ? st : cuda_status(e != cudaSuccess ? e : cudaErrorUnknown);
-    }
-    p.attn_lead = best;
-    p.attn_dp = best_dp;
-    return MSF_OK;
-}
-
 extern "C" msf_status msf_mssa_forward(msf_plan_t plan, const void* q, const void* k_win,
                                        const void* v_win, void* out, void* stream) {
     if (!plan) return MSF_ERR_INVALID_ARG;

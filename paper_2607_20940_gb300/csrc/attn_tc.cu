@@ -60,10 +60,7 @@ static_assert(4 * kCtrlRegs + 8 * kSoftmaxRegs == 12 * kLaunchRegs, "register sp
 constexpr long long kWaitLimit = 2000000000LL;  // ~1 s of SM clock
 // Lead tiles per item in the stream-K sequence: the fixed cost of a piece
 // (Q load and pipeline fill, epilogue or partial write) measured as ~5 K/V
-// tiles, so CTAs whose ranges hold many short items get fewer tiles. Where
-// the resulting range boundaries fall also decides how many items are split
-// (partial writes, merges), so msf_plan_tune_attention can pick another
-// count per plan by timing a few.
+// tiles, so CTAs whose ranges hold many short items get fewer tiles.
 constexpr int kItemLeadTiles = 5;
 
 struct TcSeg {
@@ -872,7 +869,7 @@ msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st) {
             ts.tile0 = tg.n_tiles;
             tg.n_tiles += (sg.len + kBlockN - 1) / kBlockN;
         }
-        tg.n_virt = tg.n_tiles + (P.attn_lead >= 0 ? P.attn_lead : kItemLeadTiles);
+        tg.n_virt = tg.n_tiles + kItemLeadTiles;
         tg.tile_base = total_tiles;
         tg.item_base = item_base;
         total_tiles += (long long)tg.n_items * tg.n_virt;
@@ -891,7 +888,7 @@ msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st) {
     // only the rest of the sequence is split evenly (stream-K).
     tp.dp_rounds = 0;
     tp.dp_stride = tp.g[0].n_virt;
-    if (P.attn_dp != 0 && tp.n_groups > 0) tp.dp_rounds = (int)(tp.g[0].n_items / ncta);
+    if (tp.n_groups > 0) tp.dp_rounds = (int)(tp.g[0].n_items / ncta);
     tp.t_sk = (long long)tp.dp_rounds * ncta * tp.dp_stride;
 
     if (P.D == 128) {

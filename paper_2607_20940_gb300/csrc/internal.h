@@ -36,8 +36,6 @@ struct msf_plan {
     // tensor-core attention scheduling state in the workspace
     int attn_items;     // 256-row query blocks over all groups, streams and heads
     int attn_max_ctas;  // persistent CTAs the partial-result slots are sized for
-    int attn_lead;      // lead tiles per item in the attention's stream-K sequence (-1: default)
-    int attn_dp;        // 1: whole items of the longest group first (data-parallel rounds), 0: off
     size_t ws_bytes;
     float scale;      // softmax scale
 

@@ -161,8 +161,6 @@ extern "C" msf_status msf_plan_create(const msf_plan_desc* desc, msf_plan_t* out
         p->attn_max_ctas = (int)(tiles < msf::kAttnMaxCtas ? tiles : msf::kAttnMaxCtas);
     }
     p->ws_bytes = msf::workspace_bytes(*p);
-    p->attn_lead = -1;
-    p->attn_dp = 1;
     p->hist_count = d.history_frames;
     p->hist_oldest = 0;
     p->hist_spare = d.history_frames;

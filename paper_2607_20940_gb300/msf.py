@@ -37,7 +37,6 @@ EXPORTS = (
     "msf_plan_device_status", "msf_kernel_launches", "msf_unpatchify_noalloc",
     "msf_selftest_wait_timeout", "msf_history_commit", "msf_mssa_forward_lse",
     "msf_mssa_backward", "msf_mssa_backward_simt", "msf_history_get", "msf_history_set",
-    "msf_plan_tune_attention",
 )
 
 
@@ -106,7 +105,6 @@ def _load():
         "msf_unpatchify_noalloc": (ctypes.c_int, [P, I32, VP, VP, VP, VP]),
         "msf_selftest_wait_timeout": (ctypes.c_int, [P, ctypes.c_int64, VP]),
         "msf_history_commit": (ctypes.c_int, [P]),
-        "msf_plan_tune_attention": (ctypes.c_int, [P, VP, VP, VP, VP, VP]),
         "msf_history_get": (ctypes.c_int, [P, ctypes.POINTER(msf_history_state)]),
         "msf_history_set": (ctypes.c_int, [P, ctypes.POINTER(msf_history_state)]),
         "msf_mssa_forward_lse": (ctypes.c_int, [P, VP, VP, VP, VP, VP, VP]),
@@ -254,11 +252,6 @@ def msf_history_set(plan: int, st: msf_history_state) -> None:
     _check(_lib.msf_history_set(plan, ctypes.byref(st)), "msf_history_set")
 
 
-def msf_plan_tune_attention(plan: int, q, k_win, v_win, out, stream=None) -> None:
-    _check(_lib.msf_plan_tune_attention(plan, _ptr(q), _ptr(k_win), _ptr(v_win), _ptr(out),
-                                        _stream(stream)), "msf_plan_tune_attention")
-
-
 def msf_history_commit(plan: int) -> None:
     _check(_lib.msf_history_commit(plan), "msf_history_commit")
 
@@ -365,9 +358,6 @@ class Plan:
         import torch
         return torch.empty(int(self.info.backward_workspace_bytes), dtype=torch.uint8,
                            device=device)
-
-    def tune_attention(self, q, k_win, v_win, out, stream=None):
-        msf_plan_tune_attention(self.handle, q, k_win, v_win, out, stream)
 
     def mssa_forward_simt(self, q, k_win, v_win, out, stream=None):
         msf_mssa_forward_simt(self.handle, q, k_win, v_win, out, stream)

@@ -328,22 +328,3 @@ def test_window_pass_layer(layer):
                                     synth.to_f64(m["w_out"]))
     e2 = np.abs(lat_out.double().cpu().numpy() - ref_lat)
     assert e2.max() <= 2.0 ** -7 * np.abs(ref_lat).max() + 1e-3, e2.max()
-
-
-def test_tuned_attention_matches_oracle():
-    """After msf_plan_tune_attention picks the stream-K split for the plan the
-    output is unchanged in quality (every candidate computes the same thing)."""
-    w = RAGGED
-    x = synth.attention_inputs(w, BF16)
-    plan = make_plan(w, BF16)
-    dx = device_inputs(x, w.history_capacity)
-    bind(plan, dx)
-    out = torch.empty_like(dx["q"])
-    plan.kv_resample(dx["k_win"], dx["v_win"])
-    plan.tune_attention(dx["q"], dx["k_win"], dx["v_win"], out)
-    out.fill_(float("nan"))
-    plan.mssa_forward(dx["q"], dx["k_win"], dx["v_win"], out)
-    torch.cuda.synchronize()
-    assert plan.device_status() == msf().MSF_OK
-    mx, mean = err_stats(out, oracle_mssa(x, w, 0))
-    assert mx <= BF16_MAX and mean <= BF16_MEAN, (mx, mean)
