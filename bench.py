@@ -220,7 +220,8 @@ def other_configs(msf, synth, dev, flush, peaks, rank):
     """The remaining configurations of the workload family, measured after the
     timed region: the three-scale 48x80 window, the training direction (forward
     with the row log-sum-exp and the MSSA gradient), the paper's chunked layout
-    (3 latent frames per state) beside its all-fine window, the B=4 streaming rollout
+    (3 latent frames per state) beside its all-fine window, the STRIDED Subsample
+    reading at the 480p layer, the B=4 streaming rollout
     (120 steps, history 2 -> capacity 4), the 30-layer window pass, and the
     bandwidth of the pyramid and embedding kernels."""
     import torch
@@ -266,6 +267,30 @@ def other_configs(msf, synth, dev, flush, peaks, rank):
         raise RuntimeError("device status error (three-scale)")
     plan.close()
     del t
+
+    # ---- the literal stride-2 reading of Subsample (STRIDED: top-left token
+    #      of each block) at the 480p layer: pyramid and attention
+    wl = synth.LAYER_480P
+    plan = msf.Plan(msf.make_desc(wl.scales, wl.grid_h, wl.grid_w, wl.heads, wl.head_dim, wl.sink_tokens,
+                                  wl.history_frames, wl.history_capacity, batch=wl.batch,
+                                  resample=msf.MSF_RESAMPLE_STRIDED))
+    N, G, H, D, B = plan.info.n_tokens, wl.fine_tokens, wl.heads, wl.head_dim, wl.batch
+    ts_ = {k: rnd((B, N, H, D)) for k in ("q", "k_win", "v_win")}
+    ts_["k_sink"], ts_["v_sink"] = rnd((B, wl.sink_tokens, H, D)), rnd((B, wl.sink_tokens, H, D))
+    for k in ("k_hist", "v_hist"):
+        ts_[k] = rnd((B, wl.history_capacity, G, H, D))
+    ws_s = plan.workspace(dev)
+    plan.bind(ws_s, ts_["k_sink"], ts_["v_sink"], ts_["k_hist"], ts_["v_hist"])
+    out_s = torch.empty_like(ts_["q"])
+    pyr_ms = _timed(lambda: plan.kv_resample(ts_["k_win"], ts_["v_win"], msf.MSF_RESAMPLE_WINDOW_ONLY), flush)
+    attn_ms = _timed(lambda: plan.mssa_forward(ts_["q"], ts_["k_win"], ts_["v_win"], out_s), flush)
+    fl = plan.info.attention_flops
+    if plan.device_status() != msf.MSF_OK:
+        raise RuntimeError("device status error (strided)")
+    out["strided_480p"] = {"workload": wl.name, "resample": "STRIDED", "attention_us": attn_ms * 1e3,
+                           "tflops": fl / (attn_ms * 1e-3) / 1e12, "pyramid_window_us": pyr_ms * 1e3}
+    plan.close()
+    del ts_, ws_s, out_s
 
     # ---- training direction at the 480p layer: forward with the row
     #      log-sum-exp, then the MSSA gradient (dq, dk_win, dv_win)
