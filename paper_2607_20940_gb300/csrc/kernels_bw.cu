@@ -56,63 +56,92 @@ struct Vec<float> {
 };
 
 // Two adjacent 16-byte vectors of one pooled token, K and V. With the stride
-// known at compile time every source load is issued before the first add, so
-// a thread keeps 4*S*S loads in flight. ck/cv (NULL = none) receive a copy of
-// every source vector read, at its source token index (the staged history
-// head: one read serves the ring copy and the pooled level).
+// known at compile time the loads of RG tap rows are issued before their first
+// add (all 4*S*S of them for S <= 2; one row of 4*S for S = 4, which keeps the
+// thread under ~128 registers so the kernel does not spill). ck/cv (NULL =
+// none) receive a copy of every source vector read, at its source token index
+// (the staged history head: one read serves the ring copy and the pooled
+// level). Sums run in the fixed (dy, dx) order whatever RG is.
 template <typename T, int S>
 __device__ __forceinline__ void pool_pair(const char* sk, const char* sv, char* dk, char* dv,
                                           char* ck, char* cv, int src_gw, int i, int jj,
                                           size_t row, int mode) {
-    uint4 xk[S * S][2], xv[S * S][2];
-    const int taps = (mode == MSF_RESAMPLE_STRIDED && !ck) ? 1 : S * S;
+    const bool strided = mode == MSF_RESAMPLE_STRIDED;
+    if (S == 1 || (strided && !ck)) {
+        const size_t src = (size_t)((S * i) * src_gw + S * jj) * row;
+        const uint4 k0 = __ldg(reinterpret_cast<const uint4*>(sk + src));
+        const uint4 k1 = __ldg(reinterpret_cast<const uint4*>(sk + src + 16));
+        const uint4 v0 = __ldg(reinterpret_cast<const uint4*>(sv + src));
+        const uint4 v1 = __ldg(reinterpret_cast<const uint4*>(sv + src + 16));
+        if (ck) {  // S == 1 here
+            *reinterpret_cast<uint4*>(ck + src) = k0;
+            *reinterpret_cast<uint4*>(ck + src + 16) = k1;
+            *reinterpret_cast<uint4*>(cv + src) = v0;
+            *reinterpret_cast<uint4*>(cv + src + 16) = v1;
+        }
+        *reinterpret_cast<uint4*>(dk) = k0;
+        *reinterpret_cast<uint4*>(dk + 16) = k1;
+        *reinterpret_cast<uint4*>(dv) = v0;
+        *reinterpret_cast<uint4*>(dv + 16) = v1;
+        return;
+    }
+    constexpr int RG = S <= 2 ? S : 1;  // tap rows whose loads are in flight together
+    float ak[2][Vec<T>::n], av[2][Vec<T>::n];
 #pragma unroll
-    for (int t = 0; t < S * S; ++t) {
-        if (t < taps) {
-            const int dy = t / S, dx = t % S;
+    for (int h = 0; h < 2; ++h)
+#pragma unroll
+        for (int e = 0; e < Vec<T>::n; ++e) ak[h][e] = av[h][e] = 0.f;
+#pragma unroll 1
+    for (int y0 = 0; y0 < S; y0 += RG) {
+        uint4 xk[RG * S][2], xv[RG * S][2];
+#pragma unroll
+        for (int t = 0; t < RG * S; ++t) {
+            const int dy = y0 + t / S, dx = t % S;
             const size_t src = (size_t)((S * i + dy) * src_gw + S * jj + dx) * row;
             xk[t][0] = __ldg(reinterpret_cast<const uint4*>(sk + src));
             xk[t][1] = __ldg(reinterpret_cast<const uint4*>(sk + src + 16));
             xv[t][0] = __ldg(reinterpret_cast<const uint4*>(sv + src));
             xv[t][1] = __ldg(reinterpret_cast<const uint4*>(sv + src + 16));
         }
-    }
-    if (ck) {
+        if (ck) {
 #pragma unroll
-        for (int t = 0; t < S * S; ++t) {
-            const int dy = t / S, dx = t % S;
-            const size_t src = (size_t)((S * i + dy) * src_gw + S * jj + dx) * row;
-            *reinterpret_cast<uint4*>(ck + src) = xk[t][0];
-            *reinterpret_cast<uint4*>(ck + src + 16) = xk[t][1];
-            *reinterpret_cast<uint4*>(cv + src) = xv[t][0];
-            *reinterpret_cast<uint4*>(cv + src + 16) = xv[t][1];
+            for (int t = 0; t < RG * S; ++t) {
+                const int dy = y0 + t / S, dx = t % S;
+                const size_t src = (size_t)((S * i + dy) * src_gw + S * jj + dx) * row;
+                *reinterpret_cast<uint4*>(ck + src) = xk[t][0];
+                *reinterpret_cast<uint4*>(ck + src + 16) = xk[t][1];
+                *reinterpret_cast<uint4*>(cv + src) = xv[t][0];
+                *reinterpret_cast<uint4*>(cv + src + 16) = xv[t][1];
+            }
         }
+        if (strided) {  // the block's top-left vectors
+            if (y0 == 0) {
+                *reinterpret_cast<uint4*>(dk) = xk[0][0];
+                *reinterpret_cast<uint4*>(dk + 16) = xk[0][1];
+                *reinterpret_cast<uint4*>(dv) = xv[0][0];
+                *reinterpret_cast<uint4*>(dv + 16) = xv[0][1];
+            }
+            continue;
+        }
+#pragma unroll
+        for (int t = 0; t < RG * S; ++t)
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                Vec<T>::add(ak[h], xk[t][h]);
+                Vec<T>::add(av[h], xv[t][h]);
+            }
     }
-    if (S == 1 || mode == MSF_RESAMPLE_STRIDED) {
-        *reinterpret_cast<uint4*>(dk) = xk[0][0];
-        *reinterpret_cast<uint4*>(dk + 16) = xk[0][1];
-        *reinterpret_cast<uint4*>(dv) = xv[0][0];
-        *reinterpret_cast<uint4*>(dv + 16) = xv[0][1];
-        return;
-    }
+    if (strided) return;
+    const float mul = 1.0f / (float)(S * S);
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
-        float ak[Vec<T>::n], av[Vec<T>::n];
-#pragma unroll
-        for (int e = 0; e < Vec<T>::n; ++e) ak[e] = av[e] = 0.f;
-#pragma unroll
-        for (int t = 0; t < S * S; ++t) {  // fixed (dy, dx) order
-            Vec<T>::add(ak, xk[t][h]);
-            Vec<T>::add(av, xv[t][h]);
-        }
-        const float mul = 1.0f / (float)(S * S);
-        *reinterpret_cast<uint4*>(dk + 16 * h) = Vec<T>::pack(ak, mul);
-        *reinterpret_cast<uint4*>(dv + 16 * h) = Vec<T>::pack(av, mul);
+        *reinterpret_cast<uint4*>(dk + 16 * h) = Vec<T>::pack(ak[h], mul);
+        *reinterpret_cast<uint4*>(dv + 16 * h) = Vec<T>::pack(av[h], mul);
     }
 }
 
 template <typename T>
-__global__ void __launch_bounds__(256) pool_kernel(const PoolBatch jobs) {
+__global__ void __launch_bounds__(256, 2) pool_kernel(const PoolBatch jobs) {
     ptx::grid_dep_wait();
     ptx::grid_dep_launch();
     const PoolJob& jb = jobs.j[blockIdx.y];

@@ -2,6 +2,7 @@
 synthetic inputs so that `ncu -k <kernel>` can capture it in isolation.
 
     python -m paper_2607_20940_gb300.profile_cases pool     # K/V pyramid at three sizes
+    python -m paper_2607_20940_gb300.profile_cases pool_fused  # pyramid + staged history head
     python -m paper_2607_20940_gb300.profile_cases embed    # MSP patchify + tier embedding
     python -m paper_2607_20940_gb300.profile_cases deembed  # de-embedding + unpatchify
     python -m paper_2607_20940_gb300.profile_cases backward # forward with lse + MSSA gradient
@@ -20,16 +21,17 @@ import torch
 from paper_2607_20940_gb300 import msf, synth
 
 
-def _setup(w, embed=False):
+def _setup(w, embed=False, fused=False):
     dev = torch.device("cuda", 0)
     x = synth.attention_inputs(w)
     plan = msf.Plan(msf.make_desc(w.scales, w.grid_h, w.grid_w, w.heads, w.head_dim, w.sink_tokens,
                                   w.history_frames, w.history_capacity, batch=w.batch,
                                   latent_channels=w.latent_channels, patch=w.patch,
-                                  embed_dim=w.embed_dim if embed else 0))
+                                  embed_dim=w.embed_dim if embed else 0, fused_append=int(fused)))
     d = {k: v.to(dev) for k, v in x.items()}
     for k in ("k_hist", "v_hist"):
-        ring = torch.zeros((w.batch, max(w.history_capacity, 1)) + tuple(d[k].shape[2:]),
+        slots = w.history_capacity + 1 if fused else max(w.history_capacity, 1)
+        ring = torch.zeros((w.batch, slots) + tuple(d[k].shape[2:]),
                            dtype=d[k].dtype, device=dev)
         ring[:, :w.history_frames] = d[k]
         d[k] = ring
@@ -49,6 +51,15 @@ def run(case: str) -> None:
             for _ in range(2):
                 flush.fill_(1)
                 plan.kv_resample(d["k_win"], d["v_win"], mode)
+            torch.cuda.synchronize()
+            assert plan.device_status() == msf.MSF_OK
+            plan.close()
+    elif case == "pool_fused":
+        for w in (synth.LAYER_480P, synth.STREAM_480P):
+            plan, d, _ = _setup(w, fused=True)
+            for _ in range(2):
+                flush.fill_(1)
+                plan.kv_resample(d["k_win"], d["v_win"], msf.MSF_RESAMPLE_WINDOW_ONLY)
             torch.cuda.synchronize()
             assert plan.device_status() == msf.MSF_OK
             plan.close()
@@ -101,7 +112,8 @@ def run(case: str) -> None:
         assert plan.device_status() == msf.MSF_OK
         plan.close()
     else:
-        raise SystemExit(f"unknown case {case!r}: pool, embed, deembed, backward or attention")
+        raise SystemExit(f"unknown case {case!r}: pool, pool_fused, embed, deembed, backward or "
+                         "attention")
 
 
 if __name__ == "__main__":
