@@ -36,10 +36,61 @@ __device__ __forceinline__ float st1(float x) { return x; }
 template <>
 __device__ __forceinline__ __nv_bfloat16 st1(float x) { return __float2bfloat16_rn(x); }
 
+// 8 consecutive elements (16-byte aligned) widened to fp32, in one or two
+// 16-byte loads.
+__device__ __forceinline__ void ld8(const __nv_bfloat16* p, float* x) {
+    const uint4 v = __ldg(reinterpret_cast<const uint4*>(p));
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float2 f = __bfloat1622float2(h[i]);
+        x[2 * i] = f.x;
+        x[2 * i + 1] = f.y;
+    }
+}
+__device__ __forceinline__ void ld8(const float* p, float* x) {
+    const float4 a = __ldg(reinterpret_cast<const float4*>(p));
+    const float4 b = __ldg(reinterpret_cast<const float4*>(p + 4));
+    x[0] = a.x, x[1] = a.y, x[2] = a.z, x[3] = a.w;
+    x[4] = b.x, x[5] = b.y, x[6] = b.z, x[7] = b.w;
+}
+
+// E (2 or 4) consecutive fp32 values in one aligned vector load; E values
+// stored as the dtype in one vector store.
+template <int E>
+__device__ __forceinline__ void ldE(const float* p, float* x) {
+    if (E == 4) {
+        const float4 v = __ldg(reinterpret_cast<const float4*>(p));
+        x[0] = v.x, x[1] = v.y, x[2] = v.z, x[3] = v.w;
+    } else {
+        const float2 v = __ldg(reinterpret_cast<const float2*>(p));
+        x[0] = v.x, x[1] = v.y;
+    }
+}
+template <int E>
+__device__ __forceinline__ void stE(float* p, const float* x) {
+    if (E == 4)
+        *reinterpret_cast<float4*>(p) = make_float4(x[0], x[1], x[2], x[3]);
+    else
+        *reinterpret_cast<float2*>(p) = make_float2(x[0], x[1]);
+}
+template <int E>
+__device__ __forceinline__ void stE(__nv_bfloat16* p, const float* x) {
+    if (E == 4) {
+        __nv_bfloat162 a = __floats2bfloat162_rn(x[0], x[1]), b = __floats2bfloat162_rn(x[2], x[3]);
+        *reinterpret_cast<uint2*>(p) =
+            make_uint2(*reinterpret_cast<uint32_t*>(&a), *reinterpret_cast<uint32_t*>(&b));
+    } else {
+        *reinterpret_cast<__nv_bfloat162*>(p) = __floats2bfloat162_rn(x[0], x[1]);
+    }
+}
+
 constexpr float kLog2e = 1.4426950408889634f;
 
 // delta[b, h, t] = sum_d dout * out: a row of D elements is shared by D/8
-// consecutive threads, each loading 8 elements of both tensors.
+// consecutive threads, each loading 8 elements of both tensors (one 16-byte
+// vector each for bf16). One row per thread group: giving a warp several
+// rows' loads at once (fewer, fuller warps) measured twice as slow.
 template <typename T, int D>
 __global__ void __launch_bounds__(256) bwd_delta_kernel(const BwdCommon c) {
     ptx::grid_dep_wait();
@@ -56,10 +107,11 @@ __global__ void __launch_bounds__(256) bwd_delta_kernel(const BwdCommon c) {
         t = (int)((w / c.H) % c.N);
         b = (int)(w / ((long long)c.H * c.N));
         const size_t off = (size_t)b * c.bstride + (((size_t)t * c.H + h) * D + 8 * part) * sizeof(T);
-        const T* go = (const T*)(c.dout + off);
-        const T* o = (const T*)(c.out + off);
+        float go[8], o[8];
+        ld8((const T*)(c.dout + off), go);
+        ld8((const T*)(c.out + off), o);
 #pragma unroll
-        for (int i = 0; i < 8; ++i) acc = fmaf(ld1<T>(go + i), ld1<T>(o + i), acc);
+        for (int i = 0; i < 8; ++i) acc = fmaf(go[i], o[i], acc);
     }
 #pragma unroll
     for (int s = kTpr / 2; s > 0; s >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, s);
@@ -223,7 +275,9 @@ __global__ void __launch_bounds__(128) bwd_dkdv_kernel(const BwdCommon c, const 
 }
 
 // dk_win, dv_win: one warp per (stream, token, head) row; a lane holds D/32
-// consecutive elements. Entries of the token's state come in a fixed order.
+// consecutive elements (one vector load per entry). Entries of the token's
+// state come in a fixed order. Issuing every entry's loads before the first
+// add (fewer warps resident) measured slower than this loop.
 template <typename T, int D>
 __global__ void __launch_bounds__(256) bwd_gather_kernel(const BwdCommon c, const GatherArgs g,
                                                          T* __restrict__ dk, T* __restrict__ dv) {
@@ -258,18 +312,18 @@ __global__ void __launch_bounds__(256) bwd_gather_kernel(const BwdCommon c, cons
             row = en.crow0 + (i / s) * en.out_gw + j / s;
         }
         const size_t o = (((size_t)b * c.R + row) * c.H + h) * D + E * lane;
+        float xk[E], xv[E];
+        ldE<E>(c.dk_ctx + o, xk);
+        ldE<E>(c.dv_ctx + o, xv);
 #pragma unroll
         for (int e = 0; e < E; ++e) {
-            ak[e] = fmaf(wgt, c.dk_ctx[o + e], ak[e]);
-            av[e] = fmaf(wgt, c.dv_ctx[o + e], av[e]);
+            ak[e] = fmaf(wgt, xk[e], ak[e]);
+            av[e] = fmaf(wgt, xv[e], av[e]);
         }
     }
     const size_t o = (((size_t)b * c.N + t) * c.H + h) * D + E * lane;
-#pragma unroll
-    for (int e = 0; e < E; ++e) {
-        dk[o + e] = st1<T>(ak[e]);
-        dv[o + e] = st1<T>(av[e]);
-    }
+    stE<E>(dk + o, ak);
+    stE<E>(dv + o, av);
 }
 
 }  // namespace
