@@ -179,6 +179,94 @@ def run_reference(args, w):
     print(json.dumps(line))
 
 
+def oracle_other_configs():
+    """The oracle (fp64 numpy, as it stands) on the host cores for the other
+    workloads of the family, each on a bounded sample: the tiny window whole,
+    the three-scale window on 2 of its 16 heads, the 30-layer pass on layers
+    0, 15 and 29 (each: patchify + tier embedding of the window, MSSA on 2 of
+    12 heads, de-embedding + unpatchify of the head), and the B=4 rollout on
+    steps 0, 1, 2, 60 and 119 of stream 0 (2 of 12 heads; the history holds
+    min(2 + step, 4) frames). Sampled heads, layers and steps are scaled up
+    to the whole workload and marked "extrapolated" (the oracle's time is
+    linear in heads, layers, streams and steps)."""
+    import dataclasses
+
+    import torch
+
+    from oracle import msp as omsp
+    from oracle import mssa as omssa
+    from oracle import schedule
+    from paper_2607_20940_gb300 import synth
+    f = synth.to_f64
+
+    def flops(w, n_hist, heads, batch=1):
+        return schedule.attention_flops(w.scales, w.grid_h, w.grid_w, w.sink_tokens, n_hist, heads,
+                                        w.head_dim, batch, w.frames)
+
+    def attn(w, x, heads):
+        t0 = time.perf_counter()
+        omssa.mssa_forward(f(x["q"]), f(x["k_win"]), f(x["v_win"]), f(x["k_sink"]), f(x["v_sink"]),
+                           f(x["k_hist"]), f(x["v_hist"]), w.scales, w.grid_h, w.grid_w, heads=heads,
+                           frames=w.frames)
+        return time.perf_counter() - t0
+
+    res = {}
+    # tiny window (T=3, 8x8, scales (1,1,2), 2 heads of 64): the whole call
+    w = synth.TINY
+    dt = attn(w, synth.attention_inputs(w, torch.float32), None)
+    fl = flops(w, w.history_frames, w.heads)
+    res["tiny"] = {"workload": w.name, "seconds": dt, "gflop": fl / 1e9, "tflops": fl / dt / 1e12,
+                   "sample": "whole call (fp32 inputs)"}
+    # three-scale 48x80 window: 2 of 16 heads
+    w = synth.THREE_SCALE
+    hs = [0, 8]
+    dt = attn(w, synth.attention_inputs(w, torch.bfloat16), hs) * w.heads / len(hs)
+    fl = flops(w, w.history_frames, w.heads)
+    res["three_scale"] = {"workload": w.name, "seconds": dt, "gflop": fl / 1e9, "tflops": fl / dt / 1e12,
+                          "sample": "2 of 16 heads, extrapolated to 16"}
+    # 30-layer window pass: layers 0, 15, 29
+    w = synth.PASS_480P
+    hs = [0, 6]
+    G = w.grid_h * w.grid_w
+    per_layer = []
+    for layer in (0, 15, 29):
+        x = synth.attention_inputs(w, torch.bfloat16, seed=w.seed + layer)
+        m = synth.msp_inputs(w, torch.bfloat16, seed=w.seed + layer)
+        tiers = {s: f(m["w_tier"][s]) for s in set(w.scales)}
+        lat, w_out = f(m["latent"]), f(m["w_out"])
+        t0 = time.perf_counter()
+        tok = omsp.patchify_window(lat, w.scales, w.patch, tiers)
+        t_msp = time.perf_counter() - t0
+        t_attn = attn(w, x, hs)
+        t0 = time.perf_counter()
+        omsp.unpatchify_state(tok[:, :G], w.patch, w.latent_channels, w.grid_h * w.patch,
+                              w.grid_w * w.patch, w_out)
+        t_msp += time.perf_counter() - t0
+        per_layer.append(t_msp + t_attn * w.heads / len(hs))
+    dt = statistics.mean(per_layer) * w.layers
+    fl = flops(w, w.history_frames, w.heads) * w.layers
+    res["window_pass_30"] = {"workload": w.name, "seconds": dt, "gflop": fl / 1e9,
+                             "tflops": fl / dt / 1e12,
+                             "sample": "layers 0, 15, 29 (2 of 12 heads each), extrapolated to 30 layers"}
+    # B=4 streaming rollout: steps 0, 1, 2, 60, 119 of stream 0
+    w = synth.STREAM_480P
+    w1 = dataclasses.replace(w, batch=1)
+    hs = [0, 6]
+    n_hist = lambda s: min(w.history_frames + s, w.history_capacity)  # noqa: E731
+    samples = {}
+    for s in (0, 1, 2, 60, 119):
+        x = synth.attention_inputs(w1, torch.bfloat16, seed=w.seed, history_frames=n_hist(s))
+        samples[s] = attn(w1, x, hs) * w.heads / len(hs) * w.batch
+    # steps 3..119 all run at capacity: the mean of the two sampled ones
+    full = samples[0] + samples[1] + samples[2] + (w.steps - 3) * (samples[60] + samples[119]) / 2
+    fl = sum(flops(w, n_hist(s), w.heads, w.batch) for s in range(w.steps))
+    res["stream_b4"] = {"workload": w.name, "seconds": full, "gflop": fl / 1e9, "tflops": fl / full / 1e12,
+                        "seconds_per_step_at_cap": samples[119],
+                        "sample": "steps 0, 1, 2, 60, 119 of stream 0 (2 of 12 heads), extrapolated "
+                                  "to 4 streams x 12 heads x 120 steps"}
+    return res
+
+
 def _traffic_from_profile(kernel_src: str):
     """dram bytes per launch of the attention kernel from the committed ncu
     summary, if it was taken on the current kernel source."""
@@ -715,7 +803,8 @@ def main():
         _oracle_step(w, x, mi)
         dt = time.perf_counter() - t0
         cpu = {"value": flops / dt / 1e12, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
-               "sample": f"one full 480p step (all 12 heads) in fp64 numpy, {dt:.1f} s"}
+               "sample": f"one full 480p step (all 12 heads) in fp64 numpy, {dt:.1f} s",
+               "other_configs": oracle_other_configs()}
 
     peaks, peak_src = _peaks()
     attn_avg_ms = statistics.mean(attn_ms)
@@ -766,6 +855,8 @@ def main():
                         "stream; each step's latent is read back; all copies inside the timed window",
                 "serial_ms_per_step": e2e_serial_ms / args.steps,
                 "serial_value": world * flops * args.steps / (e2e_serial_ms * 1e-3) / 1e12},
+        "step_us": {"mean": ms_per_step * 1e3, "p50": 1e3 * statistics.median(step_ms),
+                    "p99": 1e3 * sorted(step_ms)[min(len(step_ms) - 1, int(0.99 * len(step_ms)))]},
         "gpu_launches": launches,
         "clocks": clk,
         "device_status": msf.msf_status_string(status),
