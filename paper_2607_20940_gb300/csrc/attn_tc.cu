@@ -62,6 +62,8 @@ constexpr long long kWaitLimit = 2000000000LL;  // ~1 s of SM clock
 // (Q load and pipeline fill, epilogue or partial write) measured as ~5 K/V
 // tiles, so CTAs whose ranges hold many short items get fewer tiles.
 constexpr int kItemLeadTiles = 5;
+// Pieces of one item that the merging CTA combines from one batch of loads.
+constexpr int kMergeBatch = 8;
 
 struct TcSeg {
     int map;
@@ -127,6 +129,15 @@ struct Piece {
     bool whole;
     long long item_start;  // global index of the item's first real tile
     long long t_next;      // sequence position after this piece
+};
+
+// A merge handed from the softmax warps to the helper warps.
+struct MergeJob {
+    long long item_rel;  // sequence position of the item's first real tile, relative to t_sk
+    long long c1, c2;    // CTAs holding its pieces
+    unsigned int* cnt;   // the item's counter word
+    int q_row0, q_end, b, h;
+    int stop;            // no more jobs
 };
 
 __device__ __forceinline__ long long cta_begin(long long c, long long T, long long n) {
@@ -195,6 +206,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     __shared__ uint64_t k_full[kStages], k_empty[kStages], v_full[kVStages];
     __shared__ uint64_t s_full[2], p_full[2];
     __shared__ uint64_t epi_written, epi_decided;
+    __shared__ uint64_t job_full, job_empty, job_ready;
+    __shared__ MergeJob job;
     __shared__ uint32_t tmem_base_sh;
     __shared__ int abort_flag;
     __shared__ int merge_flag;
@@ -202,21 +215,24 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const long long T = p.total_tiles;
     const long long ncta = gridDim.x;
-    // Work of this CTA: dp_rounds whole items of the first group (items
-    // blockIdx.x, blockIdx.x + ncta, ...), then its equal share of the rest of
-    // the sequence (stream-K), which starts at t_sk.
+    // Work of this CTA: its equal share of the stream-K part of the sequence
+    // (which starts at t_sk) first, then dp_rounds whole items of the first
+    // group (items blockIdx.x, blockIdx.x + ncta, ...). Split items thus end
+    // early, and their merges run on the helper warps beside the whole items.
     const long long Tsk = T - p.t_sk;
     const long long r0 = p.t_sk + cta_begin(blockIdx.x, Tsk, ncta);
     const long long r1 = p.t_sk + cta_begin(blockIdx.x + 1, Tsk, ncta);
     auto phase_range = [&](int ph, long long& a0, long long& a1) {
-        if (ph < p.dp_rounds) {
-            a0 = ((long long)blockIdx.x + (long long)ph * ncta) * p.dp_stride;
-            a1 = a0 + p.dp_stride;
-        } else {
+        if (ph == 0) {
             a0 = r0;
             a1 = r1;
+        } else {
+            a0 = ((long long)blockIdx.x + (long long)(ph - 1) * ncta) * p.dp_stride;
+            a1 = a0 + p.dp_stride;
         }
     };
+    // Merges of split items go to the helper warps while whole items follow.
+    const bool helper_merges = p.dp_rounds > 0;
 
     if (threadIdx.x == 0) {
         abort_flag = 0;
@@ -236,6 +252,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         ptx::mbar_init(&epi_written, 8);
         ptx::mbar_init(&epi_decided, 1);
+        ptx::mbar_init(&job_full, 1);
+        ptx::mbar_init(&job_empty, 2);  // one arrival per helper warp
+        ptx::mbar_init(&job_ready, 1);  // the pieces of the job are all written
         ptx::fence_mbar_init();
     }
     if (warp == 2) {
@@ -442,6 +461,125 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (lane == 0) atomicOr(p.status, kDevTimeout);
             }
         }
+        } else if (helper_merges) {
+        // ========================== merge helpers ===========================
+        // Warps 2 and 3 merge the split items whose last piece this CTA
+        // finished, while the softmax warps go on with whole items: every
+        // piece's partial result is in its slot, and each of the 64 threads
+        // combines four rows, in piece order (the same bits whichever CTA
+        // merges). Loads go out in batches (m and l of every piece, then one
+        // 16-column chunk of two pieces), as each round trip to L2 costs
+        // about a microsecond.
+        const int ht = (warp - 2) * 32 + lane;
+        for (int jn = 0;; ++jn) {
+            bool okj = ptx::mbar_wait_bounded(&job_full, (uint32_t)(jn & 1), abort_p, p.wait_limit);
+            okj = __all_sync(0xffffffffu, okj);
+            if (!okj) break;
+            const volatile MergeJob& vj = job;
+            if (vj.stop) break;
+            const long long c1 = vj.c1, item_rel = vj.item_rel;
+            const int n = (int)(vj.c2 - c1) + 1;
+            const int q_row0 = vj.q_row0, q_end = vj.q_end, jb = vj.b, jh = vj.h;
+            unsigned int* const jcnt = vj.cnt;
+            // The other pieces have finished their tiles; wait (bounded) until
+            // their partial results are written and fenced, then reset the
+            // counter for the next launch.
+            if (warp == 2) {
+                if (lane == 0) {
+                    const long long w0 = clock64();
+                    while ((*(volatile unsigned int*)jcnt >> 16) != (unsigned int)(n - 1)) {
+                        if (*abort_p || clock64() - w0 > p.wait_limit) {
+                            *abort_p = 1;
+                            atomicOr(p.status, kDevTimeout);
+                            break;
+                        }
+                    }
+                    atomicExch(jcnt, 0u);
+                    __threadfence();
+                    ptx::mbar_arrive(&job_ready);
+                }
+                __syncwarp();
+            } else {
+                okj = ptx::mbar_wait_bounded(&job_ready, (uint32_t)(jn & 1), abort_p, p.wait_limit);
+                okj = __all_sync(0xffffffffu, okj);
+                if (!okj) break;
+            }
+            if (*abort_p) break;
+            int off[kMergeBatch];
+#pragma unroll
+            for (int k = 0; k < kMergeBatch; ++k)
+                off[k] = k < n ? slot_of(c1 + k, c1, item_rel, Tsk, ncta) * C::kSlotFloats : 0;
+#pragma unroll 1
+            for (int i = 0; i < 4; ++i) {
+                const int rr = i * 64 + ht;
+                const int qrow = q_row0 + rr;
+                float mv[kMergeBatch], lv[kMergeBatch];
+#pragma unroll
+                for (int k = 0; k < kMergeBatch; ++k) {
+                    mv[k] = k < n ? __ldcg(p.partials + off[k] + C::kSlotML + rr) : -INFINITY;
+                    lv[k] = k < n ? __ldcg(p.partials + off[k] + C::kSlotML + 2 * kBlockM + rr) : 0.f;
+                }
+                float M = -INFINITY;
+#pragma unroll
+                for (int k = 0; k < kMergeBatch; ++k) M = fmaxf(M, mv[k]);
+                float L = 0.f;
+#pragma unroll
+                for (int k = 0; k < kMergeBatch; ++k) {
+                    mv[k] = k < n ? ex2(mv[k] - M) : 0.f;  // piece k's weight
+                    L = fmaf(mv[k], lv[k], L);
+                }
+                const float inv = 1.0f / L;
+                const bool store = qrow < q_end;
+                if (store && p.lse)
+                    p.lse[((size_t)jb * p.H + jh) * p.N + qrow] = (M + log2f(L)) * 0.6931471805599453f;
+                __nv_bfloat16* dst = p.out + (size_t)jb * p.out_bstride + ((size_t)qrow * p.H + jh) * D;
+#pragma unroll 1
+                for (int ch = 0; ch < D / 16; ++ch) {
+                    float acc[16];
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) acc[e] = 0.f;
+#pragma unroll
+                    for (int k = 0; k < kMergeBatch; k += 2) {
+                        if (k >= n) break;
+                        const bool two = k + 1 < n;
+                        const float4* sa = reinterpret_cast<const float4*>(p.partials + off[k]) + rr;
+                        const float4* sb = reinterpret_cast<const float4*>(p.partials + off[k + 1]) + rr;
+                        float4 va[4], vb[4];
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const size_t q = (size_t)(ch * 4 + e) * 2 * kBlockM;
+                            va[e] = __ldcg(sa + q);
+                            vb[e] = two ? __ldcg(sb + q) : make_float4(0.f, 0.f, 0.f, 0.f);
+                        }
+                        const float wa = mv[k], wb = mv[k + 1];
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            acc[4 * e] = fmaf(wa, va[e].x, acc[4 * e]);
+                            acc[4 * e + 1] = fmaf(wa, va[e].y, acc[4 * e + 1]);
+                            acc[4 * e + 2] = fmaf(wa, va[e].z, acc[4 * e + 2]);
+                            acc[4 * e + 3] = fmaf(wa, va[e].w, acc[4 * e + 3]);
+                            if (two) {
+                                acc[4 * e] = fmaf(wb, vb[e].x, acc[4 * e]);
+                                acc[4 * e + 1] = fmaf(wb, vb[e].y, acc[4 * e + 1]);
+                                acc[4 * e + 2] = fmaf(wb, vb[e].z, acc[4 * e + 2]);
+                                acc[4 * e + 3] = fmaf(wb, vb[e].w, acc[4 * e + 3]);
+                            }
+                        }
+                    }
+                    if (store) {
+                        uint4* d4 = reinterpret_cast<uint4*>(dst + ch * 16);
+#pragma unroll
+                        for (int e = 0; e < 2; ++e)
+                            d4[e] = make_uint4(ptx::pack_bf16(acc[8 * e] * inv, acc[8 * e + 1] * inv),
+                                               ptx::pack_bf16(acc[8 * e + 2] * inv, acc[8 * e + 3] * inv),
+                                               ptx::pack_bf16(acc[8 * e + 4] * inv, acc[8 * e + 5] * inv),
+                                               ptx::pack_bf16(acc[8 * e + 6] * inv, acc[8 * e + 7] * inv));
+                    }
+                }
+            }
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&job_empty);
+        }
         }
     } else {
         ptx::setmaxnreg_inc<kSoftmaxRegs>();
@@ -455,7 +593,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float sl2 = p.scale_log2;
         bool ok = true;
         long long js = 0;
-        int piece = 0, nsplit = 0;
+        int piece = 0, nsplit = 0, nwritten = 0, njob = 0;
         for (int ph = 0; ph <= p.dp_rounds && ok; ++ph) {
         long long a0, a1;
         phase_range(ph, a0, a1);
@@ -465,9 +603,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (pc.u0 == pc.u1) continue;  // lead tiles only
             const TcGroup& G = p.g[pc.gi];
             float m_used = -INFINITY, l = 0.f;
+            // A split piece counts itself finished as its last tile starts (one
+            // thread, its result used only in the epilogue, so the atomic's
+            // round trip overlaps that tile): the last to count in merges.
+            unsigned int fin_old = 0;
+            unsigned int* const cnt = p.counters + G.item_base + pc.item;
             for (int u = pc.u0; u < pc.u1; ++u, ++js) {
                 int seg, row, valid;
                 tile_info(G, u, seg, row, valid);
+                if (!pc.whole && u == pc.u1 - 1 && warp == 4 && lane == 0) fin_old = atomicAdd(cnt, 1u);
                 ok = ptx::mbar_wait_bounded(&s_full[t], (uint32_t)(js & 1), abort_p, p.wait_limit);
                 ok = __all_sync(0xffffffffu, ok);
                 if (!ok) break;
@@ -589,53 +733,190 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 }
             } else {
-                // ---- split item: write this piece's partial result
-                // (only stream-K pieces are split: positions relative to t_sk)
+                // ---- split item (only stream-K pieces are split: positions
+                // relative to t_sk). The piece that counted itself finished
+                // last merges; every other piece writes its partial result.
                 const long long c1 = cta_of(pc.item_start - p.t_sk, Tsk, ncta);
                 const long long c2 = cta_of(pc.item_start + G.n_tiles - 1 - p.t_sk, Tsk, ncta);
                 const int slot = slot_of(blockIdx.x, c1, pc.item_start - p.t_sk, Tsk, ncta);
                 const int rr = t * kBlockM + r;
-                float* ps = p.partials + (size_t)slot * C::kSlotFloats;
-                float4* po = reinterpret_cast<float4*>(ps) + rr;
-#pragma unroll
-                for (int c = 0; c < D / 32; ++c) {
-                    uint32_t o[32];
-                    ptx::tmem_ld32(tO + c * 32, o);
-                    ptx::tmem_wait_ld();
-#pragma unroll
-                    for (int e = 0; e < 8; ++e)
-                        po[(size_t)(c * 8 + e) * 2 * kBlockM] =
-                            make_float4(__uint_as_float(o[4 * e]), __uint_as_float(o[4 * e + 1]),
-                                        __uint_as_float(o[4 * e + 2]), __uint_as_float(o[4 * e + 3]));
-                }
-                ps[C::kSlotML + rr] = m_used;
-                ps[C::kSlotML + 2 * kBlockM + rr] = l;
-                __threadfence();
-                __syncwarp();
-                if (lane == 0) ptx::mbar_arrive(&epi_written);
+                const int n_pieces = (int)(c2 - c1) + 1;
+                // The counter word holds the pieces finished (low 16 bits) and
+                // the partial results written (high 16 bits).
                 const uint32_t par = (uint32_t)(nsplit & 1);
                 ++nsplit;
                 if (warp == 4 && lane == 0) {
-                    // All 256 rows are written (and fenced): count this piece in.
-                    bool okw = ptx::mbar_wait_bounded(&epi_written, par, abort_p, p.wait_limit);
-                    int last = 0;
-                    if (okw) {
-                        unsigned int* cnt = p.counters + G.item_base + pc.item;
-                        const unsigned int old = atomicAdd(cnt, 1u);
-                        last = (old == (unsigned int)(c2 - c1));
-                        if (last) {
-                            atomicExch(cnt, 0u);
-                            __threadfence();
+                    int last = (fin_old & 0xffffu) == (unsigned int)(n_pieces - 1);
+                    // A merge handed to the helper warps waits there instead.
+                    if (last && !(helper_merges && n_pieces <= kMergeBatch)) {
+                        // Every other piece has finished its tiles; wait (bounded)
+                        // until their partial results are written and fenced.
+                        const long long w0 = clock64();
+                        while ((*(volatile unsigned int*)cnt >> 16) != (unsigned int)(n_pieces - 1)) {
+                            if (*abort_p || clock64() - w0 > p.wait_limit) {
+                                *abort_p = 1;
+                                atomicOr(p.status, kDevTimeout);
+                                break;
+                            }
                         }
+                        atomicExch(cnt, 0u);  // no piece updates it again in this launch
+                        __threadfence();
                     }
                     merge_flag = last;
                     ptx::mbar_arrive(&epi_decided);
                 }
                 ok = ptx::mbar_wait_bounded(&epi_decided, par, abort_p, p.wait_limit);
-                ok = __all_sync(0xffffffffu, ok);
+                ok = __all_sync(0xffffffffu, ok && !*abort_p);
                 if (!ok) break;
-                if (*(volatile int*)&merge_flag) {
-                    // ---- last piece: merge every piece of this item
+                const bool merger = *(volatile int*)&merge_flag != 0;
+                // The merge goes to the helper warps when whole items follow;
+                // otherwise the merger of an item of up to kMergeBatch pieces
+                // keeps its own piece in TMEM and merges here. Every other
+                // piece writes its partial result.
+                const bool to_helper = merger && helper_merges && n_pieces <= kMergeBatch;
+                const bool fast = merger && !helper_merges && n_pieces <= kMergeBatch;
+                if (!fast) {
+                    float* ps = p.partials + (size_t)slot * C::kSlotFloats;
+                    float4* po = reinterpret_cast<float4*>(ps) + rr;
+#pragma unroll
+                    for (int c = 0; c < D / 32; ++c) {
+                        uint32_t o[32];
+                        ptx::tmem_ld32(tO + c * 32, o);
+                        ptx::tmem_wait_ld();
+#pragma unroll
+                        for (int e = 0; e < 8; ++e)
+                            po[(size_t)(c * 8 + e) * 2 * kBlockM] =
+                                make_float4(__uint_as_float(o[4 * e]), __uint_as_float(o[4 * e + 1]),
+                                            __uint_as_float(o[4 * e + 2]), __uint_as_float(o[4 * e + 3]));
+                    }
+                    ps[C::kSlotML + rr] = m_used;
+                    ps[C::kSlotML + 2 * kBlockM + rr] = l;
+                    __threadfence();
+                    __syncwarp();
+                    if (lane == 0) ptx::mbar_arrive(&epi_written);
+                    const uint32_t pw = (uint32_t)(nwritten & 1);
+                    ++nwritten;
+                    if (warp == 4 && lane == 0 && (!merger || to_helper)) {
+                        // All 256 rows are written and fenced: count them in, or
+                        // hand the merge to the helper warps.
+                        bool okw = ptx::mbar_wait_bounded(&epi_written, pw, abort_p, p.wait_limit);
+                        if (okw && !merger) atomicAdd(cnt, 1u << 16);
+                        if (okw && to_helper) {
+                            okw = ptx::mbar_wait_bounded(&job_empty, (uint32_t)((njob & 1) ^ 1), abort_p,
+                                                         p.wait_limit);
+                            if (okw) {
+                                job.item_rel = pc.item_start - p.t_sk;
+                                job.c1 = c1;
+                                job.c2 = c2;
+                                job.cnt = cnt;
+                                job.q_row0 = pc.q_row0;
+                                job.q_end = G.q_end;
+                                job.b = pc.b;
+                                job.h = pc.h;
+                                job.stop = 0;
+                                ptx::mbar_arrive(&job_full);
+                            }
+                        }
+                        if (!okw) atomicOr(p.status, kDevTimeout);
+                    }
+                    if (to_helper) ++njob;
+                }
+                if (fast) {
+                    // ---- last piece: merge every piece of this item, in piece
+                    // order whichever CTA merges (the same bits on every run).
+                    // Its own piece is still in TMEM (O) and registers
+                    // (m_used, l); the others come from L2, and each batch of
+                    // loads (m and l of every piece, then one 32-column chunk
+                    // of two other pieces) is issued before its first use: a
+                    // round trip to L2 costs about a microsecond, so the merge
+                    // takes a few round trips instead of one per piece and
+                    // chunk. Other piece k is piece k + (k >= own) in order.
+                    const int own = (int)((long long)blockIdx.x - c1);
+                    const int n_oth = n_pieces - 1;
+                    int off[kMergeBatch];  // even length: the pairs below never index past it
+                    float mv[kMergeBatch], lv[kMergeBatch];
+#pragma unroll
+                    for (int k = 0; k < kMergeBatch; ++k) {
+                        off[k] = 0;
+                        mv[k] = -INFINITY;
+                        lv[k] = 0.f;
+                        if (k < n_oth) {
+                            off[k] = slot_of(c1 + k + (k >= own ? 1 : 0), c1, pc.item_start - p.t_sk, Tsk,
+                                             ncta) * C::kSlotFloats;
+                            mv[k] = __ldcg(p.partials + off[k] + C::kSlotML + rr);
+                            lv[k] = __ldcg(p.partials + off[k] + C::kSlotML + 2 * kBlockM + rr);
+                        }
+                    }
+                    float M = m_used;
+#pragma unroll
+                    for (int k = 0; k < kMergeBatch; ++k) M = fmaxf(M, mv[k]);
+                    const float w_own = ex2(m_used - M);
+                    float L = 0.f;
+#pragma unroll
+                    for (int k = 0; k < kMergeBatch; ++k) {
+                        if (k == own) L = fmaf(w_own, l, L);
+                        mv[k] = k < n_oth ? ex2(mv[k] - M) : 0.f;  // other piece k's weight
+                        if (k < n_oth) L = fmaf(mv[k], lv[k], L);
+                    }
+                    const float inv = 1.0f / L;
+                    if (store && p.lse)
+                        p.lse[((size_t)pc.b * p.H + pc.h) * p.N + qrow] =
+                            (M + log2f(L)) * 0.6931471805599453f;
+#pragma unroll 1
+                    for (int ch = 0; ch < D / 32; ++ch) {
+                        uint32_t o[32];
+                        ptx::tmem_ld32(tO + ch * 32, o);
+                        ptx::tmem_wait_ld();
+                        float acc[32];
+#pragma unroll
+                        for (int e = 0; e < 32; ++e) acc[e] = 0.f;
+#pragma unroll
+                        for (int k = 0; k < kMergeBatch; k += 2) {
+                            if (k >= n_oth) break;
+                            const bool two = k + 1 < n_oth;
+                            const float4* sa = reinterpret_cast<const float4*>(p.partials + off[k]) + rr;
+                            const float4* sb = reinterpret_cast<const float4*>(p.partials + off[k + 1]) + rr;
+                            float4 va[8], vb[8];
+#pragma unroll
+                            for (int e = 0; e < 8; ++e) {
+                                const size_t q = (size_t)(ch * 8 + e) * 2 * kBlockM;
+                                va[e] = __ldcg(sa + q);
+                                vb[e] = two ? __ldcg(sb + q) : make_float4(0.f, 0.f, 0.f, 0.f);
+                            }
+                            const float wa = mv[k], wb = mv[k + 1];
+#pragma unroll
+                            for (int e = 0; e < 8; ++e) {
+                                const float a4[4] = {va[e].x, va[e].y, va[e].z, va[e].w};
+                                const float b4[4] = {vb[e].x, vb[e].y, vb[e].z, vb[e].w};
+#pragma unroll
+                                for (int x = 0; x < 4; ++x) {
+                                    float v = acc[4 * e + x];
+                                    const float ov = __uint_as_float(o[4 * e + x]);
+                                    if (own == k) v = fmaf(w_own, ov, v);
+                                    v = fmaf(wa, a4[x], v);
+                                    if (two && own == k + 1) v = fmaf(w_own, ov, v);
+                                    if (two) v = fmaf(wb, b4[x], v);
+                                    acc[4 * e + x] = v;
+                                }
+                            }
+                        }
+                        if (own == n_oth) {  // the own piece is the item's last one
+#pragma unroll
+                            for (int e = 0; e < 32; ++e) acc[e] = fmaf(w_own, __uint_as_float(o[e]), acc[e]);
+                        }
+                        if (store) {
+                            uint4* d4 = reinterpret_cast<uint4*>(dst + ch * 32);
+#pragma unroll
+                            for (int e = 0; e < 4; ++e)
+                                d4[e] = make_uint4(ptx::pack_bf16(acc[8 * e] * inv, acc[8 * e + 1] * inv),
+                                                   ptx::pack_bf16(acc[8 * e + 2] * inv, acc[8 * e + 3] * inv),
+                                                   ptx::pack_bf16(acc[8 * e + 4] * inv, acc[8 * e + 5] * inv),
+                                                   ptx::pack_bf16(acc[8 * e + 6] * inv, acc[8 * e + 7] * inv));
+                        }
+                    }
+                } else if (merger && !to_helper) {
+                    // ---- last piece of an item cut into more pieces than one
+                    // batch holds: merge every piece from its partial slot
                     const int rr = t * kBlockM + r;
                     float M = -INFINITY;
                     for (long long c = c1; c <= c2; ++c) {
@@ -688,6 +969,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         }
         if (!ok && lane == 0) atomicOr(p.status, kDevTimeout);
+        if (helper_merges && warp == 4 && lane == 0) {
+            // No more merges: let the helper warps finish.
+            if (ptx::mbar_wait_bounded(&job_empty, (uint32_t)((njob & 1) ^ 1), abort_p, p.wait_limit)) {
+                job.stop = 1;
+                ptx::mbar_arrive(&job_full);
+            }
+        }
     }
 
     ptx::tc_fence_before();
@@ -887,8 +1175,8 @@ msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st) {
     // CTA, each CTA first takes whole items of it (no partial results), and
     // only the rest of the sequence is split evenly (stream-K).
     tp.dp_rounds = 0;
-    tp.dp_stride = tp.g[0].n_virt;
     if (tp.n_groups > 0) tp.dp_rounds = (int)(tp.g[0].n_items / ncta);
+    tp.dp_stride = tp.g[0].n_virt;
     tp.t_sk = (long long)tp.dp_rounds * ncta * tp.dp_stride;
 
     if (P.D == 128) {
