@@ -90,6 +90,7 @@ struct TcParams {
     TcGroup g[MSF_MAX_GROUPS];  // longest context first
     __nv_bfloat16* out;
     long long out_bstride;  // elements
+    int out_v8;             // output rows 32-byte aligned: 32-byte stores
     unsigned int* status;
     unsigned int* counters;  // per item
     float* partials;         // 2 slots per CTA
@@ -725,7 +726,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int e = 0; e < 16; ++e)
                         pk[e] = ptx::pack_bf16(__uint_as_float(o[2 * e]) * inv,
                                                __uint_as_float(o[2 * e + 1]) * inv);
-                    if (store) {
+                    if (store && p.out_v8) {
+                        ptx::st_global_v8(dst + c * 32, pk);
+                        ptx::st_global_v8(dst + c * 32 + 16, pk + 8);
+                    } else if (store) {
                         uint4* d4 = reinterpret_cast<uint4*>(dst + c * 32);
 #pragma unroll
                         for (int e = 0; e < 4; ++e)
@@ -1091,6 +1095,9 @@ msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st) {
     tp.scale_log2 = a.scale_log2;
     tp.out = (__nv_bfloat16*)a.out;
     tp.out_bstride = (long long)P.N * P.H * P.D;
+    // Rows of one head are D * 2 bytes (a multiple of 32): with a 32-byte
+    // aligned output the epilogue stores whole 32-byte sectors.
+    tp.out_v8 = ((uintptr_t)a.out % 32 == 0 && (tp.out_bstride * 2) % 32 == 0) ? 1 : 0;
     tp.status = a.status;
     tp.counters = attn_counters(P);
     tp.partials = attn_partials(P);

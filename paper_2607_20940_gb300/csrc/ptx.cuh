@@ -405,6 +405,14 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
 
 // Pack two fp32 into bf16x2 with round-to-nearest-even: `lo` lands in the
 // low 16 bits (the lower-indexed element in memory order).
+// 32 bytes from eight registers in one store (a whole L2 sector per thread);
+// the address must be 32-byte aligned.
+__device__ __forceinline__ void st_global_v8(void* ptr, const uint32_t* v) {
+    asm volatile("st.global.v8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"l"(ptr), "r"(v[0]), "r"(v[1]),
+                 "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
+                 : "memory");
+}
+
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
     uint32_t r;
     asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
