@@ -4,24 +4,30 @@
 // Work: an item is one 256-row query block (two 128-row tiles Q0, Q1) of one
 // (stream, head, query group); it walks that group's context segments (sink,
 // history or pyramid part, window suffix) in 128-row K/V tiles. All items'
-// tiles form one sequence (longest contexts first) that a persistent grid
-// splits into equal contiguous ranges, one per CTA (stream-K). A piece is the
-// part of one item inside one CTA's range. A piece that is a whole item
-// writes its normalised output; a piece of a split item writes its
-// unnormalised output with the running max and sum to a partial slot, and the
-// piece that finishes last merges all of them (per-item counter in the
-// workspace, reset by the merger).
+// tiles form one sequence (longest contexts first). While the longest group
+// has at least one item per CTA, a persistent grid takes its items whole in
+// data-parallel rounds; the rest of the sequence is split into equal
+// contiguous ranges, one per CTA (stream-K), which each CTA runs before its
+// whole items. A piece is the part of one item inside one CTA's range. A
+// piece that is a whole item writes its normalised output; a piece of a
+// split item writes its unnormalised output with the running max and sum to
+// a partial slot, and the piece that counts itself finished last (per-item
+// counter word in the workspace: pieces finished | partials written, reset
+// by the merge) has all of them merged in piece order.
 //
 // Roles inside a CTA (384 threads):
 //   warp 0      TMA producer: Q0/Q1 per piece, then K_j and V_j into a
 //               2-deep K ring and a 3-deep V ring, gated by one release per tile
-//   warp 1      MMA issuer (one thread): S_t = Q_t K_j^T into TMEM (SS form),
-//               O_t += P_t V_j with P_t read from TMEM (TS form, V MN-major)
+//   warp 1      MMA issuer (one elected lane of the converged warp):
+//               S_t = Q_t K_j^T into TMEM (SS form), O_t += P_t V_j with P_t
+//               read from TMEM (TS form, V MN-major)
 //   warp 2      TMEM allocation (all 512 columns)
+//   warps 2-3   merge helpers: combine the pieces of the split items this CTA
+//               finished last while the softmax warps run the whole items
 //   warps 4-7   softmax of tile 0, warps 8-11 softmax of tile 1: one thread
-//               per query row; tcgen05.ld of S, row max, exp2, row sum, P as
-//               bf16 written over S's first 64 columns, lazy rescale of O
-//               (only when the running max grows by more than 2^8)
+//               per query row; tcgen05.ld of S, exp2 against a running max
+//               that may lag, row sum, P as bf16 written over S's first 64
+//               columns, rescale of O only when a tile's sum passes 2^32
 // TMEM columns: S0 [0,128) S1 [128,256) O0 [256,384) O1 [384,512).
 // The MMA thread issues S_t(j+1) right after PV_t(j), so the commit that
 // signals S_t(j+1) also covers PV_t(j): a softmax warp that sees S ready may
