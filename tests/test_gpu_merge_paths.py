@@ -53,3 +53,27 @@ def test_split_merge_paths(w, heads):
     ref = oracle_mssa(x, w, heads=heads)
     mx, mean = err_stats(outs[0], ref, heads)
     assert mx <= 2e-2 and mean <= 2e-3, (mx, mean)
+
+
+def test_output_16_byte_aligned():
+    """An output that is 16-byte but not 32-byte aligned (the ABI asks for 16)
+    takes the 16-byte store path of the whole-block epilogue (the 480p layer
+    has whole blocks); the result is the same as with an aligned output, bit
+    for bit, and nothing is written outside the output."""
+    w = synth.LAYER_480P
+    x = synth.attention_inputs(w, BF16)
+    plan = make_plan(w, BF16)
+    dx = device_inputs(x, w.history_capacity)
+    bind(plan, dx)
+    plan.kv_resample(dx["k_win"], dx["v_win"])
+    aligned = torch.empty_like(dx["q"])
+    plan.mssa_forward(dx["q"], dx["k_win"], dx["v_win"], aligned)
+    n = dx["q"].numel()
+    buf = torch.full((n + 16,), float("nan"), dtype=BF16, device="cuda")
+    assert buf.data_ptr() % 32 == 0
+    shifted = buf[8:8 + n].view(dx["q"].shape)  # 16 bytes past a 32-byte boundary
+    plan.mssa_forward(dx["q"], dx["k_win"], dx["v_win"], shifted)
+    torch.cuda.synchronize()
+    assert plan.device_status() == 0
+    assert torch.equal(aligned, shifted)
+    assert torch.isnan(buf[:8]).all() and torch.isnan(buf[8 + n:]).all()
