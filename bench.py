@@ -181,14 +181,13 @@ def run_reference(args, w):
 
 def oracle_other_configs():
     """The oracle (fp64 numpy, as it stands) on the host cores for the other
-    workloads of the family, each on a bounded sample: the tiny window whole,
-    the three-scale window on 2 of its 16 heads, the 30-layer pass on layers
-    0, 15 and 29 (each: patchify + tier embedding of the window, MSSA on 2 of
-    12 heads, de-embedding + unpatchify of the head), and the B=4 rollout on
-    steps 0, 1, 2, 60 and 119 of stream 0 (2 of 12 heads; the history holds
-    min(2 + step, 4) frames). Sampled heads, layers and steps are scaled up
-    to the whole workload and marked "extrapolated" (the oracle's time is
-    linear in heads, layers, streams and steps)."""
+    workloads of the family: the tiny and the three-scale windows whole, the
+    30-layer pass on layers 0, 15 and 29 (each: patchify + tier embedding of
+    the window, MSSA on 2 of 12 heads, de-embedding + unpatchify of the head),
+    and the B=4 rollout on steps 0, 1, 2, 60 and 119 of stream 0 (2 of 12
+    heads; the history holds min(2 + step, 4) frames). Sampled heads, layers
+    and steps are scaled up to the whole workload and marked "extrapolated"
+    (the oracle's time is linear in heads, layers, streams and steps)."""
     import dataclasses
 
     import torch
@@ -217,13 +216,12 @@ def oracle_other_configs():
     fl = flops(w, w.history_frames, w.heads)
     res["tiny"] = {"workload": w.name, "seconds": dt, "gflop": fl / 1e9, "tflops": fl / dt / 1e12,
                    "sample": "whole call (fp32 inputs)"}
-    # three-scale 48x80 window: 2 of 16 heads
+    # three-scale 48x80 window: the whole call (all 16 heads)
     w = synth.THREE_SCALE
-    hs = [0, 8]
-    dt = attn(w, synth.attention_inputs(w, torch.bfloat16), hs) * w.heads / len(hs)
+    dt = attn(w, synth.attention_inputs(w, torch.bfloat16), None)
     fl = flops(w, w.history_frames, w.heads)
     res["three_scale"] = {"workload": w.name, "seconds": dt, "gflop": fl / 1e9, "tflops": fl / dt / 1e12,
-                          "sample": "2 of 16 heads, extrapolated to 16"}
+                          "sample": "whole call (all 16 heads)"}
     # 30-layer window pass: layers 0, 15, 29
     w = synth.PASS_480P
     hs = [0, 6]
