@@ -10,8 +10,9 @@ schedule (152 persistent CTAs on a GB300, fewer when the sequence is short):
 * one head over a 3072-row context (2 blocks of 24 K/V tiles, ~58 CTAs):
   blocks cut into more than 8 pieces -> the merger reads every piece's
   partial result from its slot;
-* the 480p layer (156 fine-group blocks >= 152 CTAs): one whole round, the
-  rest split -> the merge runs on the helper warps beside the whole blocks.
+* the 480p layer (156 fine-group blocks >= 152 CTAs), and a head_dim-64
+  window with 160: one whole round, the rest split -> the merge runs on the
+  helper warps beside the whole blocks.
 
 Each case is checked against the fp64 oracle and for run-to-run
 reproducibility: pieces are combined in a fixed order whichever CTA merges,
@@ -29,13 +30,16 @@ pytestmark = pytest.mark.gpu
 # One head, two fine states of 16x16 tokens, a 2048-token sink and two history
 # frames: query blocks of 256 rows over a 3072-row context (24 K/V tiles).
 LONG_CTX = synth.Workload("long_ctx_h1_t2_16x16_sink2048", 2, (1, 1), 16, 16, 1, 128, 2048, 2, 2, 1, 11)
+# head_dim 64 with whole rounds: 16 heads x 10 fine-group blocks = 160 >= 152.
+HELPER_D64 = synth.Workload("helper_d64_t3_32x40_h16", 3, (1, 1, 2), 32, 40, 16, 64, 1280, 1, 1, 1, 12)
 
 
 @pytest.mark.parametrize("w,heads", [
     (synth.TINY, None),
     (LONG_CTX, None),
     (synth.LAYER_480P, [0, 7]),
-], ids=["in_place", "from_slots", "helper_warps"])
+    (HELPER_D64, [0, 15]),
+], ids=["in_place", "from_slots", "helper_warps", "helper_warps_d64"])
 def test_split_merge_paths(w, heads):
     x = synth.attention_inputs(w, BF16)
     plan = make_plan(w, BF16)
