@@ -13,7 +13,9 @@ for both of its inputs.
 `value` is the MSSA FLOPs the schedule requires (4*D*H*sum_g Nq_g*Nkv_g =
 202.79 GFLOP) divided by the device time of the whole step, in TFLOP/s.
 Inputs are resident in HBM; the L2 is flushed (a 256 MiB write) between
-timed steps, outside the timed events.
+timed steps, outside the timed events. The CPU-baseline leg (rank 0, one GPU) times
+the oracle and also compares the attention kernel's output for the same
+inputs with the oracle's, element by element (`parity`).
 
 Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
 Under torchrun every rank runs its own stream of windows (weak scaling);
@@ -263,6 +265,32 @@ def oracle_other_configs():
                         "sample": "steps 0, 1, 2, 60, 119 of stream 0 (2 of 12 heads), extrapolated "
                                   "to 4 streams x 12 heads x 120 steps"}
     return res
+
+
+def _parity_check(msf, w, x, ref):
+    """The attention kernel's output for the step's inputs against the
+    oracle's output that the CPU baseline computed for the same inputs: max and
+    mean |err| over every element of the 480p layer. The plan here has no
+    fused history update, so its history is the inputs' initial one."""
+    import numpy as np
+    import torch
+    dev = torch.device("cuda", torch.cuda.current_device())
+    plan = msf.Plan(msf.make_desc(w.scales, w.grid_h, w.grid_w, w.heads, w.head_dim, w.sink_tokens,
+                                  w.history_frames, w.history_capacity, batch=w.batch))
+    d = {k: v.to(dev) for k, v in x.items()}
+    ws = plan.workspace(dev)
+    plan.bind(ws, d["k_sink"], d["v_sink"], d["k_hist"], d["v_hist"])
+    out = torch.empty_like(d["q"])
+    plan.kv_resample(d["k_win"], d["v_win"])
+    plan.mssa_forward(d["q"], d["k_win"], d["v_win"], out)
+    torch.cuda.synchronize()
+    status_ok = plan.device_status() == msf.MSF_OK
+    plan.close()
+    err = np.abs(out.double().cpu().numpy() - ref)
+    mx, mean = float(err.max()), float(err.mean())
+    return {"max_abs_err": mx, "mean_abs_err": mean, "elements": int(err.size),
+            "tolerance": {"max": 2e-2, "mean": 2e-3},
+            "pass": bool(status_ok and mx <= 2e-2 and mean <= 2e-3)}
 
 
 def _traffic_from_profile(kernel_src: str):
@@ -796,13 +824,15 @@ def main():
 
     # ------------------------------------------------------- CPU baseline
     cpu = None
+    parity = None
     if world == 1 and not args.no_cpu_baseline:
         t0 = time.perf_counter()
-        _oracle_step(w, x, mi)
+        ref = _oracle_step(w, x, mi)
         dt = time.perf_counter() - t0
         cpu = {"value": flops / dt / 1e12, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
                "sample": f"one full 480p step (all 12 heads) in fp64 numpy, {dt:.1f} s",
                "other_configs": oracle_other_configs()}
+        parity = _parity_check(msf, w, x, ref)
 
     peaks, peak_src = _peaks()
     attn_avg_ms = statistics.mean(attn_ms)
@@ -845,6 +875,7 @@ def main():
                      "tflops": fine_flops / (fine_attn_ms * 1e-3) / 1e12,
                      "speedup_vs_all_fine": fine_attn_ms / attn_avg_ms},
         "cpu_baseline": cpu,
+        "parity": parity,
         "other_configs": others,
         "e2e": {"value": world * flops * args.steps / (e2e_ms * 1e-3) / 1e12, "unit": UNIT,
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
