@@ -78,15 +78,14 @@ __device__ __forceinline__ uint32_t swz_offset(int row, int k) {
 // ----------------------------------------------------------------- embedding
 
 // Features [64 kc, 64 kc + 64) of one token row in (c, dy, dx) order: 64 / P
-// runs of P pixels, each run one row segment of one channel. All loads of the
-// chunk are issued before the first store so that they overlap.
+// runs of P pixels, each run one row segment of one channel. The loads and the
+// stores are apart, so a row's next chunk can be in flight while the current
+// one waits for its stage.
 template <int P, typename V>
-__device__ __forceinline__ void gather_chunk(unsigned char* dst, const __nv_bfloat16* base, size_t plane,
-                                             int Wl, int r, int kc, bool valid) {
-    constexpr int kRuns = 64 / P;
-    V v[kRuns];
+__device__ __forceinline__ void load_chunk(V (&v)[64 / P], const __nv_bfloat16* base, size_t plane, int Wl,
+                                           int kc, bool valid) {
 #pragma unroll
-    for (int g = 0; g < kRuns; ++g) {
+    for (int g = 0; g < 64 / P; ++g) {
         const int f0 = kc * 64 + g * P;
         const int c = f0 / (P * P), dy = (f0 % (P * P)) / P;
         if (valid)
@@ -94,8 +93,35 @@ __device__ __forceinline__ void gather_chunk(unsigned char* dst, const __nv_bflo
         else
             memset(&v[g], 0, sizeof(V));
     }
+}
+template <int P, typename V>
+__device__ __forceinline__ void store_chunk(unsigned char* dst, const V (&v)[64 / P], int r) {
 #pragma unroll
-    for (int g = 0; g < kRuns; ++g) *reinterpret_cast<V*>(dst + swz_offset(r, g * P)) = v[g];
+    for (int g = 0; g < 64 / P; ++g) *reinterpret_cast<V*>(dst + swz_offset(r, g * P)) = v[g];
+}
+
+// Every K chunk of one token row into the A ring, each chunk's loads issued
+// before the wait for the previous chunk's stage, so that the L2 round trips
+// of consecutive chunks overlap. Returns false if a wait gave up.
+template <int P, typename V>
+__device__ __forceinline__ bool gather_row(unsigned char* sA, uint64_t* a_full, uint64_t* a_empty,
+                                           const __nv_bfloat16* base, size_t plane, int Wl, int r, int nk,
+                                           bool valid, volatile int* abort_p) {
+    V cur[64 / P], nxt[64 / P];
+    load_chunk<P, V>(cur, base, plane, Wl, 0, valid);
+    for (int kc = 0; kc < nk; ++kc) {
+        if (kc + 1 < nk) load_chunk<P, V>(nxt, base, plane, Wl, kc + 1, valid);
+        const int st = kc % kEmbedStages;
+        const uint32_t ph = (uint32_t)((kc / kEmbedStages) & 1);
+        const bool ok = __all_sync(0xffffffffu, ptx::mbar_wait_bounded(&a_empty[st], ph ^ 1u, abort_p, kWaitLimit));
+        if (!ok) return false;
+        store_chunk<P, V>(sA + st * kChunkA, cur, r);
+        ptx::fence_proxy_async_smem();  // the tensor core reads through the async proxy
+        ptx::mbar_arrive(&a_full[st]);
+#pragma unroll
+        for (int g = 0; g < 64 / P; ++g) cur[g] = nxt[g];
+    }
+    return true;
 }
 
 struct EmbedRun {
@@ -237,20 +263,20 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
         const size_t plane = (size_t)p.Hl * p.Wl;
         bool ok = true;
-        for (int kc = 0; kc < nk; ++kc) {
+        if (P == 2) {
+            ok = gather_row<2, uint32_t>(sA, a_full, a_empty, base, plane, p.Wl, r, nk, valid, abort_p);
+        } else if (P == 4) {
+            ok = gather_row<4, uint2>(sA, a_full, a_empty, base, plane, p.Wl, r, nk, valid, abort_p);
+        } else if (P == 8) {
+            ok = gather_row<8, uint4>(sA, a_full, a_empty, base, plane, p.Wl, r, nk, valid, abort_p);
+        } else for (int kc = 0; kc < nk; ++kc) {
             const int st = kc % kEmbedStages;
             const uint32_t ph = (uint32_t)((kc / kEmbedStages) & 1);
             ok = ptx::mbar_wait_bounded(&a_empty[st], ph ^ 1u, abort_p, kWaitLimit);
             ok = __all_sync(0xffffffffu, ok);
             if (!ok) break;
             unsigned char* dst = sA + st * kChunkA;
-            if (P == 2) {
-                gather_chunk<2, uint32_t>(dst, base, plane, p.Wl, r, kc, valid);
-            } else if (P == 4) {
-                gather_chunk<4, uint2>(dst, base, plane, p.Wl, r, kc, valid);
-            } else if (P == 8) {
-                gather_chunk<8, uint4>(dst, base, plane, p.Wl, r, kc, valid);
-            } else {
+            {
                 for (int g = 0; g < 64 / P; ++g) {
                     const int f0 = kc * 64 + g * P;
                     const int c = f0 / (P * P), dy = (f0 % (P * P)) / P;
