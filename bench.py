@@ -526,12 +526,25 @@ def other_configs(msf, synth, dev, flush, peaks, rank):
                           dtype=torch.bfloat16, device=dev)
     plan.kv_resample(t["k_win"], t["v_win"], msf.MSF_RESAMPLE_FULL)
 
+    side = torch.cuda.Stream(device=dev)
+
     def one_pass():
+        # Each layer as in the single step: the K/V pyramid on a second stream
+        # beside the embedding (forked after the previous layer's launches, so
+        # it never overwrites a pyramid that attention still reads), attention
+        # after both, then the de-embedding.
+        cur = torch.cuda.current_stream()
         for _ in range(wp.layers):
-            plan.patchify(lat, w_tier, tok)
-            plan.kv_resample(t["k_win"], t["v_win"], msf.MSF_RESAMPLE_WINDOW_ONLY)
-            plan.mssa_forward(t["q"], t["k_win"], t["v_win"], t["out"])
-            plan.unpatchify(0, t["out"].view(wp.batch, N, E), w_out, lat_out)
+            fork = torch.cuda.Event()
+            fork.record(cur)
+            side.wait_event(fork)
+            plan.kv_resample(t["k_win"], t["v_win"], msf.MSF_RESAMPLE_WINDOW_ONLY, stream=side)
+            pooled = torch.cuda.Event()
+            pooled.record(side)
+            plan.patchify(lat, w_tier, tok, stream=cur)
+            cur.wait_event(pooled)
+            plan.mssa_forward(t["q"], t["k_win"], t["v_win"], t["out"], stream=cur)
+            plan.unpatchify(0, t["out"].view(wp.batch, N, E), w_out, lat_out, stream=cur)
 
     pass_ms = _timed(one_pass, flush, reps=3, warm=1, sleep=False)
     fl = plan.info.attention_flops * wp.layers
