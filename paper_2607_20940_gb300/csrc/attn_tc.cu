@@ -70,6 +70,9 @@ constexpr long long kWaitLimit = 2000000000LL;  // ~1 s of SM clock
 constexpr int kItemLeadTiles = 5;
 // Pieces of one item that the merging CTA combines from one batch of loads.
 constexpr int kMergeBatch = 8;
+// Bound of the helper warps' wait for a merge job, in units of the per-tile
+// wait bound (~1 s of SM clock): a CTA's whole items take far less.
+constexpr long long kHelperWaitFactor = 64;
 
 struct TcSeg {
     int map;
@@ -479,7 +482,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         // about a microsecond.
         const int ht = (warp - 2) * 32 + lane;
         for (int jn = 0;; ++jn) {
-            bool okj = ptx::mbar_wait_bounded(&job_full, (uint32_t)(jn & 1), abort_p, p.wait_limit);
+            // The next job may come only after this CTA's whole items (or its
+            // stop at the end), so this wait's bound is a multiple of the
+            // per-tile one; the softmax warps' own waits are bounded and raise
+            // the abort flag, which ends it at once.
+            bool okj = ptx::mbar_wait_bounded(&job_full, (uint32_t)(jn & 1), abort_p,
+                                              kHelperWaitFactor * p.wait_limit);
             okj = __all_sync(0xffffffffu, okj);
             if (!okj) break;
             const volatile MergeJob& vj = job;
