@@ -111,6 +111,54 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
+def _host_info() -> dict:
+    """The host the oracle runs on: CPU model, logical cores, and the thread
+    count of the BLAS that numpy's fp64 matmuls use (read from the loaded
+    OpenBLAS itself), with OMP_NUM_THREADS / OPENBLAS_NUM_THREADS as set."""
+    import ctypes
+    import re
+
+    import numpy  # noqa: F401  (loads its BLAS)
+    model = None
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().lower().startswith("model name"):
+                model = line.split(":", 1)[1].strip()
+                break
+    except (OSError, subprocess.SubprocessError):
+        pass
+    if model is None:
+        try:
+            with open("/proc/cpuinfo") as f:
+                for line in f:
+                    if line.lower().startswith("model name"):
+                        model = line.split(":", 1)[1].strip()
+                        break
+        except OSError:
+            pass
+    blas, threads = None, None
+    try:
+        with open("/proc/self/maps") as f:
+            libs = sorted(set(re.findall(r"/\S*openblas\S*\.so\S*", f.read())))
+        for path in libs:
+            lib = ctypes.CDLL(path)
+            for sym in ("scipy_openblas_get_num_threads64_", "openblas_get_num_threads64_",
+                        "scipy_openblas_get_num_threads", "openblas_get_num_threads"):
+                fn = getattr(lib, sym, None)
+                if fn is not None:
+                    fn.restype = ctypes.c_int
+                    blas, threads = os.path.basename(path), int(fn())
+                    break
+            if threads is not None:
+                break
+    except OSError:
+        pass
+    return {"cpu_model": model, "logical_cores": os.cpu_count(), "blas": blas,
+            "blas_threads": threads, "OMP_NUM_THREADS": os.environ.get("OMP_NUM_THREADS"),
+            "OPENBLAS_NUM_THREADS": os.environ.get("OPENBLAS_NUM_THREADS")}
+
+
 def max_over_ranks(value: float, device) -> float:
     """The largest per-rank time (the job ends when the slowest rank ends)."""
     import torch
@@ -167,7 +215,8 @@ def run_reference(args, w):
         times.append(time.perf_counter() - t0)
     tot = sum(times)
     value = fl * args.steps / tot / 1e12
-    cores = os.cpu_count()
+    host = _host_info()
+    cores = host["blas_threads"] or os.cpu_count()
     sample = f"3 of 12 heads of the 480p layer per step (oracle fp64, numpy), {fl/1e9:.2f} GFLOP"
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
@@ -175,7 +224,7 @@ def run_reference(args, w):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": {"workload": w.name, "kind": "oracle sample"},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
-                         "sample": sample},
+                         "sample": sample, "host": host},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line))
@@ -842,9 +891,11 @@ def main():
         t0 = time.perf_counter()
         ref = _oracle_step(w, x, mi)
         dt = time.perf_counter() - t0
-        cpu = {"value": flops / dt / 1e12, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+        host = _host_info()
+        cpu = {"value": flops / dt / 1e12, "unit": UNIT,
+               "cores": host["blas_threads"] or os.cpu_count(), "kind": "oracle",
                "sample": f"one full 480p step (all 12 heads) in fp64 numpy, {dt:.1f} s",
-               "other_configs": oracle_other_configs()}
+               "host": host, "other_configs": oracle_other_configs()}
         parity = _parity_check(msf, w, x, ref)
 
     peaks, peak_src = _peaks()

@@ -136,6 +136,10 @@ typedef struct msf_plan_info {
                                          Nq * (6*D*Nkv + 4*D*Nkv_window) * H * B (S, dP and
                                          dQ over the whole context; dK and dV over the rows
                                          that come from the window) */
+    uint64_t attention_counter_offset; /* byte offset, inside the workspace, of the merge
+                                          counters of the tensor-core attention (one 32-bit
+                                          word per 256-row query block; zero between launches) */
+    uint64_t attention_counter_bytes;  /* their size (0 for fp32 plans) */
 } msf_plan_info;
 
 typedef struct msf_plan* msf_plan_t;
@@ -337,14 +341,30 @@ uint64_t msf_kernel_launches(void);
  * process exits; a problem needs B * C*Hl*Wl * 2 bytes (rounded up to 256)
  * plus 256 bytes of it, and larger ones are rejected with
  * MSF_ERR_UNSUPPORTED. The first call on each device looks up that array's
- * device address (cudaGetSymbolAddress, with that device current); make that
- * first call before any stream capture. It calls no cudaMalloc/cudaFree. Every
- * call shares the one array and overwrites it, so calls that overlap on the
- * GPU (different streams, or threads without ordering) race: serialise them.
+ * device address (cudaGetSymbolAddress, with that device current) and zeroes
+ * its status word (a synchronous cudaMemset); make that first call before any
+ * stream capture. It calls no cudaMalloc/cudaFree. Every call shares the one
+ * array and overwrites it, so calls that overlap on the GPU (different
+ * streams, or threads without ordering) race: serialise them. A device-side
+ * timeout of its GEMM is recorded in the array's own status word, which
+ * msf_noalloc_device_status reads (msf_plan_device_status does not see it).
  * Errors: INVALID_ARG, UNSUPPORTED (fp32 plan, no embedding, shape too
- * large), CUDA. */
+ * large, or a shape the tensor-core GEMM does not take: E a multiple of 64,
+ * C*P^2 a multiple of 8), CUDA. */
 msf_status msf_unpatchify_noalloc(msf_plan_t plan, int32_t position, const void* tokens,
                                   const void* w_out, void* latent_out, void* stream);
+
+/* Synchronise `stream`, then read and clear the status word of
+ * msf_unpatchify_noalloc's fixed array on the current device. Returns
+ * MSF_ERR_TIMEOUT if one of its kernels gave up on a bounded wait since the
+ * last read, MSF_OK otherwise. Errors: CUDA. */
+msf_status msf_noalloc_device_status(void* stream);
+
+/* Failure-path self test of that status word (no counterpart in the paper):
+ * the same bounded-wait kernel as msf_selftest_wait_timeout, aimed at the
+ * fixed array's status word of the current device. Errors: INVALID_ARG
+ * (limit outside 1 .. 2^31), CUDA. */
+msf_status msf_noalloc_selftest_wait_timeout(int64_t limit_cycles, void* stream);
 
 /* Failure-path self test (no counterpart in the paper): launches one block
  * that waits on an mbarrier nothing ever arrives at, with the same bounded
@@ -358,7 +378,9 @@ msf_status msf_selftest_wait_timeout(msf_plan_t plan, int64_t limit_cycles, void
 
 /* Synchronise `stream`, read and clear the device status word. Returns
  * MSF_ERR_TIMEOUT if a kernel gave up on a bounded wait since the last
- * check, MSF_OK otherwise. */
+ * check, MSF_OK otherwise. After a timeout it also zeroes the attention's
+ * merge counters (a launch that gave up can leave them counted), so the next
+ * msf_mssa_forward starts from a clean state. */
 msf_status msf_plan_device_status(msf_plan_t plan, void* stream);
 
 #ifdef __cplusplus

@@ -3,6 +3,10 @@
 #include <cuda_runtime.h>
 #include <string.h>
 
+#include <mutex>
+#include <utility>
+#include <vector>
+
 #include "attn_bwd_tc.h"
 #include "attn_tc.h"
 #include "gemm_tc.h"
@@ -12,6 +16,26 @@
 #include "ptx.cuh"
 
 using msf::Plan;
+
+namespace msf {
+
+cudaError_t set_smem_attr(const void* fn, int bytes, int carveout) {
+    static std::mutex mu;
+    static std::vector<std::pair<const void*, int>> done;  // (kernel, device)
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lock(mu);
+    for (const auto& d : done)
+        if (d.first == fn && d.second == dev) return cudaSuccess;
+    e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess && carveout >= 0)
+        e = cudaFuncSetAttribute(fn, cudaFuncAttributePreferredSharedMemoryCarveout, carveout);
+    if (e == cudaSuccess) done.emplace_back(fn, dev);
+    return e;
+}
+
+}  // namespace msf
 
 namespace {
 
@@ -762,13 +786,20 @@ __global__ void wait_timeout_selftest_kernel(unsigned int* status, long long lim
 }
 }  // namespace
 
+namespace msf {
+cudaError_t launch_wait_timeout_selftest(unsigned int* status, long long limit_cycles, cudaStream_t st) {
+    note_launch();
+    wait_timeout_selftest_kernel<<<1, 32, 0, st>>>(status, limit_cycles);
+    return cudaGetLastError();
+}
+}  // namespace msf
+
 extern "C" msf_status msf_selftest_wait_timeout(msf_plan_t plan, int64_t limit_cycles, void* stream) {
     if (!plan || limit_cycles < 1 || limit_cycles > (int64_t(1) << 31)) return MSF_ERR_INVALID_ARG;
     const Plan& p = *plan;
     if (!p.bound) return MSF_ERR_STATE;
-    msf::note_launch();
-    wait_timeout_selftest_kernel<<<1, 32, 0, (cudaStream_t)stream>>>(msf::status_word(p), (long long)limit_cycles);
-    return cuda_status(cudaGetLastError());
+    return cuda_status(msf::launch_wait_timeout_selftest(msf::status_word(p), (long long)limit_cycles,
+                                                         (cudaStream_t)stream));
 }
 
 extern "C" msf_status msf_plan_device_status(msf_plan_t plan, void* stream) {
@@ -782,6 +813,13 @@ extern "C" msf_status msf_plan_device_status(msf_plan_t plan, void* stream) {
         e = cudaMemcpyAsync(&word, msf::status_word(p), sizeof(word), cudaMemcpyDeviceToHost, s);
     if (e == cudaSuccess) e = cudaMemsetAsync(msf::status_word(p), 0, sizeof(word), s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    // A launch that gave up may have left merge counters counted: the next
+    // launch's "last piece" test and its wait for the written partials would
+    // then fire early or never. Zero them before anything else runs.
+    if (e == cudaSuccess && word && msf::attn_counter_bytes(p) > 0) {
+        e = cudaMemsetAsync(msf::attn_counters(p), 0, msf::attn_counter_bytes(p), s);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    }
     if (e != cudaSuccess) return cuda_status(e);
     return word ? MSF_ERR_TIMEOUT : MSF_OK;
 }

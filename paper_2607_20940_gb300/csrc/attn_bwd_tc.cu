@@ -906,21 +906,14 @@ msf_status launch_bwd_tc(msf_plan_t plan, const BwdTcInput& in, cudaStream_t st)
     if (total == 0) return MSF_OK;
     const bool d128 = P.D == 128;
     const int smem = d128 ? QCfg<128>::kSmem : QCfg<64>::kSmem;
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(bwd_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             QCfg<128>::kSmem);
-        if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(bwd_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     QCfg<64>::kSmem);
-        if (e != cudaSuccess) {
-            set_cuda_error((int)e);
-            return MSF_ERR_CUDA;
-        }
-        attr_set = true;
+    cudaError_t e = d128 ? set_smem_attr((const void*)bwd_tc_kernel<128>, QCfg<128>::kSmem)
+                         : set_smem_attr((const void*)bwd_tc_kernel<64>, QCfg<64>::kSmem);
+    if (e != cudaSuccess) {
+        set_cuda_error((int)e);
+        return MSF_ERR_CUDA;
     }
-    cudaError_t e = d128 ? launch_pdl(bwd_tc_kernel<128>, dim3((unsigned)total), dim3(kThreads), smem, st, maps, tp)
-                         : launch_pdl(bwd_tc_kernel<64>, dim3((unsigned)total), dim3(kThreads), smem, st, maps, tp);
+    e = d128 ? launch_pdl(bwd_tc_kernel<128>, dim3((unsigned)total), dim3(kThreads), smem, st, maps, tp)
+             : launch_pdl(bwd_tc_kernel<64>, dim3((unsigned)total), dim3(kThreads), smem, st, maps, tp);
     if (e != cudaSuccess) {
         set_cuda_error((int)e);
         return MSF_ERR_CUDA;

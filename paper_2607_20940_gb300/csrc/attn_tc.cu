@@ -70,9 +70,11 @@ constexpr long long kWaitLimit = 2000000000LL;  // ~1 s of SM clock
 constexpr int kItemLeadTiles = 5;
 // Pieces of one item that the merging CTA combines from one batch of loads.
 constexpr int kMergeBatch = 8;
-// Bound of the helper warps' wait for a merge job, in units of the per-tile
-// wait bound (~1 s of SM clock): a CTA's whole items take far less.
-constexpr long long kHelperWaitFactor = 64;
+// Bound of the helper warps' wait for a merge job: the next job (or the stop)
+// comes after at most the CTA's remaining tiles, so the bound is the CTA's
+// tile count times ~0.5 ms of SM clock per tile (about 400 times what a
+// 128-row K/V step costs), and at least the per-wait bound.
+constexpr long long kHelperCyclesPerTile = 1LL << 20;
 
 struct TcSeg {
     int map;
@@ -481,13 +483,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         // 16-column chunk of two pieces), as each round trip to L2 costs
         // about a microsecond.
         const int ht = (warp - 2) * 32 + lane;
+        long long helper_limit = ((r1 - r0) + (long long)p.dp_rounds * p.dp_stride) * kHelperCyclesPerTile;
+        if (helper_limit < p.wait_limit) helper_limit = p.wait_limit;
         for (int jn = 0;; ++jn) {
             // The next job may come only after this CTA's whole items (or its
-            // stop at the end), so this wait's bound is a multiple of the
-            // per-tile one; the softmax warps' own waits are bounded and raise
-            // the abort flag, which ends it at once.
-            bool okj = ptx::mbar_wait_bounded(&job_full, (uint32_t)(jn & 1), abort_p,
-                                              kHelperWaitFactor * p.wait_limit);
+            // stop at the end), so this wait's bound scales with the CTA's
+            // tiles; the softmax warps' own waits are bounded and raise the
+            // abort flag, which ends it at once.
+            bool okj = ptx::mbar_wait_bounded(&job_full, (uint32_t)(jn & 1), abort_p, helper_limit);
             okj = __all_sync(0xffffffffu, okj);
             if (!okj) break;
             const volatile MergeJob& vj = job;
@@ -1051,7 +1054,7 @@ struct TcCache {
     const void* key_ptr[2 * kNumMaps + 1];
     int key_rows[2 * kNumMaps + 1];
     bool valid[2 * kNumMaps + 1];
-    bool attr_set[2];
+    bool attr_set[2];  // register count of the compiled kernel checked
     int num_sms;
 };
 
@@ -1210,13 +1213,12 @@ msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st) {
                 return MSF_ERR_CUDA;
             }
             if (fa.numRegs != kLaunchRegs) return MSF_ERR_UNSUPPORTED;
-            e = cudaFuncSetAttribute(mssa_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     Cfg<128>::kSmem);
-            if (e != cudaSuccess) {
-                set_cuda_error((int)e);
-                return MSF_ERR_CUDA;
-            }
             cache.attr_set[1] = true;
+        }
+        e = set_smem_attr((const void*)mssa_tc_kernel<128>, Cfg<128>::kSmem);
+        if (e != cudaSuccess) {
+            set_cuda_error((int)e);
+            return MSF_ERR_CUDA;
         }
         e = launch_pdl(mssa_tc_kernel<128>, dim3((unsigned)ncta), dim3(kThreads), Cfg<128>::kSmem, st,
                        cache.maps, tp);
@@ -1229,13 +1231,12 @@ msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st) {
                 return MSF_ERR_CUDA;
             }
             if (fa.numRegs != kLaunchRegs) return MSF_ERR_UNSUPPORTED;
-            e = cudaFuncSetAttribute(mssa_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     Cfg<64>::kSmem);
-            if (e != cudaSuccess) {
-                set_cuda_error((int)e);
-                return MSF_ERR_CUDA;
-            }
             cache.attr_set[0] = true;
+        }
+        e = set_smem_attr((const void*)mssa_tc_kernel<64>, Cfg<64>::kSmem);
+        if (e != cudaSuccess) {
+            set_cuda_error((int)e);
+            return MSF_ERR_CUDA;
         }
         e = launch_pdl(mssa_tc_kernel<64>, dim3((unsigned)ncta), dim3(kThreads), Cfg<64>::kSmem, st,
                        cache.maps, tp);

@@ -278,14 +278,8 @@ cudaError_t launch_bn(const GemmTcArgs* gs, int n, int batch, int splits, cudaSt
     p.splits = splits;
     p.C32 = gs[0].C32;
     p.status = gs[0].status;
-    static bool attr = false;
-    if (!attr) {
-        cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             GCfg<BN, STAGES>::kSmem);
-        if (e != cudaSuccess) return e;
-        attr = true;
-    }
+    cudaError_t e = set_smem_attr((const void*)gemm_tc_kernel<BN, STAGES>, GCfg<BN, STAGES>::kSmem);
+    if (e != cudaSuccess) return e;
     dim3 grid((unsigned)tiles, 1, (unsigned)(batch * splits));
     return launch_pdl(gemm_tc_kernel<BN, STAGES>, grid, dim3(kThreads), GCfg<BN, STAGES>::kSmem, st,
                       maps, p);

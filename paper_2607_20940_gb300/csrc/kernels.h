@@ -9,6 +9,17 @@
 
 namespace msf {
 
+// Set the dynamic shared-memory limit of kernel `fn` to `bytes` (and, if
+// carveout >= 0, its preferred shared-memory carveout in percent) on the
+// current device, once per (kernel, device): the attribute belongs to a
+// device's context, so a process that launches on several devices needs it on
+// each. Thread-safe.
+cudaError_t set_smem_attr(const void* fn, int bytes, int carveout = -1);
+
+// One block that waits, with the bounded wait of the tcgen05 kernels, on an
+// mbarrier nothing arrives at, then raises the TIMEOUT bit of *status.
+cudaError_t launch_wait_timeout_selftest(unsigned int* status, long long limit_cycles, cudaStream_t st);
+
 // Launch with programmatic stream serialisation (see grid_dep_wait in
 // ptx.cuh): the kernel's launch and prologue may overlap the previous kernel.
 template <typename... KArgs, typename... Args>

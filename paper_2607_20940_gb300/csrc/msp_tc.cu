@@ -581,15 +581,8 @@ cudaError_t launch_msp_embed(const MspEmbedRun* runs, int n, const MspShape& sh,
     p.tokens = (__nv_bfloat16*)tokens;
     p.tok_bstride = tok_bstride;
     p.status = status;
-    static bool attr = false;
-    if (!attr) {
-        cudaError_t e = cudaFuncSetAttribute(msp_embed_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             kEmbedSmem);
-        if (e != cudaSuccess) return e;
-        e = cudaFuncSetAttribute(msp_embed_kernel, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
-        if (e != cudaSuccess) return e;
-        attr = true;
-    }
+    cudaError_t e = set_smem_attr((const void*)msp_embed_kernel, kEmbedSmem, 100);
+    if (e != cudaSuccess) return e;
     return launch_pdl(msp_embed_kernel, dim3((unsigned)tiles, 1, (unsigned)batch), dim3(kThreads), kEmbedSmem,
                       st, maps, p);
 }
@@ -634,13 +627,8 @@ cudaError_t launch_msp_deembed(const void* tokens, long long tok_bstride_elems, 
     p.tok_row0 = tok_row0;
     p.latent = (__nv_bfloat16*)latent;
     p.status = status;
-    static bool attr = false;
-    if (!attr) {
-        cudaError_t e = cudaFuncSetAttribute(msp_deembed_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             kDeSmem);
-        if (e != cudaSuccess) return e;
-        attr = true;
-    }
+    cudaError_t e = set_smem_attr((const void*)msp_deembed_kernel, kDeSmem);
+    if (e != cudaSuccess) return e;
     const dim3 grid((unsigned)(p.m_tiles * (F / kDeBN)), (unsigned)splits, (unsigned)batch);
     return launch_pdl_cluster(msp_deembed_kernel, grid, dim3(kThreads), kDeSmem, st, dim3(1, splits, 1), maps, p);
 }

@@ -35,7 +35,11 @@ void* g_noalloc_addr[kNoAllocMaxDevices];
 
 // Device address of g_noalloc_scratch on the current device. In host code the
 // symbol is only a stand-in, not a device address: kernels must be given the
-// address looked up here, once per device, with that device current.
+// address looked up here, once per device, with that device current. The
+// first lookup on a device also zeroes the status word at the start of the
+// array (a synchronous cudaMemset, so it must not run under stream capture);
+// after that only msf_noalloc_device_status clears it, so a timeout stays
+// visible until it is read.
 msf_status scratch_address(void** out) {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -48,8 +52,10 @@ msf_status scratch_address(void** out) {
     if (!g_noalloc_addr[dev]) {
         void* ptr = nullptr;
         e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
-        if (e != cudaSuccess || !ptr) {
-            msf::set_cuda_error((int)(e != cudaSuccess ? e : cudaErrorInvalidSymbol));
+        if (e == cudaSuccess && !ptr) e = cudaErrorInvalidSymbol;
+        if (e == cudaSuccess) e = cudaMemset(ptr, 0, kNoAllocStatusBytes);
+        if (e != cudaSuccess) {
+            msf::set_cuda_error((int)e);
             return MSF_ERR_CUDA;
         }
         g_noalloc_addr[dev] = ptr;
@@ -96,13 +102,9 @@ extern "C" msf_status msf_unpatchify_noalloc(msf_plan_t plan, int32_t position, 
     float* part = (float*)(raw + raw_bytes);
     cudaStream_t s = (cudaStream_t)stream;
 
-    // The status word must start at zero; the partial sums and raw tokens
-    // are fully overwritten by every call.
-    cudaError_t e = cudaMemsetAsync(status, 0, sizeof(unsigned int), s);
-    if (e != cudaSuccess) {
-        msf::set_cuda_error((int)e);
-        return MSF_ERR_CUDA;
-    }
+    // The partial sums and raw tokens are fully overwritten by every call;
+    // the status word keeps a timeout until msf_noalloc_device_status reads it.
+    cudaError_t e;
     const int P = p.d.patch * p.d.scales[position];
     const int F = sh.C * P * P;
     const int E = p.d.embed_dim;
@@ -130,6 +132,37 @@ extern "C" msf_status msf_unpatchify_noalloc(msf_plan_t plan, int32_t position, 
             e = msf::launch_unpatchify_raw(raw, latent_out, sh, position, (long long)per, 0, p.B,
                                            true, s);
     }
+    if (e != cudaSuccess) {
+        msf::set_cuda_error((int)e);
+        return MSF_ERR_CUDA;
+    }
+    return MSF_OK;
+}
+
+extern "C" msf_status msf_noalloc_device_status(void* stream) {
+    void* base = nullptr;
+    msf_status st = scratch_address(&base);
+    if (st != MSF_OK) return st;
+    cudaStream_t s = (cudaStream_t)stream;
+    unsigned int word = 0;
+    cudaError_t e = cudaStreamSynchronize(s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&word, base, sizeof(word), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(base, 0, sizeof(word), s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) {
+        msf::set_cuda_error((int)e);
+        return MSF_ERR_CUDA;
+    }
+    return word ? MSF_ERR_TIMEOUT : MSF_OK;
+}
+
+extern "C" msf_status msf_noalloc_selftest_wait_timeout(int64_t limit_cycles, void* stream) {
+    if (limit_cycles < 1 || limit_cycles > (int64_t(1) << 31)) return MSF_ERR_INVALID_ARG;
+    void* base = nullptr;
+    msf_status st = scratch_address(&base);
+    if (st != MSF_OK) return st;
+    cudaError_t e = msf::launch_wait_timeout_selftest((unsigned int*)base, (long long)limit_cycles,
+                                                      (cudaStream_t)stream);
     if (e != cudaSuccess) {
         msf::set_cuda_error((int)e);
         return MSF_ERR_CUDA;

@@ -246,6 +246,9 @@ extern "C" msf_status msf_plan_query(msf_plan_t plan, msf_plan_info* info) {
     info->resample_bytes = 2 * bytes * p.B;
     info->pyramid_k_offset = msf::kStatusBytes;
     info->pyramid_v_offset = msf::kStatusBytes + msf::pyramid_bytes(p);
+    info->attention_counter_offset =
+        msf::kStatusBytes + 2 * msf::pyramid_bytes(p) + msf::msp_scratch_bytes(p);
+    info->attention_counter_bytes = msf::attn_counter_bytes(p);
     return MSF_OK;
 }
 

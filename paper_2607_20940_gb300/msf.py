@@ -37,6 +37,7 @@ EXPORTS = (
     "msf_plan_device_status", "msf_kernel_launches", "msf_unpatchify_noalloc",
     "msf_selftest_wait_timeout", "msf_history_commit", "msf_mssa_forward_lse",
     "msf_mssa_backward", "msf_mssa_backward_simt", "msf_history_get", "msf_history_set",
+    "msf_noalloc_device_status", "msf_noalloc_selftest_wait_timeout",
 )
 
 
@@ -77,6 +78,7 @@ class msf_plan_info(ctypes.Structure):
         ("dense_flops", ctypes.c_uint64), ("resample_bytes", ctypes.c_uint64),
         ("pyramid_k_offset", ctypes.c_uint64), ("pyramid_v_offset", ctypes.c_uint64),
         ("backward_workspace_bytes", ctypes.c_uint64), ("backward_flops", ctypes.c_uint64),
+        ("attention_counter_offset", ctypes.c_uint64), ("attention_counter_bytes", ctypes.c_uint64),
     ]
 
 
@@ -104,6 +106,8 @@ def _load():
         "msf_kernel_launches": (ctypes.c_uint64, []),
         "msf_unpatchify_noalloc": (ctypes.c_int, [P, I32, VP, VP, VP, VP]),
         "msf_selftest_wait_timeout": (ctypes.c_int, [P, ctypes.c_int64, VP]),
+        "msf_noalloc_device_status": (ctypes.c_int, [VP]),
+        "msf_noalloc_selftest_wait_timeout": (ctypes.c_int, [ctypes.c_int64, VP]),
         "msf_history_commit": (ctypes.c_int, [P]),
         "msf_history_get": (ctypes.c_int, [P, ctypes.POINTER(msf_history_state)]),
         "msf_history_set": (ctypes.c_int, [P, ctypes.POINTER(msf_history_state)]),
@@ -263,6 +267,15 @@ def msf_plan_device_status(plan: int, stream=None) -> int:
 def msf_unpatchify_noalloc(plan: int, position: int, tokens, w_out, latent_out, stream=None) -> None:
     _check(_lib.msf_unpatchify_noalloc(plan, position, _ptr(tokens), _ptr(w_out), _ptr(latent_out),
                                        _stream(stream)), "msf_unpatchify_noalloc")
+
+
+def msf_noalloc_device_status(stream=None) -> int:
+    return _lib.msf_noalloc_device_status(_stream(stream))
+
+
+def msf_noalloc_selftest_wait_timeout(limit_cycles: int, stream=None) -> None:
+    _check(_lib.msf_noalloc_selftest_wait_timeout(limit_cycles, _stream(stream)),
+           "msf_noalloc_selftest_wait_timeout")
 
 
 def msf_selftest_wait_timeout(plan: int, limit_cycles: int, stream=None) -> None:

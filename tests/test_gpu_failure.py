@@ -104,3 +104,34 @@ def test_canaries_around_every_output():
         assert guards_intact(buf), name
     assert torch.isfinite(out.float()).all() and torch.isfinite(tok.float()).all()
     assert torch.isfinite(lat.float()).all()
+
+
+def test_timeout_clears_attention_merge_counters():
+    """A launch that gives up can leave the per-block merge counters counted.
+    The status read that reports the timeout must zero them, so that the next
+    launch merges only finished pieces. The stale counters are planted from
+    the host and the TIMEOUT bit comes from the self-test wait: no attention
+    launch is made to fail."""
+    m = msf()
+    w = synth.TINY  # every block is split over several CTAs: merges use the counters
+    x = synth.attention_inputs(w, BF16)
+    plan = make_plan(w, BF16)
+    dx = device_inputs(x, w.history_capacity)
+    ws = bind(plan, dx)
+    off, nb = int(plan.info.attention_counter_offset), int(plan.info.attention_counter_bytes)
+    assert nb > 0 and off % 256 == 0 and off + nb <= ws.numel()
+    cnt = ws[off:off + nb].view(torch.int32)
+    out = torch.empty_like(dx["q"])
+    plan.kv_resample(dx["k_win"], dx["v_win"])
+    plan.mssa_forward(dx["q"], dx["k_win"], dx["v_win"], out)
+    assert plan.device_status() == m.MSF_OK
+    assert bool((cnt == 0).all())  # every merge resets the counter it used
+    cnt.fill_(0x00010001)  # one piece finished and one written, left behind
+    plan.selftest_wait_timeout(200_000)
+    assert plan.device_status() == m.MSF_ERR_TIMEOUT
+    assert bool((cnt == 0).all())
+    out.fill_(float("nan"))
+    plan.mssa_forward(dx["q"], dx["k_win"], dx["v_win"], out)
+    assert plan.device_status() == m.MSF_OK
+    mx, mean = err_stats(out, oracle_mssa(x, w, 0))
+    assert mx <= 2e-2 and mean <= 2e-3

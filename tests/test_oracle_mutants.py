@@ -161,3 +161,71 @@ def test_strided_adjoint_to_the_wrong_token(monkeypatch):
         return np.roll(grid, 1, axis=2).reshape(y.shape)   # one column to the right
     monkeypatch.setattr(mssa_bwd, "resample_adjoint", bad)
     _fails(bpins.test_backward_equals_torch_autograd, mssa.STRIDED, (1, 2), 4, 4, 1, 3, 1)
+
+
+# ------------------------------------------- pyramid part, tier projections --
+
+def test_pyramid_states_before_history(monkeypatch):
+    good = mssa.pyramid_segment
+
+    def bad(kv_win, kv_hist, scales, gh, gw, g, mode=mssa.AVG, frames=1):
+        seg = good(kv_win, kv_hist, scales, gh, gw, g, mode, frames)
+        nh = np.asarray(kv_hist).shape[1] * frames * (gh // g) * (gw // g)
+        return np.concatenate([seg[:, nh:], seg[:, :nh]], axis=1)
+    monkeypatch.setattr(mssa, "pyramid_segment", bad)
+    _fails(pins.test_pyramid_segment_is_context_rows_pooled_by_loops, mssa.AVG, (1, 1, 2, 2, 2),
+           4, 8, 2, 1)
+
+
+def test_pyramid_finer_states_pooled_by_g_not_g_over_s(monkeypatch):
+    def bad(kv_win, kv_hist, scales, gh, gw, g, mode=mssa.AVG, frames=1):
+        offs = schedule.token_offsets(scales, gh, gw, frames)
+        cnt = schedule.token_counts(scales, gh, gw, frames)
+        parts = [mssa.resample_frames(kv_hist[:, f], frames, gh, gw, g, mode)
+                 for f in range(kv_hist.shape[1])]
+        for l, s in enumerate(scales):
+            if s < g:
+                st = np.asarray(kv_win[:, offs[l]:offs[l] + cnt[l]], dtype=np.float64)
+                # stride g on a state that is already s times coarser
+                parts.append(mssa.resample_frames(st, frames, gh // s, gw // s, g, mode))
+        return np.concatenate(parts, axis=1)
+    monkeypatch.setattr(mssa, "pyramid_segment", bad)
+    _fails(pins.test_pyramid_segment_is_context_rows_pooled_by_loops, mssa.AVG, (1, 2, 4, 4),
+           8, 8, 1, 1)
+
+
+def test_tier_weights_swapped_between_states(monkeypatch):
+    good = msp.patchify_window
+
+    def bad(latent, scales, patch, w_tier=None):
+        if w_tier is None:
+            return good(latent, scales, patch, w_tier)
+        # the window's states embedded in reverse position order
+        x = np.asarray(latent, dtype=np.float64)
+        cut = msp.patchify_chunk if x.ndim == 6 else msp.patchify
+        blocks = [cut(x[:, l], patch * s) @ np.asarray(w_tier[s]) for l, s in enumerate(scales)]
+        return np.concatenate(blocks[::-1], axis=1)
+    monkeypatch.setattr(msp, "patchify_window", bad)
+    _fails(pins.test_tier_embedding_is_a_strided_conv_per_state, 1)
+
+
+def test_tier_embedding_weight_transposed(monkeypatch):
+    good = msp.patchify_window
+
+    def bad(latent, scales, patch, w_tier=None):
+        if w_tier is None:
+            return good(latent, scales, patch, w_tier)
+        sq = {s: (np.asarray(w).T if np.asarray(w).shape[0] == np.asarray(w).shape[1] else w)
+              for s, w in w_tier.items()}
+        return good(latent, scales, patch, sq)
+    monkeypatch.setattr(msp, "patchify_window", bad)
+    _fails(pins.test_tier_embedding_is_a_strided_conv_per_state, 1)
+
+
+def test_deembedding_weight_transposed(monkeypatch):
+    good = msp.unpatchify_state
+
+    def bad(tokens, P, C, Hl, Wl, w_out=None, frames=0):
+        return good(tokens, P, C, Hl, Wl, None if w_out is None else np.asarray(w_out).T, frames)
+    monkeypatch.setattr(msp, "unpatchify_state", bad)
+    _fails(pins.test_deembedding_is_linear_then_fold, 2)

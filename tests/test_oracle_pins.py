@@ -377,3 +377,105 @@ def test_chunked_patch_embedding_equals_conv3d():
     ref = conv.numpy().reshape(B, E, -1).transpose(0, 2, 1)
     np.testing.assert_allclose(t @ W, ref, rtol=0, atol=1e-12)
     assert np.array_equal(msp.unpatchify_chunk(t, P, C, F, Hl, Wl), x)
+
+
+# ------------------------------------------- pyramid part and tier projections --
+
+def _pooled_row_by_loops(src, kind_grid, st, row, col, mode):
+    """One Subsample row of Eq. 4 built by explicit loops from its source
+    frame. src [B, F*gh*gw, H, D] holds F latent-frame grids of gh x gw (the
+    source grid before pooling); (row, col) is on the pooled grid with the
+    latent frame folded into the row (row = f * (gh/st) + i)."""
+    gh, gw = kind_grid
+    ph = gh // st
+    f, i = divmod(row, ph)
+    base = f * gh * gw
+    if mode == mssa.STRIDED:
+        return src[:, base + (st * i) * gw + st * col]
+    acc = np.zeros(src.shape[:1] + src.shape[2:])
+    for dy in range(st):
+        for dx in range(st):
+            acc = acc + src[:, base + (st * i + dy) * gw + (st * col + dx)]
+    return acc / (st * st)
+
+
+@pytest.mark.parametrize("mode", [mssa.AVG, mssa.STRIDED])
+@pytest.mark.parametrize("scales,gh,gw,nh,F", [
+    ((1, 1, 2, 2, 2), 4, 8, 2, 1),
+    ((1, 2, 4, 4), 8, 8, 1, 1),
+    ((1, 1, 2, 4), 8, 4, 2, 2),
+])
+def test_pyramid_segment_is_context_rows_pooled_by_loops(mode, scales, gh, gw, nh, F):
+    """The resampled part of group g's context (the segment the GPU pyramid
+    holds) is, row for row, the history and finer-window rows of Eq. 4's
+    context in context order, each pooled from its source by explicit loops."""
+    rng = np.random.default_rng(11)
+    B, H, D = 2, 2, 3
+    N = sum(schedule.token_counts(scales, gh, gw, F))
+    kv_win = rng.standard_normal((B, N, H, D))
+    kv_hist = rng.standard_normal((B, nh, F * gh * gw, H, D))
+    offs = schedule.token_offsets(scales, gh, gw, F)
+    cnt = schedule.token_counts(scales, gh, gw, F)
+    for g in sorted(set(scales)):
+        if g == 1:
+            continue
+        seg = mssa.pyramid_segment(kv_win, kv_hist, scales, gh, gw, g, mode, F)
+        rows = [r for r in schedule.context_rows(scales, gh, gw, 0, nh, g, F)
+                if r[0] == schedule.HIST or (r[0] == schedule.WIN and scales[r[1]] < g)]
+        assert seg.shape == (B, len(rows), H, D)
+        for n, (kind, frame, st, row, col) in enumerate(rows):
+            if kind == schedule.HIST:
+                src, grid = kv_hist[:, frame], (gh, gw)
+            else:
+                s = scales[frame]
+                src, grid = kv_win[:, offs[frame]:offs[frame] + cnt[frame]], (gh // s, gw // s)
+            want = _pooled_row_by_loops(src, grid, st, row, col, mode)
+            np.testing.assert_allclose(seg[:, n], want, rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("F", [1, 2])
+def test_tier_embedding_is_a_strided_conv_per_state(F):
+    """MSP of a window with tier projections: each state is embedded by the
+    patch-embedding conv (kernel = stride = its patch P_l) of its own tier's
+    weight, and the states' token blocks follow in position order. Weights of
+    the patch-2 tier are square (C*P^2 = E) so that using one transposed
+    cannot go unnoticed."""
+    rng = np.random.default_rng(12)
+    scales, patch, C, E, B = (1, 1, 2, 2), 2, 4, 16, 2
+    Hl, Wl = 8, 16
+    lat_shape = (B, len(scales), C, Hl, Wl) if F == 1 else (B, len(scales), C, F, Hl, Wl)
+    latent = rng.standard_normal(lat_shape)
+    w_tier = {s: rng.standard_normal((C * (patch * s) ** 2, E)) for s in set(scales)}
+    got = msp.patchify_window(latent, scales, patch, w_tier)
+    blocks = []
+    for l, s in enumerate(scales):
+        P = patch * s
+        wt = torch.from_numpy(w_tier[s].T.reshape(E, C, P, P).copy())
+        x = torch.from_numpy(latent[:, l].copy())
+        if F == 1:
+            y = torch.nn.functional.conv2d(x, wt, stride=P)              # [B, E, gh, gw]
+            blocks.append(y.flatten(2).transpose(1, 2))
+        else:
+            y = torch.nn.functional.conv3d(x, wt.unsqueeze(2), stride=(1, P, P))  # [B, E, F, gh, gw]
+            blocks.append(y.flatten(2).transpose(1, 2))
+    want = torch.cat(blocks, dim=1).numpy()
+    assert got.shape == want.shape
+    np.testing.assert_allclose(got, want, rtol=0, atol=1e-10)
+
+
+@pytest.mark.parametrize("P", [2, 4])
+def test_deembedding_is_linear_then_fold(P):
+    """De-embedding + unpatchify of one state: the nn.Linear map E -> C*P^2
+    of every token, then torch's fold with kernel = stride = P (the inverse
+    patch rearrangement, feature order (c, dy, dx)). E = C*P^2 makes the
+    weight square, so a transposed use changes the values, not the shape."""
+    rng = np.random.default_rng(13)
+    B, C, gh, gw = 2, 3, 3, 5
+    E = C * P * P
+    tokens = rng.standard_normal((B, gh * gw, E))
+    w_out = rng.standard_normal((E, C * P * P))  # [E, C*P^2]: tokens @ w_out
+    got = msp.unpatchify_state(tokens, P, C, gh * P, gw * P, w_out=w_out)
+    lin = torch.nn.functional.linear(torch.from_numpy(tokens), torch.from_numpy(w_out.T.copy()))
+    want = torch.nn.functional.fold(lin.transpose(1, 2), output_size=(gh * P, gw * P),
+                                    kernel_size=P, stride=P).numpy()
+    np.testing.assert_allclose(got, want, rtol=0, atol=1e-10)
