@@ -88,3 +88,65 @@ def unpatchify_state(tokens: np.ndarray, P: int, C: int, Hl: int, Wl: int, w_out
     if frames:
         return unpatchify_chunk(t, P, C, frames, Hl, Wl)
     return unpatchify(t, P, C, Hl, Wl)
+
+
+# ------------------------------------------------------------ tier modules --
+#
+# Sec. 4.1 gives every coarse tier its own module: patch embedding and
+# de-embedding, LoRA adapters and a latent residual branch; the native tier
+# keeps the pretrained path and has none of the extras. The paper does not
+# fix where the adapters sit or what the residual branch computes; the
+# reading taken here (row vectors, x @ W):
+#   embedding      t = x W + g (x A) B          W [K, E], A [K, r], B [r, E]
+#   de-embedding   y = h Wo + g (h Ao) Bo + x R  Wo [E, K], Ao [E, r], Bo [r, K]
+# where x is the state's raw patch vector (K = C*P^2 features, the input
+# latent of the same state), h its token after the backbone, g the LoRA
+# scale and R [K, K] the latent residual branch: a learned linear map of the
+# input patch added to the de-embedded output before the patches are put back.
+# Every term is an fp64 matrix product in the order written.
+
+def embed_tier(x, w, lora_a=None, lora_b=None, gamma=1.0):
+    """Tier patch embedding of raw patch vectors x [..., K] -> [..., E]."""
+    x = np.asarray(x, dtype=np.float64)
+    t = x @ np.asarray(w, dtype=np.float64)
+    if lora_a is not None:
+        t = t + gamma * ((x @ np.asarray(lora_a, dtype=np.float64)) @ np.asarray(lora_b, dtype=np.float64))
+    return t
+
+
+def deembed_tier(h, w_out, lora_a=None, lora_b=None, gamma=1.0, x=None, residual=None):
+    """Tier de-embedding of tokens h [..., E] -> patch vectors [..., K], with
+    the latent residual x R of the state's input patch vectors x [..., K]."""
+    h = np.asarray(h, dtype=np.float64)
+    y = h @ np.asarray(w_out, dtype=np.float64)
+    if lora_a is not None:
+        y = y + gamma * ((h @ np.asarray(lora_a, dtype=np.float64)) @ np.asarray(lora_b, dtype=np.float64))
+    if residual is not None:
+        y = y + np.asarray(x, dtype=np.float64) @ np.asarray(residual, dtype=np.float64)
+    return y
+
+
+def patchify_window_tiers(latent, scales, patch, tiers):
+    """MSP of a window with tier modules: latent [B, T, C, Hl, Wl] ->
+    [B, N_MSP, E], states in position order. tiers: dict scale -> dict with
+    'w' [K, E] and optionally 'lora_a' [K, r], 'lora_b' [r, E], 'gamma'."""
+    x = np.asarray(latent, dtype=np.float64)
+    out = []
+    for l, s in enumerate(scales):
+        t = tiers[s]
+        xp = patchify(x[:, l], patch * s)
+        out.append(embed_tier(xp, t["w"], t.get("lora_a"), t.get("lora_b"), t.get("gamma", 1.0)))
+    return np.concatenate(out, axis=1)
+
+
+def unpatchify_state_tier(tokens, latent_state, P, tier):
+    """De-embedding of one state with its tier module: tokens [B, N_l, E] and
+    the state's input latent [B, C, Hl, Wl] -> output latent [B, C, Hl, Wl].
+    tier: dict with 'w_out' [E, K] and optionally 'out_a' [E, r], 'out_b'
+    [r, K], 'gamma', 'residual' [K, K]."""
+    lat = np.asarray(latent_state, dtype=np.float64)
+    B, C, Hl, Wl = lat.shape
+    x = patchify(lat, P)
+    y = deembed_tier(tokens, tier["w_out"], tier.get("out_a"), tier.get("out_b"),
+                     tier.get("gamma", 1.0), x, tier.get("residual"))
+    return unpatchify(y, P, C, Hl, Wl)

@@ -160,6 +160,36 @@ def msp_inputs(w: Workload, dtype: torch.dtype = torch.bfloat16, seed: Optional[
     return out
 
 
+def tier_inputs(w: Workload, rank: int, dtype: torch.dtype = torch.bfloat16,
+                seed: Optional[int] = None, gamma: float = 0.5) -> dict:
+    """Seeded weights of the coarse tiers' modules (every scale s > 1 of the
+    window), in the row-vector orientation x @ W, for each scale s with
+    K = C*(patch*s)^2: LoRA of the embedding ``lora_a`` [K, r] ~ N(0, 1/K),
+    ``lora_b`` [r, E] ~ N(0, 1/r); a de-embedding ``w_out`` [E, K] ~ N(0, 1/E)
+    with LoRA ``out_a`` [E, r] ~ N(0, 1/E), ``out_b`` [r, K] ~ N(0, 1/r); the
+    latent residual ``residual`` [K, K] ~ N(0, 1/K); and the LoRA scale
+    ``gamma``. The tier's embedding ``w`` is msp_inputs' w_tier[s]. Drawn
+    from their own generator, after nothing else."""
+    seed = (w.seed if seed is None else seed) + 104729
+    gen = torch.Generator().manual_seed(seed)
+    C, E, r = w.latent_channels, w.embed_dim, rank
+    out = {}
+    for s in sorted(set(w.scales)):
+        if s == 1:
+            continue
+        K = C * (w.patch * s) ** 2
+        out[s] = {
+            "lora_a": _randn(gen, (K, r), K ** -0.5, dtype),
+            "lora_b": _randn(gen, (r, E), r ** -0.5, dtype),
+            "w_out": _randn(gen, (E, K), E ** -0.5, dtype),
+            "out_a": _randn(gen, (E, r), E ** -0.5, dtype),
+            "out_b": _randn(gen, (r, K), r ** -0.5, dtype),
+            "residual": _randn(gen, (K, K), K ** -0.5, dtype),
+            "gamma": gamma,
+        }
+    return out
+
+
 def to_f64(t: torch.Tensor):
     """Exact widening of the stored values to a float64 numpy array."""
     return t.to(torch.float64).numpy()

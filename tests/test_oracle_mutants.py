@@ -229,3 +229,34 @@ def test_deembedding_weight_transposed(monkeypatch):
         return good(tokens, P, C, Hl, Wl, None if w_out is None else np.asarray(w_out).T, frames)
     monkeypatch.setattr(msp, "unpatchify_state", bad)
     _fails(pins.test_deembedding_is_linear_then_fold, 2)
+
+
+# ------------------------------------------------------- tier modules --
+
+def test_tier_lora_scale_dropped(monkeypatch):
+    good = msp.embed_tier
+    monkeypatch.setattr(msp, "embed_tier", lambda x, w, a=None, b=None, gamma=1.0: good(x, w, a, b, 1.0))
+    _fails(pins.test_tier_lora_embedding_is_a_conv_with_the_merged_weight)
+    good_d = msp.deembed_tier
+    monkeypatch.setattr(msp, "deembed_tier",
+                        lambda h, wo, a=None, b=None, gamma=1.0, x=None, r=None: good_d(h, wo, a, b, 1.0, x, r))
+    _fails(pins.test_tier_deembedding_lora_is_linear_with_the_merged_weight_then_fold)
+
+
+def test_latent_residual_transposed(monkeypatch):
+    good = msp.deembed_tier
+
+    def bad(h, w_out, a=None, b=None, gamma=1.0, x=None, residual=None):
+        return good(h, w_out, a, b, gamma, x, None if residual is None else np.asarray(residual).T)
+    monkeypatch.setattr(msp, "deembed_tier", bad)
+    _fails(pins.test_latent_residual_is_a_patch_conv_then_fold, 2)
+
+
+def test_latent_residual_of_the_output_not_the_input(monkeypatch):
+    good = msp.deembed_tier
+
+    def bad(h, w_out, a=None, b=None, gamma=1.0, x=None, residual=None):
+        y = good(h, w_out, a, b, gamma)
+        return y if residual is None else y + y @ np.asarray(residual)
+    monkeypatch.setattr(msp, "deembed_tier", bad)
+    _fails(pins.test_latent_residual_identity_passes_the_input_latent_through, 2)

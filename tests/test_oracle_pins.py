@@ -479,3 +479,100 @@ def test_deembedding_is_linear_then_fold(P):
     want = torch.nn.functional.fold(lin.transpose(1, 2), output_size=(gh * P, gw * P),
                                     kernel_size=P, stride=P).numpy()
     np.testing.assert_allclose(got, want, rtol=0, atol=1e-10)
+
+
+# ------------------------------------------------------- tier modules --
+
+def _tier_weights(rng, K, E, r):
+    return {"w": rng.standard_normal((K, E)), "lora_a": rng.standard_normal((K, r)),
+            "lora_b": rng.standard_normal((r, E)), "gamma": 0.375}
+
+
+def test_tier_lora_embedding_is_a_conv_with_the_merged_weight():
+    """Embedding with LoRA = the patch-embedding conv whose kernel is the tier
+    weight plus the scaled rank-r product (linearity of the conv in its
+    weight); the native tier (no adapters) is the plain conv."""
+    rng = np.random.default_rng(21)
+    scales, patch, C, E, B, r = (1, 2, 2), 2, 4, 24, 2, 8
+    latent = rng.standard_normal((B, len(scales), C, 8, 16))
+    tiers = {1: {"w": rng.standard_normal((C * 4, E))},
+             2: _tier_weights(rng, C * 16, E, r)}
+    got = msp.patchify_window_tiers(latent, scales, patch, tiers)
+    blocks = []
+    for l, s in enumerate(scales):
+        P, t = patch * s, tiers[s]
+        merged = t["w"] + (t["gamma"] * (t["lora_a"] @ t["lora_b"]) if "lora_a" in t else 0.0)
+        wt = torch.from_numpy(np.ascontiguousarray(merged.T).reshape(E, C, P, P))
+        y = torch.nn.functional.conv2d(torch.from_numpy(latent[:, l].copy()), wt, stride=P)
+        blocks.append(y.flatten(2).transpose(1, 2))
+    np.testing.assert_allclose(got, torch.cat(blocks, 1).numpy(), rtol=0, atol=1e-9)
+
+
+def test_tier_lora_update_has_rank_r_and_vanishes_with_a_zero_up_projection():
+    rng = np.random.default_rng(22)
+    K, E, r, n = 64, 48, 8, 200
+    t = _tier_weights(rng, K, E, r)
+    x = rng.standard_normal((n, K))
+    delta = msp.embed_tier(x, t["w"], t["lora_a"], t["lora_b"], t["gamma"]) - msp.embed_tier(x, t["w"])
+    sv = np.linalg.svd(delta, compute_uv=False)
+    assert sv[r - 1] > 1e-3 * sv[0] and sv[r] < 1e-10 * sv[0]
+    zero = msp.embed_tier(x, t["w"], t["lora_a"], np.zeros_like(t["lora_b"]), t["gamma"])
+    assert np.array_equal(zero, msp.embed_tier(x, t["w"]))
+    d2 = msp.deembed_tier(x[:, :E], t["w"].T, t["lora_b"].T, t["lora_a"].T, t["gamma"]) - \
+        msp.deembed_tier(x[:, :E], t["w"].T)
+    sv = np.linalg.svd(d2, compute_uv=False)
+    assert sv[r] < 1e-10 * sv[0]
+
+
+@pytest.mark.parametrize("P", [2, 4])
+def test_latent_residual_identity_passes_the_input_latent_through(P):
+    """With R = I, no de-embedding weight and no adapters the tier's output
+    latent is its input latent, exactly; with a de-embedding it is that
+    de-embedding plus the input latent."""
+    rng = np.random.default_rng(23)
+    B, C, gh, gw, E = 2, 3, 3, 4, 20
+    K = C * P * P
+    lat = rng.standard_normal((B, C, gh * P, gw * P))
+    tok = rng.standard_normal((B, gh * gw, E))
+    ident = {"w_out": np.zeros((E, K)), "residual": np.eye(K)}
+    assert np.array_equal(msp.unpatchify_state_tier(tok, lat, P, ident), lat)
+    w_out = rng.standard_normal((E, K))
+    got = msp.unpatchify_state_tier(tok, lat, P, {"w_out": w_out, "residual": np.eye(K)})
+    base = msp.unpatchify_state(tok, P, C, gh * P, gw * P, w_out=w_out)
+    np.testing.assert_allclose(got, base + lat, rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("P", [2, 4])
+def test_latent_residual_is_a_patch_conv_then_fold(P):
+    """The residual branch alone (zero de-embedding) is a strided conv of the
+    input latent (kernel = stride = P, weight R as C*P^2 filters) followed by
+    fold, torch's inverse patch rearrangement. R is square, so a transposed
+    use changes the values."""
+    rng = np.random.default_rng(24)
+    B, C, gh, gw, E = 2, 2, 3, 5, 8
+    K = C * P * P
+    lat = rng.standard_normal((B, C, gh * P, gw * P))
+    R = rng.standard_normal((K, K))
+    got = msp.unpatchify_state_tier(np.zeros((B, gh * gw, E)), lat, P,
+                                    {"w_out": np.zeros((E, K)), "residual": R})
+    wt = torch.from_numpy(np.ascontiguousarray(R.T).reshape(K, C, P, P))
+    y = torch.nn.functional.conv2d(torch.from_numpy(lat), wt, stride=P)  # [B, K, gh, gw]
+    want = torch.nn.functional.fold(y.flatten(2), output_size=(gh * P, gw * P), kernel_size=P,
+                                    stride=P).numpy()
+    np.testing.assert_allclose(got, want, rtol=0, atol=1e-10)
+
+
+def test_tier_deembedding_lora_is_linear_with_the_merged_weight_then_fold():
+    rng = np.random.default_rng(25)
+    B, C, P, gh, gw, E, r = 2, 2, 4, 2, 3, 40, 8
+    K = C * P * P
+    tok = rng.standard_normal((B, gh * gw, E))
+    lat = rng.standard_normal((B, C, gh * P, gw * P))
+    t = {"w_out": rng.standard_normal((E, K)), "out_a": rng.standard_normal((E, r)),
+         "out_b": rng.standard_normal((r, K)), "gamma": 0.625}
+    got = msp.unpatchify_state_tier(tok, lat, P, t)
+    merged = t["w_out"] + t["gamma"] * (t["out_a"] @ t["out_b"])
+    lin = torch.nn.functional.linear(torch.from_numpy(tok), torch.from_numpy(merged.T.copy()))
+    want = torch.nn.functional.fold(lin.transpose(1, 2), output_size=(gh * P, gw * P),
+                                    kernel_size=P, stride=P).numpy()
+    np.testing.assert_allclose(got, want, rtol=0, atol=1e-9)
