@@ -222,6 +222,64 @@ msf_status msf_patchify(msf_plan_t plan, const void* latent, const void* const* 
 msf_status msf_unpatchify(msf_plan_t plan, int32_t position, const void* tokens,
                           const void* w_out, void* latent_out, void* stream);
 
+/* One tier's module (Sec. 4.1: every patch size has its own patch embedding
+ * and de-embedding, LoRA adapters and a latent residual branch; the native
+ * tier keeps the pretrained path). The paper does not define where the
+ * adapters sit or what the residual branch computes; this library takes:
+ *   embedding     t = W x + g * U (A x)          (x: the K = C*P^2 raw patch
+ *                                                 vector of a token)
+ *   de-embedding  y = Wo h + g * Uo (Ao h) + R x  (h: the token after the
+ *                                                 backbone, x: the raw patch
+ *                                                 vector of the same token of
+ *                                                 the state's input latent)
+ * with rank-r LoRA factors A/U, Ao/Uo, scale g and the latent residual R.
+ * All device pointers, bf16, 16-byte aligned, nn.Linear layouts:
+ *   w_embed [E, K], embed_down (A) [r, K], embed_up (U) [E, r],
+ *   w_out [K, E], out_down (Ao) [r, E], out_up (Uo) [K, r], residual [K, K].
+ * A NULL embed_down / out_down means no adapter on that projection (its up
+ * pointer is then ignored), a NULL residual no residual branch. */
+typedef struct msf_tier_module {
+    const void* w_embed;
+    const void* embed_down;
+    const void* embed_up;
+    const void* w_out;
+    const void* out_down;
+    const void* out_up;
+    const void* residual;
+    int32_t lora_rank;   /* r: 8..64, a multiple of 8, when an adapter is given */
+    float lora_scale;    /* g */
+} msf_tier_module;
+
+/* MSP patchify with tier modules (Sec. 4.1): tokens [B, N, E] of the window
+ * latent [B, T, C, Hl, Wl] (as msf_patchify), state l embedded by
+ * tiers[l] (an array of T pointers; consecutive states with the same pointer
+ * and scale share one run). With an embedding adapter the tokens get
+ * g * U (A x): the codes g * A x (fp32 sums, rounded once to bf16) are
+ * computed by one launch of the fused gather + GEMM kernel into the
+ * workspace, and the embedding launch adds one K chunk (codes x U) to the
+ * same fp32 accumulation. bf16 plans with an embedding, bound (the codes
+ * live in the workspace). Errors: INVALID_ARG (NULL or misaligned pointers,
+ * rank outside 8..64 or not a multiple of 8), UNSUPPORTED (fp32 plan, no
+ * embedding, E not a multiple of 64, a patch edge that does not divide 64),
+ * STATE (not bound), CUDA. */
+msf_status msf_patchify_tiers(msf_plan_t plan, const void* latent, const msf_tier_module* const* tiers,
+                              void* tokens, void* stream);
+
+/* De-embedding + unpatchify of window position `position` with its tier's
+ * module: tokens [B, N, E] (for example the attention output viewed as
+ * [B, N, H*D]), latent_in the window latent [B, T, C, Hl, Wl] the pass
+ * started from (read only when tier->residual is set), latent_out
+ * [B, C, Hl, Wl]. The adapter's codes g * Ao h come from a tensor-core GEMM
+ * into the workspace; the residual's raw patch vectors from the raw
+ * patchify kernel into the workspace; the de-embedding kernel then sums the
+ * E/64 token chunks, the code chunk and the K/64 residual chunks in one fp32
+ * accumulation (split over a cluster) and rounds once. Errors: INVALID_ARG,
+ * UNSUPPORTED (fp32 plan, no embedding, K or E not a multiple of 64), STATE,
+ * CUDA. */
+msf_status msf_unpatchify_tier(msf_plan_t plan, int32_t position, const void* tokens,
+                               const void* latent_in, const msf_tier_module* tier, void* latent_out,
+                               void* stream);
+
 /* Build the per-scale key/value pyramid in the workspace: for every query
  * group g > 1, the bound history frames (fine, pooled by g) and the window
  * states with s_l < g (pooled by g/s_l), from k_win, v_win [B, N, H, D].

@@ -770,6 +770,152 @@ extern "C" msf_status msf_unpatchify(msf_plan_t plan, int32_t position, const vo
 }
 
 namespace {
+
+bool tier_lora_ok(const void* down, const void* up, int rank) {
+    if (!down) return true;
+    return up && rank >= 8 && rank <= msf::kTierCodeCols && rank % 8 == 0 && aligned16(down) && aligned16(up);
+}
+
+}  // namespace
+
+extern "C" msf_status msf_patchify_tiers(msf_plan_t plan, const void* latent,
+                                         const msf_tier_module* const* tiers, void* tokens, void* stream) {
+    if (!plan || !latent || !tokens || !tiers) return MSF_ERR_INVALID_ARG;
+    const Plan& p = *plan;
+    if (p.d.latent_channels <= 0 || p.d.patch <= 0 || p.d.embed_dim <= 0 || p.elem != 2)
+        return MSF_ERR_UNSUPPORTED;
+    if (!p.bound) return MSF_ERR_STATE;  // the LoRA codes go through the workspace
+    if (!aligned16(latent) || !aligned16(tokens)) return MSF_ERR_INVALID_ARG;
+    for (int l = 0; l < p.T; ++l) {
+        const msf_tier_module* t = tiers[l];
+        if (!t || !t->w_embed || !aligned16(t->w_embed)) return MSF_ERR_INVALID_ARG;
+        if (!tier_lora_ok(t->embed_down, t->embed_up, t->lora_rank)) return MSF_ERR_INVALID_ARG;
+    }
+    const msf::MspShape sh = msp_shape(p);
+    cudaStream_t s = (cudaStream_t)stream;
+    const int E = p.d.embed_dim;
+    char* codes = msf::tier_codes(p);
+    const long long codes_bstride = (long long)p.N * msf::kTierCodeCols;
+    // Runs of consecutive states that share a tier module.
+    msf::MspEmbedRun runs[MSF_MAX_STATES], code_runs[MSF_MAX_STATES];
+    int n_runs = 0, n_code = 0;
+    for (int l0 = 0; l0 < p.T;) {
+        int l1 = l0 + 1;
+        while (l1 < p.T && p.d.scales[l1] == p.d.scales[l0] && tiers[l1] == tiers[l0]) ++l1;
+        const msf_tier_module* t = tiers[l0];
+        msf::MspEmbedRun& r = runs[n_runs++];
+        r.w = t->w_embed;
+        r.P = p.d.patch * p.d.scales[l0];
+        r.K = sh.C * r.P * r.P;
+        r.l0 = l0;
+        r.n_l = p.st_n[l0];
+        r.M = p.st_off[l1 - 1] + p.st_n[l1 - 1] - p.st_off[l0];
+        r.gw = sh.Wl / r.P;
+        r.tok_off = p.st_off[l0];
+        if (t->embed_down) {
+            // The rank-r codes gamma * x A^T of the run's tokens, by the same
+            // fused gather + GEMM kernel with A as its weight (rows past r and
+            // columns past 64 are zero), then the embedding with one more K
+            // chunk: codes x the up projection.
+            msf::MspEmbedRun& c = code_runs[n_code++];
+            c = r;
+            c.w = t->embed_down;
+            c.w_rows = t->lora_rank;
+            c.scale = t->lora_scale;
+            r.lora_up = t->embed_up;
+            r.rank = t->lora_rank;
+            r.codes = codes + (size_t)r.tok_off * msf::kTierCodeCols * 2;
+            r.codes_bstride = codes_bstride;
+        }
+        l0 = l1;
+    }
+    for (int r0 = 0; r0 < n_code; r0 += msf::kMaxGemmProblems) {
+        const int n = n_code - r0 < msf::kMaxGemmProblems ? n_code - r0 : msf::kMaxGemmProblems;
+        if (!msf::msp_embed_supported(code_runs + r0, n, msf::kTierCodeCols)) return MSF_ERR_UNSUPPORTED;
+    }
+    for (int r0 = 0; r0 < n_runs; r0 += msf::kMaxGemmProblems) {
+        const int n = n_runs - r0 < msf::kMaxGemmProblems ? n_runs - r0 : msf::kMaxGemmProblems;
+        if (!msf::msp_embed_supported(runs + r0, n, E)) return MSF_ERR_UNSUPPORTED;
+    }
+    for (int r0 = 0; r0 < n_code; r0 += msf::kMaxGemmProblems) {
+        const int n = n_code - r0 < msf::kMaxGemmProblems ? n_code - r0 : msf::kMaxGemmProblems;
+        cudaError_t e = msf::launch_msp_embed(code_runs + r0, n, sh, msf::kTierCodeCols, latent, codes,
+                                              codes_bstride, p.B, msf::status_word(p), s);
+        if (e != cudaSuccess) return cuda_status(e);
+    }
+    for (int r0 = 0; r0 < n_runs; r0 += msf::kMaxGemmProblems) {
+        const int n = n_runs - r0 < msf::kMaxGemmProblems ? n_runs - r0 : msf::kMaxGemmProblems;
+        cudaError_t e = msf::launch_msp_embed(runs + r0, n, sh, E, latent, tokens, (long long)p.N * E, p.B,
+                                              msf::status_word(p), s);
+        if (e != cudaSuccess) return cuda_status(e);
+    }
+    return MSF_OK;
+}
+
+extern "C" msf_status msf_unpatchify_tier(msf_plan_t plan, int32_t position, const void* tokens,
+                                          const void* latent_in, const msf_tier_module* tier,
+                                          void* latent_out, void* stream) {
+    if (!plan || !tokens || !tier || !latent_out) return MSF_ERR_INVALID_ARG;
+    const Plan& p = *plan;
+    if (p.d.latent_channels <= 0 || p.d.patch <= 0 || p.d.embed_dim <= 0 || p.elem != 2)
+        return MSF_ERR_UNSUPPORTED;
+    if (position < 0 || position >= p.T) return MSF_ERR_INVALID_ARG;
+    if (!p.bound) return MSF_ERR_STATE;
+    if (!aligned16(tokens) || !aligned16(latent_out) || !tier->w_out || !aligned16(tier->w_out))
+        return MSF_ERR_INVALID_ARG;
+    if (!tier_lora_ok(tier->out_down, tier->out_up, tier->lora_rank)) return MSF_ERR_INVALID_ARG;
+    if (tier->residual && (!latent_in || !aligned16(latent_in) || !aligned16(tier->residual)))
+        return MSF_ERR_INVALID_ARG;
+    const msf::MspShape sh = msp_shape(p);
+    cudaStream_t s = (cudaStream_t)stream;
+    const int P = p.d.patch * p.d.scales[position];
+    const int F = sh.C * P * P;
+    const int E = p.d.embed_dim;
+    const int M = p.st_n[position];
+    const long long per = (long long)sh.C * sh.Hl * sh.Wl;
+    if (!msf::msp_deembed_supported(M, F, E)) return MSF_ERR_UNSUPPORTED;
+    char* codes = msf::tier_codes(p);
+    msf::DeembedTier extra;
+    if (tier->out_down) {
+        // codes = gamma * h A^T for the state's tokens (columns past r zero)
+        msf::GemmTcArgs g;
+        g.A = (const char*)tokens + (size_t)p.st_off[position] * E * 2;
+        g.B = tier->out_down;
+        g.C = codes + (size_t)p.st_off[position] * msf::kTierCodeCols * 2;
+        g.M = M;
+        g.N = msf::kTierCodeCols;
+        g.K = E;
+        g.lda = E;
+        g.ldb = E;
+        g.ldc = msf::kTierCodeCols;
+        g.a_bstride = (long long)p.N * E;
+        g.c_bstride = (long long)p.N * msf::kTierCodeCols;
+        g.status = msf::status_word(p);
+        g.alpha = tier->lora_scale;
+        g.b_rows = tier->lora_rank;
+        if (!msf::gemm_tc_supported(g)) return MSF_ERR_UNSUPPORTED;
+        cudaError_t e = msf::launch_gemm_tc(g, p.B, s);
+        if (e != cudaSuccess) return cuda_status(e);
+        extra.codes = codes;
+        extra.codes_bstride = (long long)p.N * msf::kTierCodeCols;
+        extra.up = tier->out_up;
+        extra.rank = tier->lora_rank;
+    }
+    if (tier->residual) {
+        // the window's raw patch vectors; the state's block feeds the residual
+        char* raw = msf::msp_scratch(p);
+        cudaError_t e = msf::launch_patchify_raw(latent_in, raw, sh, p.B, true, s);
+        if (e != cudaSuccess) return cuda_status(e);
+        extra.xraw = raw + (size_t)position * per * 2;
+        extra.xraw_bstride = (long long)p.T * per;
+        extra.residual = tier->residual;
+    }
+    return cuda_status(msf::launch_msp_deembed(tokens, (long long)p.N * E, p.N, p.st_off[position], tier->w_out,
+                                               M, F, E, sh, P, latent_out, p.B, msf::status_word(p), s,
+                                               &extra));
+}
+
+namespace {
 // Waits on a barrier that nothing arrives at; the bounded wait must give up.
 __global__ void wait_timeout_selftest_kernel(unsigned int* status, long long limit) {
     __shared__ uint64_t bar;

@@ -49,6 +49,7 @@ struct GemmTcProblem {
     __nv_bfloat16* C;     // splits == 1: bf16 output
     long long ldc;        // elements
     long long c_bstride;  // elements
+    float alpha;          // accumulator scale
 };
 struct GemmTcParams {
     int n_prob;
@@ -175,7 +176,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     uint32_t pk[16];
 #pragma unroll
                     for (int e = 0; e < 16; ++e)
-                        pk[e] = ptx::pack_bf16(__uint_as_float(v[2 * e]), __uint_as_float(v[2 * e + 1]));
+                        pk[e] = ptx::pack_bf16(P.alpha * __uint_as_float(v[2 * e]),
+                                               P.alpha * __uint_as_float(v[2 * e + 1]));
                     const int ncol = n0 + c * 32;
                     if (store && ncol + 32 <= P.N) {
                         uint4* d4 = reinterpret_cast<uint4*>(crow + c * 32);
@@ -195,6 +197,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ptx::tmem_ld32(taddr + c * 32, v);
                     ptx::tmem_wait_ld();
                     const int ncol = n0 + c * 32;
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) v[e] = __float_as_uint(P.alpha * __uint_as_float(v[e]));
                     if (store && ncol + 32 <= P.N) {
                         float4* d4 = reinterpret_cast<float4*>(crow + c * 32);
 #pragma unroll
@@ -255,7 +259,7 @@ cudaError_t launch_bn(const GemmTcArgs* gs, int n, int batch, int splits, cudaSt
                 abox, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                 CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return cudaErrorInvalidValue;
-        cuuint64_t bdims[2] = {(cuuint64_t)g.K, (cuuint64_t)g.N};
+        cuuint64_t bdims[2] = {(cuuint64_t)g.K, (cuuint64_t)(g.b_rows > 0 ? g.b_rows : g.N)};
         cuuint64_t bstrides[1] = {(cuuint64_t)g.ldb * 2};
         cuuint32_t bbox[2] = {64, (cuuint32_t)BN};
         if (enc(&maps.b[i], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(g.B), bdims, bstrides,
@@ -266,6 +270,7 @@ cudaError_t launch_bn(const GemmTcArgs* gs, int n, int batch, int splits, cudaSt
         pr.M = g.M;
         pr.N = g.N;
         pr.K = g.K;
+        pr.alpha = g.alpha;
         pr.m_tiles = (g.M + 127) / 128;
         pr.tile_base = tiles;
         pr.C = (__nv_bfloat16*)g.C;

@@ -22,6 +22,11 @@ struct GemmTcArgs {
     float* C32 = nullptr;
     int max_splits = 1;
     mutable int splits_used = 1;
+    // Scale applied to the accumulator before the output is written.
+    float alpha = 1.0f;
+    // Rows of B actually present (0: N). Rows [b_rows, N) read as zeros, so
+    // output columns past b_rows are written as zeros.
+    int b_rows = 0;
 };
 
 constexpr int kMaxGemmProblems = 4;

@@ -60,7 +60,8 @@ struct msf_plan {
 namespace msf {
 using Plan = ::msf_plan;
 
-// Workspace layout: [status area | pyramid K | pyramid V | MSP scratch]
+// Workspace layout: [status area | pyramid K | pyramid V | MSP scratch | attention
+// merge counters | attention partial slots | de-embedding split partials | tier codes]
 constexpr size_t kStatusBytes = 256;
 inline size_t round256(size_t x) { return (x + 255) / 256 * 256; }
 inline size_t pyramid_bytes(const Plan& p) {
@@ -91,6 +92,13 @@ inline size_t msp_split_bytes(const Plan& p) {
     size_t per = (size_t)p.d.latent_channels * p.d.patch * p.gh * p.d.patch * p.d.grid_w;
     return round256((size_t)kMaxDeembedSplits * p.B * per * 4);
 }
+// LoRA codes of the tier modules (msf_patchify_tiers, msf_unpatchify_tier):
+// [B, N, 64] bf16, the rank-r code of every window token zero-padded to 64.
+constexpr int kTierCodeCols = 64;
+inline size_t tier_codes_bytes(const Plan& p) {
+    if (p.d.latent_channels <= 0 || p.d.patch <= 0 || p.elem != 2 || p.d.embed_dim <= 0) return 0;
+    return round256((size_t)p.B * p.N * kTierCodeCols * 2);
+}
 // Backward workspace (caller-provided per msf_mssa_backward call):
 // [delta fp32 [B, H, N] | dk_ctx fp32 [B, R, H, D] | dv_ctx fp32 [B, R, H, D]],
 // R = rows of every group's context that come from the window (the rows
@@ -111,7 +119,7 @@ inline size_t bwd_ctx_bytes(const Plan& p) {
 inline size_t bwd_workspace_bytes(const Plan& p) { return bwd_delta_bytes(p) + 2 * bwd_ctx_bytes(p); }
 inline size_t workspace_bytes(const Plan& p) {
     return kStatusBytes + 2 * pyramid_bytes(p) + msp_scratch_bytes(p) + attn_counter_bytes(p) +
-           attn_partial_bytes(p) + msp_split_bytes(p);
+           attn_partial_bytes(p) + msp_split_bytes(p) + tier_codes_bytes(p);
 }
 inline unsigned int* status_word(const Plan& p) { return (unsigned int*)p.ws; }
 inline char* pyr_k(const Plan& p) { return (char*)p.ws + kStatusBytes; }
@@ -128,6 +136,7 @@ inline float* attn_partials(const Plan& p) {
 inline float* msp_split(const Plan& p) {
     return (float*)((char*)attn_partials(p) + attn_partial_bytes(p));
 }
+inline char* tier_codes(const Plan& p) { return (char*)msp_split(p) + msp_split_bytes(p); }
 
 // Number of context tokens of group gi with the current history count.
 inline int group_nkv(const Plan& p, int gi) {

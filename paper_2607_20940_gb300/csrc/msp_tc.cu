@@ -134,19 +134,24 @@ struct EmbedRun {
     int P;          // patch edge in latent pixels
     int K;          // C * P * P
     int tok_off;    // first token row of the run in the output
+    int lora;       // 1: one more K chunk (LoRA codes x up projection)
+    float scale;    // accumulator scale
 };
 struct EmbedParams {
     int n_runs;
     EmbedRun run[kMaxGemmProblems];
     int T, C, Hl, Wl, E;
+    int n_tiles_n;  // 256-column tiles per 128-row tile: ceil(E / 256)
     const __nv_bfloat16* latent;  // [B, T, C, Hl, Wl]
     __nv_bfloat16* tokens;        // [B, N, E]
     long long tok_bstride;        // elements
     unsigned int* status;
 };
 struct EmbedMaps {
-    CUtensorMap w[kMaxGemmProblems];    // [E, K] weight of each run: dims {K, E}
-    CUtensorMap out[kMaxGemmProblems];  // the run's tokens: dims {E, M, B}, rows past M clipped
+    CUtensorMap w[kMaxGemmProblems];      // [E, K] weight of each run: dims {K, E}
+    CUtensorMap out[kMaxGemmProblems];    // the run's tokens: dims {E, M, B}, rows past M clipped
+    CUtensorMap codes[kMaxGemmProblems];  // LoRA codes of the run's tokens: dims {64, M, B}
+    CUtensorMap up[kMaxGemmProblems];     // LoRA up projection [E, r]: dims {r, E}
 };
 
 // 128 tokens x 256 embedding columns per CTA (one N=256 MMA per K step, half
@@ -171,7 +176,8 @@ __global__ void __launch_bounds__(kThreads, 2)
     const int local = (int)blockIdx.x - R.tile_base;
     const int mt = local % R.m_tiles, nt = local / R.m_tiles;
     const int b = blockIdx.z;
-    const int nk = R.K / 64;
+    const int nk_patch = R.K / 64;      // chunks gathered from the latent
+    const int nk = nk_patch + R.lora;   // plus the LoRA chunk
 
     if (threadIdx.x == 0) {
         abort_flag = 0;
@@ -210,7 +216,10 @@ __global__ void __launch_bounds__(kThreads, 2)
                     break;
                 }
                 ptx::mbar_arrive_expect_tx(&b_full[st], kBBytes);
-                ptx::tma_load_2d(sB + st * kBBytes, &maps.w[ri], &b_full[st], kc * 64, nt * kEmbedBN);
+                if (kc < nk_patch)
+                    ptx::tma_load_2d(sB + st * kBBytes, &maps.w[ri], &b_full[st], kc * 64, nt * kEmbedBN);
+                else
+                    ptx::tma_load_2d(sB + st * kBBytes, &maps.up[ri], &b_full[st], 0, nt * kEmbedBN);
                 ++issued;
             }
             if (!ok) {
@@ -264,12 +273,12 @@ __global__ void __launch_bounds__(kThreads, 2)
         const size_t plane = (size_t)p.Hl * p.Wl;
         bool ok = true;
         if (P == 2) {
-            ok = gather_row<2, uint32_t>(sA, a_full, a_empty, base, plane, p.Wl, r, nk, valid, abort_p);
+            ok = gather_row<2, uint32_t>(sA, a_full, a_empty, base, plane, p.Wl, r, nk_patch, valid, abort_p);
         } else if (P == 4) {
-            ok = gather_row<4, uint2>(sA, a_full, a_empty, base, plane, p.Wl, r, nk, valid, abort_p);
+            ok = gather_row<4, uint2>(sA, a_full, a_empty, base, plane, p.Wl, r, nk_patch, valid, abort_p);
         } else if (P == 8) {
-            ok = gather_row<8, uint4>(sA, a_full, a_empty, base, plane, p.Wl, r, nk, valid, abort_p);
-        } else for (int kc = 0; kc < nk; ++kc) {
+            ok = gather_row<8, uint4>(sA, a_full, a_empty, base, plane, p.Wl, r, nk_patch, valid, abort_p);
+        } else for (int kc = 0; kc < nk_patch; ++kc) {
             const int st = kc % kEmbedStages;
             const uint32_t ph = (uint32_t)((kc / kEmbedStages) & 1);
             ok = ptx::mbar_wait_bounded(&a_empty[st], ph ^ 1u, abort_p, kWaitLimit);
@@ -289,6 +298,22 @@ __global__ void __launch_bounds__(kThreads, 2)
             ptx::fence_proxy_async_smem();  // the tensor core reads through the async proxy
             ptx::mbar_arrive(&a_full[st]);
         }
+        if (ok && R.lora) {
+            // ---- LoRA chunk: the 128 rows' codes arrive by TMA into the A
+            // stage; one thread adds the bytes to the stage's barrier, the
+            // others arrive as for a gathered chunk.
+            const int st = nk_patch % kEmbedStages;
+            const uint32_t ph = (uint32_t)((nk_patch / kEmbedStages) & 1);
+            ok = __all_sync(0xffffffffu, ptx::mbar_wait_bounded(&a_empty[st], ph ^ 1u, abort_p, kWaitLimit));
+            if (ok) {
+                if (r == 0) {
+                    ptx::mbar_arrive_expect_tx(&a_full[st], kChunkA);
+                    ptx::tma_load_3d(sA + st * kChunkA, &maps.codes[ri], &a_full[st], 0, mt * 128, b);
+                } else {
+                    ptx::mbar_arrive(&a_full[st]);
+                }
+            }
+        }
         // ---- epilogue: bf16 tile staged in the (now idle) A and B stages in
         // the 128-byte swizzle layout, then TMA stores of 128 rows x 64 columns.
         ok = ok && ptx::mbar_wait_bounded(&acc_full, 0, abort_p, kWaitLimit);
@@ -302,20 +327,21 @@ __global__ void __launch_bounds__(kThreads, 2)
                 ptx::tmem_ld32(taddr + c * 32, v);
                 ptx::tmem_wait_ld();
                 unsigned char* stage = sA + (c / 2) * kChunkA;
+                const float sc = R.scale;
 #pragma unroll
                 for (int e = 0; e < 4; ++e)
-                    *reinterpret_cast<uint4*>(stage + swz_offset(r, (c % 2) * 32 + 8 * e)) =
-                        make_uint4(ptx::pack_bf16(__uint_as_float(v[8 * e]), __uint_as_float(v[8 * e + 1])),
-                                   ptx::pack_bf16(__uint_as_float(v[8 * e + 2]), __uint_as_float(v[8 * e + 3])),
-                                   ptx::pack_bf16(__uint_as_float(v[8 * e + 4]), __uint_as_float(v[8 * e + 5])),
-                                   ptx::pack_bf16(__uint_as_float(v[8 * e + 6]), __uint_as_float(v[8 * e + 7])));
+                    *reinterpret_cast<uint4*>(stage + swz_offset(r, (c % 2) * 32 + 8 * e)) = make_uint4(
+                        ptx::pack_bf16(sc * __uint_as_float(v[8 * e]), sc * __uint_as_float(v[8 * e + 1])),
+                        ptx::pack_bf16(sc * __uint_as_float(v[8 * e + 2]), sc * __uint_as_float(v[8 * e + 3])),
+                        ptx::pack_bf16(sc * __uint_as_float(v[8 * e + 4]), sc * __uint_as_float(v[8 * e + 5])),
+                        ptx::pack_bf16(sc * __uint_as_float(v[8 * e + 6]), sc * __uint_as_float(v[8 * e + 7])));
             }
             ptx::fence_proxy_async_smem();
         }
         // The four epilogue warps meet before one thread stores the tile.
         ok = ptx::named_bar_and(1, 128, ok);
         if (ok && warp == 4 && lane == 0) {
-            for (int h = 0; h < kEmbedBN / 64; ++h)
+            for (int h = 0; h < kEmbedBN / 64 && nt * kEmbedBN + h * 64 < p.E; ++h)
                 ptx::tma_store_3d(&maps.out[ri], sA + h * kChunkA, nt * kEmbedBN + h * 64, mt * 128, b);
             ptx::bulk_commit();
             ptx::bulk_wait_read_all();
@@ -349,6 +375,9 @@ constexpr int kDePartStride = kDeBN + 4;  // floats per staged row (padding spre
 struct DeembedParams {
     int M;              // tokens of the position (per stream)
     int K;              // embedding width E
+    int nk_all;         // K chunks: E / 64 token chunks, then the tier's extras
+    int lora;           // 1: chunk E/64 is (LoRA codes, up projection)
+    int nk_res;         // then this many (raw patch vector, latent residual) chunks
     int m_tiles;
     int splits;         // cluster size along y
     int P, gw, C, Hl, Wl;
@@ -357,8 +386,12 @@ struct DeembedParams {
     unsigned int* status;
 };
 struct DeembedMaps {
-    CUtensorMap a;  // tokens {E, rows, B}
-    CUtensorMap b;  // W_out {E, F}
+    CUtensorMap a;      // tokens {E, rows, B}
+    CUtensorMap b;      // W_out {E, F}
+    CUtensorMap codes;  // LoRA codes of the tokens {64, rows, B}
+    CUtensorMap up;     // LoRA up projection [F, r]: {r, F}
+    CUtensorMap xraw;   // the state's raw patch vectors {F, M, B}
+    CUtensorMap res;    // latent residual [F, F]: {F, F}
 };
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -377,7 +410,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int mt = tile % p.m_tiles, nt = tile / p.m_tiles;
     const int split = (int)ptx::cluster_rank();
     const int b = blockIdx.z;
-    const int nk_all = p.K / 64;
+    const int nk_all = p.nk_all;
+    const int nk_tok = p.K / 64;
     const int kc0 = (int)((long long)split * nk_all / p.splits);
     const int nk = (int)((long long)(split + 1) * nk_all / p.splits) - kc0;
 
@@ -418,8 +452,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 unsigned char* sa = smem + st * kStageBytes;
                 ptx::mbar_arrive_expect_tx(&full[st], kStageBytes);
-                ptx::tma_load_3d(sa, &maps.a, &full[st], (kc0 + kc) * 64, p.tok_row0 + mt * 128, b);
-                ptx::tma_load_2d(sa + kChunkA, &maps.b, &full[st], (kc0 + kc) * 64, nt * kDeBN);
+                const int g = kc0 + kc;
+                if (g < nk_tok) {
+                    ptx::tma_load_3d(sa, &maps.a, &full[st], g * 64, p.tok_row0 + mt * 128, b);
+                    ptx::tma_load_2d(sa + kChunkA, &maps.b, &full[st], g * 64, nt * kDeBN);
+                } else if (g == nk_tok && p.lora) {
+                    ptx::tma_load_3d(sa, &maps.codes, &full[st], 0, p.tok_row0 + mt * 128, b);
+                    ptx::tma_load_2d(sa + kChunkA, &maps.up, &full[st], 0, nt * kDeBN);
+                } else {
+                    const int j = g - nk_tok - p.lora;
+                    ptx::tma_load_3d(sa, &maps.xraw, &full[st], j * 64, mt * 128, b);
+                    ptx::tma_load_2d(sa + kChunkA, &maps.res, &full[st], j * 64, nt * kDeBN);
+                }
                 ++issued;
             }
             if (!ok) {
@@ -528,10 +572,14 @@ constexpr int kEmbedSmem = kEmbedStages * (kChunkA + kEmbedBN * 128) + 1024;
 }  // namespace
 
 bool msp_embed_supported(const MspEmbedRun* runs, int n, int E) {
-    if (n < 1 || n > kMaxGemmProblems || E % kEmbedBN != 0) return false;
+    if (n < 1 || n > kMaxGemmProblems || E % 64 != 0 || E <= 0) return false;
     for (int i = 0; i < n; ++i) {
         const MspEmbedRun& r = runs[i];
         if (r.K % 64 != 0 || r.P < 1 || 64 % r.P != 0 || ((uintptr_t)r.w & 15) || r.M <= 0) return false;
+        if (r.w_rows < 0 || r.w_rows > E) return false;
+        if (r.lora_up && (r.rank < 8 || r.rank > 64 || r.rank % 8 != 0 || !r.codes ||
+                          ((uintptr_t)r.lora_up & 15) || ((uintptr_t)r.codes & 15) || r.codes_bstride % 8))
+            return false;
     }
     return true;
 }
@@ -546,7 +594,21 @@ cudaError_t launch_msp_embed(const MspEmbedRun* runs, int n, const MspShape& sh,
     int tiles = 0;
     for (int i = 0; i < n; ++i) {
         const MspEmbedRun& r = runs[i];
-        if (!encode_2d(&maps.w[i], r.w, r.K, E, (long long)r.K * 2, 64, kEmbedBN)) return cudaErrorInvalidValue;
+        if (!encode_2d(&maps.w[i], r.w, r.K, r.w_rows > 0 ? r.w_rows : E, (long long)r.K * 2, 64, kEmbedBN))
+            return cudaErrorInvalidValue;
+        if (r.lora_up) {
+            EncodeTiledFn enc = encoder();
+            if (!encode_2d(&maps.up[i], r.lora_up, r.rank, E, (long long)r.rank * 2, 64, kEmbedBN))
+                return cudaErrorInvalidValue;
+            cuuint64_t dims[3] = {64, (cuuint64_t)r.M, (cuuint64_t)batch};
+            cuuint64_t strides[2] = {128, (cuuint64_t)r.codes_bstride * 2};
+            cuuint32_t box[3] = {64, 128, 1};
+            cuuint32_t es[3] = {1, 1, 1};
+            if (!enc || enc(&maps.codes[i], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(r.codes), dims,
+                            strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+                return cudaErrorInvalidValue;
+        }
         {
             EncodeTiledFn enc = encoder();
             cuuint64_t dims[3] = {(cuuint64_t)E, (cuuint64_t)r.M, (cuuint64_t)batch};
@@ -569,8 +631,11 @@ cudaError_t launch_msp_embed(const MspEmbedRun* runs, int n, const MspShape& sh,
         R.P = r.P;
         R.K = r.K;
         R.tok_off = r.tok_off;
-        tiles += R.m_tiles * (E / kEmbedBN);
+        R.lora = r.lora_up ? 1 : 0;
+        R.scale = r.scale;
+        tiles += R.m_tiles * ((E + kEmbedBN - 1) / kEmbedBN);
     }
+    p.n_tiles_n = (E + kEmbedBN - 1) / kEmbedBN;
     p.n_runs = n;
     p.T = sh.T;
     p.C = sh.C;
@@ -594,7 +659,7 @@ bool msp_deembed_supported(int M, int F, int E) {
 
 cudaError_t launch_msp_deembed(const void* tokens, long long tok_bstride_elems, int tok_rows, int tok_row0,
                                const void* w_out, int M, int F, int E, const MspShape& sh, int P, void* latent,
-                               int batch, unsigned int* status, cudaStream_t st) {
+                               int batch, unsigned int* status, cudaStream_t st, const DeembedTier* tier) {
     DeembedMaps maps;
     memset(&maps, 0, sizeof(maps));
     EncodeTiledFn enc = encoder();
@@ -610,13 +675,44 @@ cudaError_t launch_msp_deembed(const void* tokens, long long tok_bstride_elems, 
             return cudaErrorInvalidValue;
     }
     if (!encode_2d(&maps.b, w_out, E, F, (long long)E * 2, 64, kDeBN)) return cudaErrorInvalidValue;
+    const bool lora = tier && tier->up;
+    const bool res = tier && tier->residual;
+    if (lora) {
+        EncodeTiledFn enc = encoder();
+        cuuint64_t dims[3] = {64, (cuuint64_t)tok_rows, (cuuint64_t)batch};
+        cuuint64_t strides[2] = {128, (cuuint64_t)tier->codes_bstride * 2};
+        cuuint32_t box[3] = {64, 128, 1};
+        cuuint32_t es[3] = {1, 1, 1};
+        if (!enc || enc(&maps.codes, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(tier->codes), dims,
+                        strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+        if (!encode_2d(&maps.up, tier->up, tier->rank, F, (long long)tier->rank * 2, 64, kDeBN))
+            return cudaErrorInvalidValue;
+    }
+    if (res) {
+        EncodeTiledFn enc = encoder();
+        cuuint64_t dims[3] = {(cuuint64_t)F, (cuuint64_t)M, (cuuint64_t)batch};
+        cuuint64_t strides[2] = {(cuuint64_t)F * 2, (cuuint64_t)tier->xraw_bstride * 2};
+        cuuint32_t box[3] = {64, 128, 1};
+        cuuint32_t es[3] = {1, 1, 1};
+        if (!enc || enc(&maps.xraw, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(tier->xraw), dims,
+                        strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+        if (!encode_2d(&maps.res, tier->residual, F, F, (long long)F * 2, 64, kDeBN)) return cudaErrorInvalidValue;
+    }
+    const int nk_all = E / 64 + (lora ? 1 : 0) + (res ? F / 64 : 0);
     // The largest power of two <= 8 that leaves each split at least one K chunk.
     int splits = 8;
-    while (splits > 1 && splits > E / 64) splits /= 2;
+    while (splits > 1 && splits > nk_all) splits /= 2;
     DeembedParams p;
     memset(&p, 0, sizeof(p));
     p.M = M;
     p.K = E;
+    p.nk_all = nk_all;
+    p.lora = lora ? 1 : 0;
+    p.nk_res = res ? F / 64 : 0;
     p.m_tiles = (M + 127) / 128;
     p.splits = splits;
     p.P = P;

@@ -37,7 +37,8 @@ EXPORTS = (
     "msf_plan_device_status", "msf_kernel_launches", "msf_unpatchify_noalloc",
     "msf_selftest_wait_timeout", "msf_history_commit", "msf_mssa_forward_lse",
     "msf_mssa_backward", "msf_mssa_backward_simt", "msf_history_get", "msf_history_set",
-    "msf_noalloc_device_status", "msf_noalloc_selftest_wait_timeout",
+    "msf_noalloc_device_status", "msf_noalloc_selftest_wait_timeout", "msf_patchify_tiers",
+    "msf_unpatchify_tier",
 )
 
 
@@ -51,6 +52,14 @@ class msf_plan_desc(ctypes.Structure):
         ("softmax_scale", ctypes.c_float), ("latent_channels", ctypes.c_int32),
         ("patch", ctypes.c_int32), ("embed_dim", ctypes.c_int32),
         ("frames_per_state", ctypes.c_int32), ("fused_append", ctypes.c_int32),
+    ]
+
+
+class msf_tier_module(ctypes.Structure):
+    _fields_ = [
+        ("w_embed", ctypes.c_void_p), ("embed_down", ctypes.c_void_p), ("embed_up", ctypes.c_void_p),
+        ("w_out", ctypes.c_void_p), ("out_down", ctypes.c_void_p), ("out_up", ctypes.c_void_p),
+        ("residual", ctypes.c_void_p), ("lora_rank", ctypes.c_int32), ("lora_scale", ctypes.c_float),
     ]
 
 
@@ -107,6 +116,9 @@ def _load():
         "msf_unpatchify_noalloc": (ctypes.c_int, [P, I32, VP, VP, VP, VP]),
         "msf_selftest_wait_timeout": (ctypes.c_int, [P, ctypes.c_int64, VP]),
         "msf_noalloc_device_status": (ctypes.c_int, [VP]),
+        "msf_patchify_tiers": (ctypes.c_int, [P, VP, ctypes.POINTER(ctypes.POINTER(msf_tier_module)), VP,
+                                              VP]),
+        "msf_unpatchify_tier": (ctypes.c_int, [P, I32, VP, VP, ctypes.POINTER(msf_tier_module), VP, VP]),
         "msf_noalloc_selftest_wait_timeout": (ctypes.c_int, [ctypes.c_int64, VP]),
         "msf_history_commit": (ctypes.c_int, [P]),
         "msf_history_get": (ctypes.c_int, [P, ctypes.POINTER(msf_history_state)]),
@@ -202,6 +214,28 @@ def msf_patchify(plan: int, latent, w_tier: Optional[Sequence], tokens, stream=N
 def msf_unpatchify(plan: int, position: int, tokens, w_out, latent_out, stream=None) -> None:
     _check(_lib.msf_unpatchify(plan, position, _ptr(tokens), _ptr(w_out), _ptr(latent_out),
                                _stream(stream)), "msf_unpatchify")
+
+
+def tier_module(w_embed, w_out, embed_down=None, embed_up=None, out_down=None, out_up=None,
+                residual=None, lora_rank=0, lora_scale=1.0) -> msf_tier_module:
+    """An msf_tier_module of device tensors (nn.Linear layouts, see msf.h)."""
+    return msf_tier_module(_ptr(w_embed), _ptr(embed_down), _ptr(embed_up), _ptr(w_out),
+                           _ptr(out_down), _ptr(out_up), _ptr(residual), int(lora_rank),
+                           float(lora_scale))
+
+
+def msf_patchify_tiers(plan: int, latent, tiers: Sequence[msf_tier_module], tokens, stream=None) -> None:
+    """tiers: one msf_tier_module per window position (the same object for
+    positions that share a tier)."""
+    ptrs = (ctypes.POINTER(msf_tier_module) * len(tiers))(*[ctypes.pointer(t) for t in tiers])
+    _check(_lib.msf_patchify_tiers(plan, _ptr(latent), ptrs, _ptr(tokens), _stream(stream)),
+           "msf_patchify_tiers")
+
+
+def msf_unpatchify_tier(plan: int, position: int, tokens, latent_in, tier: msf_tier_module,
+                        latent_out, stream=None) -> None:
+    _check(_lib.msf_unpatchify_tier(plan, position, _ptr(tokens), _ptr(latent_in), ctypes.byref(tier),
+                                    _ptr(latent_out), _stream(stream)), "msf_unpatchify_tier")
 
 
 def msf_kv_resample(plan: int, k_win, v_win, flags: int = MSF_RESAMPLE_FULL, stream=None) -> None:
@@ -347,6 +381,12 @@ class Plan:
 
     def unpatchify(self, position, tokens, w_out, latent_out, stream=None):
         msf_unpatchify(self.handle, position, tokens, w_out, latent_out, stream)
+
+    def patchify_tiers(self, latent, tiers, tokens, stream=None):
+        msf_patchify_tiers(self.handle, latent, tiers, tokens, stream)
+
+    def unpatchify_tier(self, position, tokens, latent_in, tier, latent_out, stream=None):
+        msf_unpatchify_tier(self.handle, position, tokens, latent_in, tier, latent_out, stream)
 
     def kv_resample(self, k_win, v_win, flags=MSF_RESAMPLE_FULL, stream=None):
         msf_kv_resample(self.handle, k_win, v_win, flags, stream)
