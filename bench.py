@@ -385,8 +385,9 @@ def other_configs(msf, synth, dev, flush, peaks, rank):
     with the row log-sum-exp and the MSSA gradient), the paper's chunked layout
     (3 latent frames per state) beside its all-fine window, the STRIDED Subsample
     reading at the 480p layer, the B=4 streaming rollout
-    (120 steps, history 2 -> capacity 4), the 30-layer window pass, and the
-    bandwidth of the pyramid and embedding kernels."""
+    (120 steps, history 2 -> capacity 4), the 30-layer window pass, the
+    bandwidth of the pyramid and embedding kernels, and the coarse tiers'
+    modules (LoRA adapters and latent residual) beside the plain projections."""
     import torch
     out = {}
     hbm = float(peaks["hbm_gbs"])
@@ -645,6 +646,56 @@ def other_configs(msf, synth, dev, flush, peaks, rank):
     out["bandwidth"] = bw
     out["bandwidth_note"] = ("event time per call including ~4 us of launch latency; bytes are the "
                              "algorithmic reads + writes")
+
+    # ---- tier modules (Sec. 4.1): coarse tiers with rank-32 LoRA on the embedding and
+    # de-embedding and a latent residual branch, beside the plain tier projections
+    tier = {}
+    rank = 32
+    for w in (synth.LAYER_480P, synth.STREAM_480P):
+        plan_t, tt = setup(w, embed=True)
+        B, N, E, C = w.batch, plan_t.info.n_tokens, w.embed_dim, w.latent_channels
+        mi_t = synth.msp_inputs(w, torch.bfloat16)
+        ti = synth.tier_inputs(w, rank, torch.bfloat16)
+        lat_t = mi_t["latent"].to(dev)
+        keep, mods, plain_w = [], {}, {}
+        for sc in sorted(set(w.scales)):
+            w_emb = mi_t["w_tier"][sc].t().contiguous().to(dev)
+            plain_w[sc] = w_emb
+            if sc == 1:
+                w_o = mi_t["w_out"].t().contiguous().to(dev)
+                mods[sc] = msf.tier_module(w_emb, w_o)
+                keep += [w_emb, w_o]
+                continue
+            t = {k: (v.t().contiguous().to(dev) if torch.is_tensor(v) else v) for k, v in ti[sc].items()}
+            mods[sc] = msf.tier_module(w_emb, t["w_out"], embed_down=t["lora_a"], embed_up=t["lora_b"],
+                                       out_down=t["out_a"], out_up=t["out_b"], residual=t["residual"],
+                                       lora_rank=rank, lora_scale=t["gamma"])
+            keep += [w_emb] + [v for v in t.values() if torch.is_tensor(v)]
+            plain_w[("out", sc)] = t["w_out"]
+        tok_t = torch.empty((B, N, E), dtype=torch.bfloat16, device=dev)
+        emb_base = _timed(lambda: plan_t.patchify(lat_t, [plain_w[sc] for sc in w.scales], tok_t), flush)
+        emb_tier = _timed(lambda: plan_t.patchify_tiers(lat_t, [mods[sc] for sc in w.scales], tok_t), flush)
+        pos = w.scales.index(2)
+        Hl, Wl = w.grid_h * w.patch, w.grid_w * w.patch
+        lat_o = torch.empty((B, C, Hl, Wl), dtype=torch.bfloat16, device=dev)
+        de_base = _timed(lambda: plan_t.unpatchify(pos, tok_t, plain_w[("out", 2)], lat_o), flush)
+        de_tier = _timed(lambda: plan_t.unpatchify_tier(pos, tok_t, lat_t, mods[2], lat_o), flush)
+        if plan_t.device_status() != msf.MSF_OK:
+            raise RuntimeError("device status error (tier modules)")
+        n_coarse = sum(plan_t.info.state_tokens[l] for l, sc in enumerate(w.scales) if sc > 1)
+        M = plan_t.info.state_tokens[pos]
+        emb_bytes = lat_t.numel() * 2 + tok_t.numel() * 2 + 2 * B * n_coarse * 64 * 2
+        de_bytes = B * M * E * 2 + 2 * B * C * Hl * Wl * 2 + B * M * 64 * 2 * 2
+        tier[w.name] = {
+            "lora_rank": rank, "embed_plain_us": emb_base * 1e3, "embed_tier_us": emb_tier * 1e3,
+            "embed_tier_gbs": emb_bytes / (emb_tier * 1e-3) / 1e9,
+            "deembed_position": pos, "deembed_plain_us": de_base * 1e3, "deembed_tier_us": de_tier * 1e3,
+            "deembed_tier_gbs": de_bytes / (de_tier * 1e-3) / 1e9,
+            "launches": {"embed_tier": 2, "deembed_tier": 3},
+        }
+        del keep
+        plan_t.close()
+    out["tier_module"] = tier
     return out
 
 

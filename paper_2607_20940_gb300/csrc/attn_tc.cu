@@ -246,6 +246,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Merges of split items go to the helper warps while whole items follow.
     const bool helper_merges = p.dp_rounds > 0;
 
+
     if (threadIdx.x == 0) {
         abort_flag = 0;
         merge_flag = 0;
@@ -733,11 +734,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (store && p.lse)
                     p.lse[((size_t)pc.b * p.H + pc.h) * p.N + qrow] =
                         (m_used + log2f(l)) * 0.6931471805599453f;
+                // The whole row of O in one batch of TMEM loads and one wait (the
+                // registers of S are free here), then packed and stored.
+                uint32_t ob[D / 32][32];
+#pragma unroll
+                for (int c = 0; c < D / 32; ++c) ptx::tmem_ld32(tO + c * 32, ob[c]);
+                ptx::tmem_wait_ld();
 #pragma unroll
                 for (int c = 0; c < D / 32; ++c) {
-                    uint32_t o[32];
-                    ptx::tmem_ld32(tO + c * 32, o);
-                    ptx::tmem_wait_ld();
+                    const uint32_t* o = ob[c];
                     uint32_t pk[16];
 #pragma unroll
                     for (int e = 0; e < 16; ++e)
@@ -799,11 +804,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!fast) {
                     float* ps = p.partials + (size_t)slot * C::kSlotFloats;
                     float4* po = reinterpret_cast<float4*>(ps) + rr;
+                    uint32_t ob[D / 32][32];
+#pragma unroll
+                    for (int c = 0; c < D / 32; ++c) ptx::tmem_ld32(tO + c * 32, ob[c]);
+                    ptx::tmem_wait_ld();
 #pragma unroll
                     for (int c = 0; c < D / 32; ++c) {
-                        uint32_t o[32];
-                        ptx::tmem_ld32(tO + c * 32, o);
-                        ptx::tmem_wait_ld();
+                        const uint32_t* o = ob[c];
 #pragma unroll
                         for (int e = 0; e < 8; ++e)
                             po[(size_t)(c * 8 + e) * 2 * kBlockM] =
@@ -812,15 +819,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     ps[C::kSlotML + rr] = m_used;
                     ps[C::kSlotML + 2 * kBlockM + rr] = l;
-                    __threadfence();
                     __syncwarp();
-                    if (lane == 0) ptx::mbar_arrive(&epi_written);
+                    if (lane == 0) ptx::mbar_arrive(&epi_written);  // release, CTA scope
                     const uint32_t pw = (uint32_t)(nwritten & 1);
                     ++nwritten;
                     if (warp == 4 && lane == 0 && (!merger || to_helper)) {
-                        // All 256 rows are written and fenced: count them in, or
-                        // hand the merge to the helper warps.
+                        // All 256 rows are written (acquired through the barrier);
+                        // one GPU-scope fence, which is cumulative over the writes
+                        // of the eight warps, orders them before the count or the
+                        // hand-over to the helper warps.
                         bool okw = ptx::mbar_wait_bounded(&epi_written, pw, abort_p, p.wait_limit);
+                        if (okw) __threadfence();
                         if (okw && !merger) atomicAdd(cnt, 1u << 16);
                         if (okw && to_helper) {
                             okw = ptx::mbar_wait_bounded(&job_empty, (uint32_t)((njob & 1) ^ 1), abort_p,
