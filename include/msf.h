@@ -211,6 +211,18 @@ msf_status msf_plan_bind(msf_plan_t plan, void* workspace, size_t workspace_byte
 msf_status msf_patchify(msf_plan_t plan, const void* latent, const void* const* w_tier,
                         void* tokens, void* stream);
 
+/* msf_patchify with tier weights (w_tier != NULL) and msf_kv_resample(k_win,
+ * v_win, flags) in one launch, for bf16 plans with an embedding: the tokens,
+ * the pyramid and (fused_append) the staged head are exactly those of the
+ * two calls. The two read and write disjoint buffers, so the pooling runs on
+ * the CTA slots of the wave that the embedding tiles leave free (the
+ * embedding holds two CTAs per SM) instead of a second launch. Errors:
+ * INVALID_ARG, UNSUPPORTED (fp32 plan, no embedding, a shape the fused
+ * embedding kernel does not take), STATE (not bound), CUDA. */
+msf_status msf_patchify_resample(msf_plan_t plan, const void* latent, const void* const* w_tier,
+                                 void* tokens, const void* k_win, const void* v_win, int32_t flags,
+                                 void* stream);
+
 /* MSP unpatchify of window position `position` (0-based): the inverse of
  * msf_patchify for that state.
  *   w_out == NULL: tokens is the raw layout [B, T, C*Hl*Wl] of msf_patchify.

@@ -699,6 +699,68 @@ extern "C" msf_status msf_patchify(msf_plan_t plan, const void* latent, const vo
     return MSF_OK;
 }
 
+extern "C" msf_status msf_patchify_resample(msf_plan_t plan, const void* latent, const void* const* w_tier,
+                                            void* tokens, const void* k_win, const void* v_win, int32_t flags,
+                                            void* stream) {
+    if (!plan || !latent || !tokens || !w_tier || !k_win || !v_win) return MSF_ERR_INVALID_ARG;
+    const Plan& p = *plan;
+    if (p.d.latent_channels <= 0 || p.d.patch <= 0 || p.d.embed_dim <= 0 || p.elem != 2)
+        return MSF_ERR_UNSUPPORTED;
+    if (!p.bound) return MSF_ERR_STATE;
+    if (!aligned16(latent) || !aligned16(tokens) || !aligned16(k_win) || !aligned16(v_win))
+        return MSF_ERR_INVALID_ARG;
+    for (int l = 0; l < p.T; ++l)
+        if (!w_tier[l] || !aligned16(w_tier[l])) return MSF_ERR_INVALID_ARG;
+    if (flags != MSF_RESAMPLE_FULL && flags != MSF_RESAMPLE_WINDOW_ONLY) return MSF_ERR_INVALID_ARG;
+    const bool with_hist = flags == MSF_RESAMPLE_FULL;
+    if (count_window_jobs(p, with_hist) > msf::kMaxPoolJobs) return MSF_ERR_UNSUPPORTED;
+    const msf::MspShape sh = msp_shape(p);
+    const int E = p.d.embed_dim;
+    msf::MspEmbedRun runs[MSF_MAX_STATES];
+    int n_runs = 0, tiles = 0;
+    for (int l0 = 0; l0 < p.T;) {
+        int l1 = l0 + 1;
+        while (l1 < p.T && p.d.scales[l1] == p.d.scales[l0] && w_tier[l1] == w_tier[l0]) ++l1;
+        msf::MspEmbedRun& r = runs[n_runs++];
+        r.w = w_tier[l0];
+        r.P = p.d.patch * p.d.scales[l0];
+        r.K = sh.C * r.P * r.P;
+        r.l0 = l0;
+        r.n_l = p.st_n[l0];
+        r.M = p.st_off[l1 - 1] + p.st_n[l1 - 1] - p.st_off[l0];
+        r.gw = sh.Wl / r.P;
+        r.tok_off = p.st_off[l0];
+        if (n_runs <= msf::kMaxGemmProblems) tiles += ((r.M + 127) / 128) * ((E + 255) / 256);
+        l0 = l1;
+    }
+    for (int r0 = 0; r0 < n_runs; r0 += msf::kMaxGemmProblems) {
+        const int n = n_runs - r0 < msf::kMaxGemmProblems ? n_runs - r0 : msf::kMaxGemmProblems;
+        if (!msf::msp_embed_supported(runs + r0, n, E)) return MSF_ERR_UNSUPPORTED;
+    }
+    msf::PoolBatch jb;
+    memset(&jb, 0, sizeof(jb));
+    jb.row_vecs = (int)(row_bytes(p) / 16);
+    jb.mode = p.d.resample;
+    add_window_jobs(p, k_win, v_win, with_hist, jb);
+    // Pool CTAs per stream: one 256-thread block per 256 tasks, as the pool
+    // kernel launches them; they come first in the grid, and the embedding
+    // tiles take the slots they free.
+    int max_n = 0;
+    for (int k = 0; k < jb.n; ++k) max_n = jb.j[k].out_n > max_n ? jb.j[k].out_n : max_n;
+    long long pool_ctas = ((long long)jb.n * max_n * (jb.row_vecs / 2) + 255) / 256;
+    if (pool_ctas < 1) pool_ctas = 1;
+    (void)tiles;
+    cudaError_t e = cudaSuccess;
+    cudaStream_t s = (cudaStream_t)stream;
+    for (int r0 = 0; r0 < n_runs; r0 += msf::kMaxGemmProblems) {
+        const int n = n_runs - r0 < msf::kMaxGemmProblems ? n_runs - r0 : msf::kMaxGemmProblems;
+        e = msf::launch_msp_embed(runs + r0, n, sh, E, latent, tokens, (long long)p.N * E, p.B, msf::status_word(p), s,
+                                  r0 == 0 && jb.n > 0 ? &jb : nullptr, (int)pool_ctas);
+        if (e != cudaSuccess) return cuda_status(e);
+    }
+    return MSF_OK;
+}
+
 extern "C" msf_status msf_unpatchify(msf_plan_t plan, int32_t position, const void* tokens,
                                      const void* w_out, void* latent_out, void* stream) {
     if (!plan || !tokens || !latent_out) return MSF_ERR_INVALID_ARG;

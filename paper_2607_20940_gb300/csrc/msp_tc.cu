@@ -23,6 +23,7 @@
 #include "gemm_tc.h"
 #include "kernels.h"
 #include "msp_tc.h"
+#include "pool.cuh"
 #include "ptx.cuh"
 
 namespace msf {
@@ -142,6 +143,9 @@ struct EmbedParams {
     EmbedRun run[kMaxGemmProblems];
     int T, C, Hl, Wl, E;
     int n_tiles_n;  // 256-column tiles per 128-row tile: ceil(E / 256)
+    int n_embed_tiles;  // embedding tiles per stream
+    int pool_ctas;      // CTAs [0, pool_ctas) of a stream run the pyramid jobs; the rest embed
+    int pool_tasks;     // vector-pair tasks per pyramid job
     const __nv_bfloat16* latent;  // [B, T, C, Hl, Wl]
     __nv_bfloat16* tokens;        // [B, N, E]
     long long tok_bstride;        // elements
@@ -158,7 +162,20 @@ struct EmbedMaps {
 // the gathers of 128-column tiles); two CTAs per SM (97 KB of shared memory
 // each), so the 480p window's 210 tiles run in one wave on 152 SMs.
 __global__ void __launch_bounds__(kThreads, 2)
-    msp_embed_kernel(const __grid_constant__ EmbedMaps maps, const __grid_constant__ EmbedParams p) {
+    msp_embed_kernel(const __grid_constant__ EmbedMaps maps, const __grid_constant__ EmbedParams p,
+                     const __grid_constant__ PoolBatch pool) {
+    if ((int)blockIdx.x < p.pool_ctas) {
+        // ---- K/V pyramid jobs in the first CTAs of the launch: the same
+        // per-thread pooling as pool_kernel, strided over the pool CTAs of
+        // this stream (the two parts read and write disjoint buffers).
+        ptx::grid_dep_wait();
+        ptx::grid_dep_launch();
+        const int stride = p.pool_ctas * kThreads;
+        const int total = pool.n * p.pool_tasks;
+        for (int t = (int)blockIdx.x * kThreads + (int)threadIdx.x; t < total; t += stride)
+            pool_task<__nv_bfloat16>(pool, t / p.pool_tasks, blockIdx.z, t % p.pool_tasks);
+        return;
+    }
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     unsigned char* sA = smem;                                   // [stage][chunk]
@@ -170,10 +187,11 @@ __global__ void __launch_bounds__(kThreads, 2)
     __shared__ int abort_flag;
 
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    const int tile = (int)blockIdx.x - p.pool_ctas;
     int ri = 0;
-    while (ri < p.n_runs - 1 && (int)blockIdx.x >= p.run[ri + 1].tile_base) ++ri;
+    while (ri < p.n_runs - 1 && tile >= p.run[ri + 1].tile_base) ++ri;
     const EmbedRun& R = p.run[ri];
-    const int local = (int)blockIdx.x - R.tile_base;
+    const int local = tile - R.tile_base;
     const int mt = local % R.m_tiles, nt = local / R.m_tiles;
     const int b = blockIdx.z;
     const int nk_patch = R.K / 64;      // chunks gathered from the latent
@@ -586,7 +604,7 @@ bool msp_embed_supported(const MspEmbedRun* runs, int n, int E) {
 
 cudaError_t launch_msp_embed(const MspEmbedRun* runs, int n, const MspShape& sh, int E, const void* latent,
                              void* tokens, long long tok_bstride, int batch, unsigned int* status,
-                             cudaStream_t st) {
+                             cudaStream_t st, const PoolBatch* pool, int pool_ctas) {
     EmbedMaps maps;
     memset(&maps, 0, sizeof(maps));
     EmbedParams p;
@@ -648,8 +666,19 @@ cudaError_t launch_msp_embed(const MspEmbedRun* runs, int n, const MspShape& sh,
     p.status = status;
     cudaError_t e = set_smem_attr((const void*)msp_embed_kernel, kEmbedSmem, 100);
     if (e != cudaSuccess) return e;
-    return launch_pdl(msp_embed_kernel, dim3((unsigned)tiles, 1, (unsigned)batch), dim3(kThreads), kEmbedSmem,
-                      st, maps, p);
+    p.n_embed_tiles = tiles;
+    PoolBatch pb;
+    if (pool && pool->n > 0 && pool_ctas > 0) {
+        pb = *pool;
+        int max_n = 0;
+        for (int k = 0; k < pb.n; ++k) max_n = pb.j[k].out_n > max_n ? pb.j[k].out_n : max_n;
+        p.pool_tasks = max_n * (pb.row_vecs / 2);
+        p.pool_ctas = pool_ctas;
+    } else {
+        memset(&pb, 0, sizeof(pb));
+    }
+    return launch_pdl(msp_embed_kernel, dim3((unsigned)(tiles + p.pool_ctas), 1, (unsigned)batch), dim3(kThreads),
+                      kEmbedSmem, st, maps, p, pb);
 }
 
 

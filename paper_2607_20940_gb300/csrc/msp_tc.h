@@ -32,10 +32,13 @@ struct MspEmbedRun {
 };
 
 bool msp_embed_supported(const MspEmbedRun* runs, int n, int E);
-// Up to kMaxGemmProblems runs in one launch.
+// Up to kMaxGemmProblems runs in one launch. With `pool` (bf16 jobs) the
+// same launch also runs those K/V pyramid jobs on `pool_ctas` extra CTAs per
+// stream: they read and write buffers the embedding does not touch, so the
+// two share the SMs of one wave instead of two launches.
 cudaError_t launch_msp_embed(const MspEmbedRun* runs, int n, const MspShape& sh, int E, const void* latent,
                              void* tokens, long long tok_bstride, int batch, unsigned int* status,
-                             cudaStream_t st);
+                             cudaStream_t st, const PoolBatch* pool = nullptr, int pool_ctas = 0);
 
 // The coarse tier's extras of a de-embedding (Sec. 4.1): K chunks added to
 // the E / 64 token chunks of the same accumulation.

@@ -38,7 +38,7 @@ EXPORTS = (
     "msf_selftest_wait_timeout", "msf_history_commit", "msf_mssa_forward_lse",
     "msf_mssa_backward", "msf_mssa_backward_simt", "msf_history_get", "msf_history_set",
     "msf_noalloc_device_status", "msf_noalloc_selftest_wait_timeout", "msf_patchify_tiers",
-    "msf_unpatchify_tier",
+    "msf_unpatchify_tier", "msf_patchify_resample",
 )
 
 
@@ -107,6 +107,7 @@ def _load():
         "msf_plan_bind": (ctypes.c_int, [P, VP, SZ, VP, VP, VP, VP]),
         "msf_patchify": (ctypes.c_int, [P, VP, ctypes.POINTER(VP), VP, VP]),
         "msf_unpatchify": (ctypes.c_int, [P, I32, VP, VP, VP, VP]),
+        "msf_patchify_resample": (ctypes.c_int, [P, VP, ctypes.POINTER(VP), VP, VP, VP, I32, VP]),
         "msf_kv_resample": (ctypes.c_int, [P, VP, VP, I32, VP]),
         "msf_mssa_forward": (ctypes.c_int, [P, VP, VP, VP, VP, VP]),
         "msf_mssa_forward_simt": (ctypes.c_int, [P, VP, VP, VP, VP, VP]),
@@ -209,6 +210,13 @@ def msf_patchify(plan: int, latent, w_tier: Optional[Sequence], tokens, stream=N
         arr = (ctypes.c_void_p * len(w_tier))(*[_ptr(w) for w in w_tier])
     _check(_lib.msf_patchify(plan, _ptr(latent), arr, _ptr(tokens), _stream(stream)),
            "msf_patchify")
+
+
+def msf_patchify_resample(plan: int, latent, w_tier: Sequence, tokens, k_win, v_win,
+                          flags: int = MSF_RESAMPLE_FULL, stream=None) -> None:
+    arr = (ctypes.c_void_p * len(w_tier))(*[_ptr(w) for w in w_tier])
+    _check(_lib.msf_patchify_resample(plan, _ptr(latent), arr, _ptr(tokens), _ptr(k_win), _ptr(v_win), flags,
+                                      _stream(stream)), "msf_patchify_resample")
 
 
 def msf_unpatchify(plan: int, position: int, tokens, w_out, latent_out, stream=None) -> None:
@@ -381,6 +389,9 @@ class Plan:
 
     def unpatchify(self, position, tokens, w_out, latent_out, stream=None):
         msf_unpatchify(self.handle, position, tokens, w_out, latent_out, stream)
+
+    def patchify_resample(self, latent, w_tier, tokens, k_win, v_win, flags=MSF_RESAMPLE_FULL, stream=None):
+        msf_patchify_resample(self.handle, latent, w_tier, tokens, k_win, v_win, flags, stream)
 
     def patchify_tiers(self, latent, tiers, tokens, stream=None):
         msf_patchify_tiers(self.handle, latent, tiers, tokens, stream)
