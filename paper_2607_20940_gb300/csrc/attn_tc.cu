@@ -334,6 +334,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int c = 0; c < C::kChunks; ++c)
                         ptx::tma_load_4d(sV + sv * C::kTileBytes + c * (kBlockN * 128),
                                          &maps.v[G.seg[seg].map], &v_full[sv], c * 64, pc.h, row, pc.b);
+                    if (js == 0) {
+                        // Cold start: every CTA asks HBM for its first tiles at
+                        // once. The ring's deeper tiles wait until Q has landed,
+                        // so the first tile's bytes are not queued behind them.
+                        if (!ptx::mbar_wait_bounded(&q_full, 0, abort_p, p.wait_limit)) {
+                            ok = false;
+                            ++js;  // tile 0's copies are in flight: drain them
+                            break;
+                        }
+                    }
                 }
                 ++piece;
             }
