@@ -939,24 +939,12 @@ extern "C" msf_status msf_unpatchify_tier(msf_plan_t plan, int32_t position, con
     char* codes = msf::tier_codes(p);
     msf::DeembedTier extra;
     if (tier->out_down) {
-        // codes = gamma * h A^T for the state's tokens (columns past r zero)
-        msf::GemmTcArgs g;
-        g.A = (const char*)tokens + (size_t)p.st_off[position] * E * 2;
-        g.B = tier->out_down;
-        g.C = codes + (size_t)p.st_off[position] * msf::kTierCodeCols * 2;
-        g.M = M;
-        g.N = msf::kTierCodeCols;
-        g.K = E;
-        g.lda = E;
-        g.ldb = E;
-        g.ldc = msf::kTierCodeCols;
-        g.a_bstride = (long long)p.N * E;
-        g.c_bstride = (long long)p.N * msf::kTierCodeCols;
-        g.status = msf::status_word(p);
-        g.alpha = tier->lora_scale;
-        g.b_rows = tier->lora_rank;
-        if (!msf::gemm_tc_supported(g)) return MSF_ERR_UNSUPPORTED;
-        cudaError_t e = msf::launch_gemm_tc(g, p.B, s);
+        // codes = gamma * h A^T for the state's tokens (columns past r zero),
+        // by the de-embedding's cluster split-K kernel with a row output
+        cudaError_t e = msf::launch_msp_rows_splitk(
+            tokens, (long long)p.N * E, p.N, p.st_off[position], tier->out_down, tier->lora_rank, M, E,
+            codes + (size_t)p.st_off[position] * msf::kTierCodeCols * 2, (long long)p.N * msf::kTierCodeCols,
+            msf::kTierCodeCols, tier->lora_scale, p.B, msf::status_word(p), s);
         if (e != cudaSuccess) return cuda_status(e);
         extra.codes = codes;
         extra.codes_bstride = (long long)p.N * msf::kTierCodeCols;
@@ -964,9 +952,9 @@ extern "C" msf_status msf_unpatchify_tier(msf_plan_t plan, int32_t position, con
         extra.rank = tier->lora_rank;
     }
     if (tier->residual) {
-        // the window's raw patch vectors; the state's block feeds the residual
+        // the state's raw patch vectors (its block of the raw layout) feed the residual
         char* raw = msf::msp_scratch(p);
-        cudaError_t e = msf::launch_patchify_raw(latent_in, raw, sh, p.B, true, s);
+        cudaError_t e = msf::launch_patchify_raw(latent_in, raw, sh, p.B, true, s, position, 1);
         if (e != cudaSuccess) return cuda_status(e);
         extra.xraw = raw + (size_t)position * per * 2;
         extra.xraw_bstride = (long long)p.T * per;

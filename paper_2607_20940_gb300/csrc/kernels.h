@@ -94,8 +94,10 @@ struct MspShape {
     int T, C, Hl, Wl, patch;
     int scales[MSF_MAX_STATES];
 };
+// Raw patchify of states [l0, l0 + n_states) (n_states < 0: to the end) into
+// their blocks of the [B, T, C*Hl*Wl] raw layout.
 cudaError_t launch_patchify_raw(const void* latent, void* raw, const MspShape& sh, int batch,
-                                bool bf16, cudaStream_t st);
+                                bool bf16, cudaStream_t st, int l0 = 0, int n_states = -1);
 cudaError_t launch_unpatchify_raw(const void* raw, void* latent, const MspShape& sh, int position,
                                   long long raw_bstride, int raw_offset, int batch, bool bf16,
                                   cudaStream_t st);

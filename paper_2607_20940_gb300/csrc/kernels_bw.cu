@@ -42,10 +42,10 @@ cudaError_t launch_pool(const PoolBatch& jobs, int batch, bool bf16, cudaStream_
 
 template <typename T>
 __global__ void __launch_bounds__(256) patchify_raw_kernel(const T* __restrict__ latent,
-                                                           T* __restrict__ raw, MspShape sh) {
+                                                           T* __restrict__ raw, MspShape sh, int l0) {
     ptx::grid_dep_wait();
     ptx::grid_dep_launch();
-    const int l = blockIdx.y, b = blockIdx.z;
+    const int l = l0 + (int)blockIdx.y, b = blockIdx.z;
     const int per = sh.C * sh.Hl * sh.Wl;
     const int o = blockIdx.x * blockDim.x + threadIdx.x;
     if (o >= per) return;
@@ -79,14 +79,15 @@ __global__ void __launch_bounds__(256) unpatchify_raw_kernel(const T* __restrict
 }
 
 cudaError_t launch_patchify_raw(const void* latent, void* raw, const MspShape& sh, int batch,
-                                bool bf16, cudaStream_t st) {
+                                bool bf16, cudaStream_t st, int l0, int n_states) {
     const int per = sh.C * sh.Hl * sh.Wl;
-    dim3 grid((unsigned)((per + 255) / 256), (unsigned)sh.T, (unsigned)batch);
+    if (n_states < 0) n_states = sh.T - l0;
+    dim3 grid((unsigned)((per + 255) / 256), (unsigned)n_states, (unsigned)batch);
     if (bf16)
         return launch_pdl(patchify_raw_kernel<__nv_bfloat16>, grid, dim3(256), 0, st,
-                          (const __nv_bfloat16*)latent, (__nv_bfloat16*)raw, sh);
+                          (const __nv_bfloat16*)latent, (__nv_bfloat16*)raw, sh, l0);
     return launch_pdl(patchify_raw_kernel<float>, grid, dim3(256), 0, st, (const float*)latent,
-                      (float*)raw, sh);
+                      (float*)raw, sh, l0);
 }
 
 cudaError_t launch_unpatchify_raw(const void* raw, void* latent, const MspShape& sh, int position,

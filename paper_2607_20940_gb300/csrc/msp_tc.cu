@@ -402,6 +402,13 @@ struct DeembedParams {
     int tok_row0;       // first token row of the position
     __nv_bfloat16* latent;  // [B, C, Hl, Wl]
     unsigned int* status;
+    // Row output instead of the latent scatter (NULL: scatter): row m of
+    // stream b, columns [0, F), at rows_out + b * rows_bstride + m * rows_ld,
+    // each value scaled by rows_scale before the one rounding.
+    __nv_bfloat16* rows_out;
+    long long rows_bstride;
+    int rows_ld;
+    float rows_scale;
 };
 struct DeembedMaps {
     CUtensorMap a;      // tokens {E, rows, B}
@@ -559,7 +566,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 acc.z += v.z;
                 acc.w += v.w;
             }
-            if (m < p.M) {
+            if (m < p.M && p.rows_out) {
+                const float sc = p.rows_scale;
+                uint2 v2;
+                v2.x = ptx::pack_bf16(sc * acc.x, sc * acc.y);
+                v2.y = ptx::pack_bf16(sc * acc.z, sc * acc.w);
+                *reinterpret_cast<uint2*>(p.rows_out + (size_t)b * p.rows_bstride + (size_t)m * p.rows_ld +
+                                          nt * kDeBN + 4 * c4) = v2;
+            } else if (m < p.M) {
                 const int i = m / p.gw, jj = m % p.gw;
                 __nv_bfloat16* lat =
                     p.latent + (size_t)b * p.C * plane + (size_t)(P * i) * p.Wl + (size_t)P * jj;
@@ -755,6 +769,48 @@ cudaError_t launch_msp_deembed(const void* tokens, long long tok_bstride_elems, 
     cudaError_t e = set_smem_attr((const void*)msp_deembed_kernel, kDeSmem);
     if (e != cudaSuccess) return e;
     const dim3 grid((unsigned)(p.m_tiles * (F / kDeBN)), (unsigned)splits, (unsigned)batch);
+    return launch_pdl_cluster(msp_deembed_kernel, grid, dim3(kThreads), kDeSmem, st, dim3(1, splits, 1), maps, p);
+}
+
+cudaError_t launch_msp_rows_splitk(const void* tokens, long long tok_bstride_elems, int tok_rows, int tok_row0,
+                                   const void* w, int w_rows, int M, int E, void* out, long long out_bstride,
+                                   int out_ld, float scale, int batch, unsigned int* status, cudaStream_t st) {
+    DeembedMaps maps;
+    memset(&maps, 0, sizeof(maps));
+    EncodeTiledFn enc = encoder();
+    if (!enc) return cudaErrorNotSupported;
+    {
+        cuuint64_t dims[3] = {(cuuint64_t)E, (cuuint64_t)tok_rows, (cuuint64_t)batch};
+        cuuint64_t strides[2] = {(cuuint64_t)E * 2, (cuuint64_t)tok_bstride_elems * 2};
+        cuuint32_t box[3] = {64, 128, 1};
+        cuuint32_t es[3] = {1, 1, 1};
+        if (enc(&maps.a, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(tokens), dims, strides, box, es,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+    }
+    if (!encode_2d(&maps.b, w, E, w_rows, (long long)E * 2, 64, kDeBN)) return cudaErrorInvalidValue;
+    const int nk_all = E / 64;
+    int splits = 8;
+    while (splits > 1 && splits > nk_all) splits /= 2;
+    DeembedParams p;
+    memset(&p, 0, sizeof(p));
+    p.M = M;
+    p.K = E;
+    p.nk_all = nk_all;
+    p.m_tiles = (M + 127) / 128;
+    p.splits = splits;
+    p.P = 1;
+    p.gw = 1;
+    p.tok_row0 = tok_row0;
+    p.status = status;
+    p.rows_out = (__nv_bfloat16*)out;
+    p.rows_bstride = out_bstride;
+    p.rows_ld = out_ld;
+    p.rows_scale = scale;
+    cudaError_t e = set_smem_attr((const void*)msp_deembed_kernel, kDeSmem);
+    if (e != cudaSuccess) return e;
+    const dim3 grid((unsigned)p.m_tiles, (unsigned)splits, (unsigned)batch);
     return launch_pdl_cluster(msp_deembed_kernel, grid, dim3(kThreads), kDeSmem, st, dim3(1, splits, 1), maps, p);
 }
 

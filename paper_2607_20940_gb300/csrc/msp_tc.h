@@ -65,4 +65,12 @@ cudaError_t launch_msp_deembed(const void* tokens, long long tok_bstride_elems, 
                                int batch, unsigned int* status, cudaStream_t st,
                                const DeembedTier* tier = nullptr);
 
+// The same cluster split-K kernel with a plain row output: out[b][m][0, 64)
+// = scale * sum_k tokens[b][tok_row0 + m][k] * w[n][k] for the 64 output
+// columns n (w has w_rows <= 64 rows; the others read as zeros), rounded once
+// to bf16; E a multiple of 64.
+cudaError_t launch_msp_rows_splitk(const void* tokens, long long tok_bstride_elems, int tok_rows, int tok_row0,
+                                   const void* w, int w_rows, int M, int E, void* out, long long out_bstride,
+                                   int out_ld, float scale, int batch, unsigned int* status, cudaStream_t st);
+
 }  // namespace msf
