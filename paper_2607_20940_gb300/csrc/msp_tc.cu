@@ -388,6 +388,7 @@ __global__ void __launch_bounds__(kThreads, 2)
 
 constexpr int kDeBN = 64;
 constexpr int kDeStages = 4;
+constexpr int kDeMaxSplits = 8;  // cluster size along the split (portable limit)
 constexpr int kDePartStride = kDeBN + 4;  // floats per staged row (padding spreads the banks)
 
 struct DeembedParams {
@@ -528,11 +529,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (ok) {
             ptx::tc_fence_after();
             const uint32_t taddr = tbase + ((uint32_t)((warp - 4) * 32) << 16);
+            uint32_t vb[kDeBN / 32][32];
+#pragma unroll
+            for (int c = 0; c < kDeBN / 32; ++c) ptx::tmem_ld32(taddr + c * 32, vb[c]);
+            ptx::tmem_wait_ld();
 #pragma unroll
             for (int c = 0; c < kDeBN / 32; ++c) {
-                uint32_t v[32];
-                ptx::tmem_ld32(taddr + c * 32, v);
-                ptx::tmem_wait_ld();
+                const uint32_t* v = vb[c];
                 float4* d4 = reinterpret_cast<float4*>(part + r * kDePartStride + c * 32);
 #pragma unroll
                 for (int e = 0; e < 8; ++e)
@@ -558,13 +561,20 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int row = split * R + q / per_row;
             const int c4 = q % per_row;
             const int m = mt * 128 + row;
+            // All splits' partials requested before the first add (remote
+            // shared-memory loads are independent), summed in split order.
+            float4 v[kDeMaxSplits];
+#pragma unroll
+            for (int sp = 0; sp < kDeMaxSplits; ++sp)
+                v[sp] = sp < p.splits ? ptx::ld_cluster_f4(part + row * kDePartStride + 4 * c4, (uint32_t)sp)
+                                      : make_float4(0.f, 0.f, 0.f, 0.f);
             float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-            for (int s = 0; s < p.splits; ++s) {
-                const float4 v = ptx::ld_cluster_f4(part + row * kDePartStride + 4 * c4, (uint32_t)s);
-                acc.x += v.x;
-                acc.y += v.y;
-                acc.z += v.z;
-                acc.w += v.w;
+#pragma unroll
+            for (int sp = 0; sp < kDeMaxSplits; ++sp) {
+                acc.x += v[sp].x;
+                acc.y += v[sp].y;
+                acc.z += v[sp].z;
+                acc.w += v[sp].w;
             }
             if (m < p.M && p.rows_out) {
                 const float sc = p.rows_scale;
