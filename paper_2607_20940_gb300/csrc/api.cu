@@ -733,6 +733,14 @@ extern "C" msf_status msf_patchify_resample(msf_plan_t plan, const void* latent,
         if (n_runs <= msf::kMaxGemmProblems) tiles += ((r.M + 127) / 128) * ((E + 255) / 256);
         l0 = l1;
     }
+    // Runs with the widest patch vectors (most K chunks, the longest tiles)
+    // first in the grid, so that the block scheduler starts them first.
+    for (int i = 1; i < n_runs; ++i)
+        for (int k = i; k > 0 && runs[k].K > runs[k - 1].K; --k) {
+            const msf::MspEmbedRun t = runs[k];
+            runs[k] = runs[k - 1];
+            runs[k - 1] = t;
+        }
     for (int r0 = 0; r0 < n_runs; r0 += msf::kMaxGemmProblems) {
         const int n = n_runs - r0 < msf::kMaxGemmProblems ? n_runs - r0 : msf::kMaxGemmProblems;
         if (!msf::msp_embed_supported(runs + r0, n, E)) return MSF_ERR_UNSUPPORTED;
@@ -743,8 +751,8 @@ extern "C" msf_status msf_patchify_resample(msf_plan_t plan, const void* latent,
     jb.mode = p.d.resample;
     add_window_jobs(p, k_win, v_win, with_hist, jb);
     // Pool CTAs per stream: one 256-thread block per 256 tasks, as the pool
-    // kernel launches them; they come first in the grid, and the embedding
-    // tiles take the slots they free.
+    // kernel launches them, after the embedding tiles in the grid (the
+    // longest tiles, those of the widest patch vectors, first).
     int max_n = 0;
     for (int k = 0; k < jb.n; ++k) max_n = jb.j[k].out_n > max_n ? jb.j[k].out_n : max_n;
     long long pool_ctas = ((long long)jb.n * max_n * (jb.row_vecs / 2) + 255) / 256;

@@ -143,8 +143,8 @@ struct EmbedParams {
     EmbedRun run[kMaxGemmProblems];
     int T, C, Hl, Wl, E;
     int n_tiles_n;  // 256-column tiles per 128-row tile: ceil(E / 256)
-    int n_embed_tiles;  // embedding tiles per stream
-    int pool_ctas;      // CTAs [0, pool_ctas) of a stream run the pyramid jobs; the rest embed
+    int n_embed_tiles;  // CTAs [0, n_embed_tiles) of a stream embed; the rest pool
+    int pool_ctas;      // CTAs per stream that run the pyramid jobs (0: none)
     int pool_tasks;     // vector-pair tasks per pyramid job
     const __nv_bfloat16* latent;  // [B, T, C, Hl, Wl]
     __nv_bfloat16* tokens;        // [B, N, E]
@@ -164,15 +164,18 @@ struct EmbedMaps {
 __global__ void __launch_bounds__(kThreads, 2)
     msp_embed_kernel(const __grid_constant__ EmbedMaps maps, const __grid_constant__ EmbedParams p,
                      const __grid_constant__ PoolBatch pool) {
-    if ((int)blockIdx.x < p.pool_ctas) {
-        // ---- K/V pyramid jobs in the first CTAs of the launch: the same
-        // per-thread pooling as pool_kernel, strided over the pool CTAs of
-        // this stream (the two parts read and write disjoint buffers).
+    if ((int)blockIdx.x >= p.n_embed_tiles) {
+        // ---- K/V pyramid jobs in the CTAs after the embedding tiles (the
+        // longest tiles, those of the runs with the most K chunks, come
+        // first): the same per-thread pooling as pool_kernel, one task per
+        // thread. The two parts read and write disjoint buffers; the block
+        // scheduler starts these CTAs in the slots the embedding leaves free
+        // and, as its short tiles finish, in theirs.
         ptx::grid_dep_wait();
         ptx::grid_dep_launch();
         const int stride = p.pool_ctas * kThreads;
         const int total = pool.n * p.pool_tasks;
-        for (int t = (int)blockIdx.x * kThreads + (int)threadIdx.x; t < total; t += stride)
+        for (int t = ((int)blockIdx.x - p.n_embed_tiles) * kThreads + (int)threadIdx.x; t < total; t += stride)
             pool_task<__nv_bfloat16>(pool, t / p.pool_tasks, blockIdx.z, t % p.pool_tasks);
         return;
     }
@@ -187,7 +190,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     __shared__ int abort_flag;
 
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-    const int tile = (int)blockIdx.x - p.pool_ctas;
+    const int tile = (int)blockIdx.x;
     int ri = 0;
     while (ri < p.n_runs - 1 && tile >= p.run[ri + 1].tile_base) ++ri;
     const EmbedRun& R = p.run[ri];
@@ -692,12 +695,12 @@ cudaError_t launch_msp_embed(const MspEmbedRun* runs, int n, const MspShape& sh,
     if (e != cudaSuccess) return e;
     p.n_embed_tiles = tiles;
     PoolBatch pb;
-    if (pool && pool->n > 0 && pool_ctas > 0) {
+    if (pool && pool->n > 0) {
         pb = *pool;
         int max_n = 0;
         for (int k = 0; k < pb.n; ++k) max_n = pb.j[k].out_n > max_n ? pb.j[k].out_n : max_n;
         p.pool_tasks = max_n * (pb.row_vecs / 2);
-        p.pool_ctas = pool_ctas;
+        p.pool_ctas = pool_ctas > 0 ? pool_ctas : 1;
     } else {
         memset(&pb, 0, sizeof(pb));
     }

@@ -33,9 +33,9 @@ struct MspEmbedRun {
 
 bool msp_embed_supported(const MspEmbedRun* runs, int n, int E);
 // Up to kMaxGemmProblems runs in one launch. With `pool` (bf16 jobs) the
-// same launch also runs those K/V pyramid jobs on `pool_ctas` extra CTAs per
-// stream: they read and write buffers the embedding does not touch, so the
-// two share the SMs of one wave instead of two launches.
+// same launch also runs those K/V pyramid jobs on `pool_ctas` more CTAs per
+// stream after the embedding tiles: they read and write buffers the
+// embedding does not touch, so the two share the SMs of one launch.
 cudaError_t launch_msp_embed(const MspEmbedRun* runs, int n, const MspShape& sh, int E, const void* latent,
                              void* tokens, long long tok_bstride, int batch, unsigned int* status,
                              cudaStream_t st, const PoolBatch* pool = nullptr, int pool_ctas = 0);
