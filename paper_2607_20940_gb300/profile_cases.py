@@ -5,6 +5,8 @@ synthetic inputs so that `ncu -k <kernel>` can capture it in isolation.
     python -m paper_2607_20940_gb300.profile_cases pool_fused  # pyramid + staged history head
     python -m paper_2607_20940_gb300.profile_cases embed    # MSP patchify + tier embedding
     python -m paper_2607_20940_gb300.profile_cases deembed  # de-embedding + unpatchify
+    python -m paper_2607_20940_gb300.profile_cases embed_pool  # embedding + pyramid, one launch
+    python -m paper_2607_20940_gb300.profile_cases tier     # coarse-tier modules (LoRA, residual)
     python -m paper_2607_20940_gb300.profile_cases backward # forward with lse + MSSA gradient
     python -m paper_2607_20940_gb300.profile_cases attention # MSSA forward, 480p layer
 
@@ -83,6 +85,51 @@ def run(case: str) -> None:
             torch.cuda.synchronize()
             assert plan.device_status() == msf.MSF_OK
             plan.close()
+    elif case == "embed_pool":
+        # the one-launch MSP embedding + window pyramid with the staged head
+        for w in (synth.LAYER_480P, synth.STREAM_480P):
+            plan, d, _ = _setup(w, embed=True, fused=True)
+            mi = synth.msp_inputs(w)
+            lat = mi["latent"].to(dev)
+            tiers = {s: mi["w_tier"][s].t().contiguous().to(dev) for s in set(w.scales)}
+            tok = torch.empty((w.batch, plan.info.n_tokens, w.embed_dim), dtype=torch.bfloat16, device=dev)
+            for _ in range(2):
+                flush.fill_(1)
+                plan.patchify_resample(lat, [tiers[s] for s in w.scales], tok, d["k_win"], d["v_win"],
+                                       msf.MSF_RESAMPLE_WINDOW_ONLY)
+            torch.cuda.synchronize()
+            assert plan.device_status() == msf.MSF_OK
+            plan.close()
+    elif case == "tier":
+        # coarse-tier modules: rank-32 LoRA on embedding and de-embedding, latent residual
+        w = synth.LAYER_480P
+        plan, d, _ = _setup(w, embed=True)
+        mi = synth.msp_inputs(w)
+        ti = synth.tier_inputs(w, 32)
+        lat = mi["latent"].to(dev)
+        keep, mods = [], {}
+        for s in sorted(set(w.scales)):
+            w_emb = mi["w_tier"][s].t().contiguous().to(dev)
+            if s == 1:
+                w_o = mi["w_out"].t().contiguous().to(dev)
+                mods[s] = msf.tier_module(w_emb, w_o)
+                keep += [w_emb, w_o]
+                continue
+            t = {k: (v.t().contiguous().to(dev) if torch.is_tensor(v) else v) for k, v in ti[s].items()}
+            mods[s] = msf.tier_module(w_emb, t["w_out"], embed_down=t["lora_a"], embed_up=t["lora_b"],
+                                      out_down=t["out_a"], out_up=t["out_b"], residual=t["residual"],
+                                      lora_rank=32, lora_scale=t["gamma"])
+            keep += [w_emb] + [v for v in t.values() if torch.is_tensor(v)]
+        tok = torch.empty((w.batch, plan.info.n_tokens, w.embed_dim), dtype=torch.bfloat16, device=dev)
+        lat_out = torch.empty((w.batch, w.latent_channels, w.grid_h * w.patch, w.grid_w * w.patch),
+                              dtype=torch.bfloat16, device=dev)
+        for _ in range(2):
+            flush.fill_(1)
+            plan.patchify_tiers(lat, [mods[s] for s in w.scales], tok)
+            plan.unpatchify_tier(2, tok, lat, mods[2], lat_out)
+        torch.cuda.synchronize()
+        assert plan.device_status() == msf.MSF_OK
+        plan.close()
     elif case == "attention":
         w = synth.LAYER_480P
         plan, d, _ = _setup(w)
@@ -112,8 +159,8 @@ def run(case: str) -> None:
         assert plan.device_status() == msf.MSF_OK
         plan.close()
     else:
-        raise SystemExit(f"unknown case {case!r}: pool, pool_fused, embed, deembed, backward or "
-                         "attention")
+        raise SystemExit(f"unknown case {case!r}: pool, pool_fused, embed, embed_pool, deembed, tier, "
+                         "backward or attention")
 
 
 if __name__ == "__main__":

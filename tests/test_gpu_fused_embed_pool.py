@@ -70,3 +70,40 @@ def test_fused_embed_pool_matches_separate_calls(name, w, fused_append, window_o
     for k in ("tok", "pyr", "ring_k", "ring_v", "out"):
         assert torch.equal(a[k], b[k]), (name, k)
     assert torch.isfinite(b["tok"].float()).all()
+
+
+def test_fused_embed_pool_with_more_runs_than_one_launch_holds():
+    """Six positions with six distinct tier-weight tensors make six runs:
+    the embedding goes out in two launches (at most four runs each) and the
+    pyramid jobs ride with the first; the result must still equal the two
+    separate calls bit for bit."""
+    m = msf()
+    w = dataclasses.replace(synth.THREE_SCALE, heads=2, embed_dim=256)
+    plan = m.Plan(m.make_desc(w.scales, w.grid_h, w.grid_w, w.heads, w.head_dim, w.sink_tokens,
+                              w.history_frames, w.history_capacity, batch=w.batch,
+                              latent_channels=w.latent_channels, patch=w.patch, embed_dim=w.embed_dim))
+    x = synth.attention_inputs(w, BF16, seed=5)
+    mi = synth.msp_inputs(w, BF16)
+    d = {k: v.cuda() for k, v in x.items()}
+    ws = plan.workspace()
+    plan.bind(ws, d["k_sink"], d["v_sink"], d["k_hist"], d["v_hist"])
+    lat = mi["latent"].cuda()
+    # one distinct copy of the tier weight per position
+    w_tier = [mi["w_tier"][s].t().contiguous().cuda().clone() for s in w.scales]
+    info = plan.info
+    pyr = int(info.pyramid_v_offset - info.pyramid_k_offset)
+    outs = []
+    for fused_call in (False, True):
+        tok = torch.full((w.batch, info.n_tokens, w.embed_dim), float("nan"), dtype=BF16, device="cuda")
+        ws[int(info.pyramid_k_offset):int(info.pyramid_k_offset) + 2 * pyr].zero_()
+        if fused_call:
+            plan.patchify_resample(lat, w_tier, tok, d["k_win"], d["v_win"], m.MSF_RESAMPLE_FULL)
+        else:
+            plan.patchify(lat, w_tier, tok)
+            plan.kv_resample(d["k_win"], d["v_win"], m.MSF_RESAMPLE_FULL)
+        torch.cuda.synchronize()
+        assert plan.device_status() == m.MSF_OK
+        outs.append((tok.cpu(), ws[int(info.pyramid_k_offset):int(info.pyramid_k_offset) + 2 * pyr].cpu()))
+    assert torch.equal(outs[0][0], outs[1][0])
+    assert torch.equal(outs[0][1], outs[1][1])
+    assert torch.isfinite(outs[1][0].float()).all()
