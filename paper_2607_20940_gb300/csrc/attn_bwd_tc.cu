@@ -297,17 +297,35 @@ __device__ __forceinline__ void dq_item(const BwdMaps& maps, const BwdTcParams& 
                 }
             }
         }
+        // Two probe points per tile. A tcgen05.mma holds its issuing thread
+        // about as long as the tensor pipe takes to run it, and only ~250
+        // cycles of work stay in flight after the last issue, so every
+        // barrier check here is pipe time: the probes of each point go out
+        // together, and the bounded waits run only if one is not ready.
         for (int j = 0; j < n && ok; ++j) {
-            ok = wait_all(&dp_free, (uint32_t)(j & 1));
+            const bool next = j + 1 < n, next2 = j + 2 < n;
+            {
+                const bool rd = ptx::mbar_try_wait(&dp_free, (uint32_t)(j & 1));
+                const bool rv = !next || ptx::mbar_try_wait(&v_full[(j + 1) & 1], (uint32_t)(((j + 1) >> 1) & 1));
+                if (!__all_sync(0xffffffffu, rd && rv))
+                    ok = wait_all(&dp_free, (uint32_t)(j & 1)) &&
+                         (!next || wait_all(&v_full[(j + 1) & 1], (uint32_t)(((j + 1) >> 1) & 1)));
+            }
             if (!ok) break;
-            if (j + 1 < n) {
-                ok = wait_all(&v_full[(j + 1) & 1], (uint32_t)(((j + 1) >> 1) & 1));
-                if (!ok) break;
+            if (next) {
                 ptx::tc_fence_after();
                 if (ptx::elect_one_sync()) issue_dp(j + 1);
                 __syncwarp();
             }
-            ok = wait_all(&ds_full, (uint32_t)(j & 1));
+            // dS_j, and K_{j+2} for the S two tiles ahead; if K has not
+            // landed yet, dQ_j goes first and S_{j+2} after its own wait.
+            bool k_ready;
+            {
+                const bool rs = ptx::mbar_try_wait(&ds_full, (uint32_t)(j & 1));
+                k_ready = !next2 || ptx::mbar_try_wait(&k_full[(j + 2) % 3], (uint32_t)(((j + 2) / 3) & 1));
+                k_ready = __all_sync(0xffffffffu, k_ready);
+                if (!__all_sync(0xffffffffu, rs)) ok = wait_all(&ds_full, (uint32_t)(j & 1));
+            }
             if (!ok) break;
             ptx::tc_fence_after();
             if (ptx::elect_one_sync()) {
@@ -318,9 +336,10 @@ __device__ __forceinline__ void dq_item(const BwdMaps& maps, const BwdTcParams& 
                                 kd + (uint64_t)(kk * (2048 >> 4)), idQ, (j > 0 || kk > 0) ? 1u : 0u);
                 ptx::mma_commit(&k_empty[j % 3]);
                 if (j + 1 == n) ptx::mma_commit(&dq_full);
+                if (next2 && k_ready) issue_s(j + 2);
             }
             __syncwarp();
-            if (j + 2 < n) {
+            if (next2 && !k_ready) {
                 ok = wait_all(&k_full[(j + 2) % 3], (uint32_t)(((j + 2) / 3) & 1));
                 if (!ok) break;
                 ptx::tc_fence_after();
@@ -580,12 +599,24 @@ __device__ __forceinline__ void dkdv_item(const BwdMaps& maps, const BwdTcParams
         for (int i = 0; i < nq && ok; ++i) {
             const int st = i & 1;
             const bool more = i + 1 < nq;
-            ok = wait_all(&pds_full[0], (uint32_t)(i & 1));
+            // P/dS of half 0 and the next query tile's Q/dO, probed together
+            // (each barrier check of this thread is pipe time); if Q/dO has
+            // not landed, half 0's dV/dK go first.
+            bool q_ready;
+            {
+                const bool rp = ptx::mbar_try_wait(&pds_full[0], (uint32_t)(i & 1));
+                q_ready = !more || ptx::mbar_try_wait(&qg_full[st ^ 1], (uint32_t)(((i + 1) >> 1) & 1));
+                q_ready = __all_sync(0xffffffffu, q_ready);
+                if (!__all_sync(0xffffffffu, rp)) ok = wait_all(&pds_full[0], (uint32_t)(i & 1));
+            }
             if (!ok) break;
             ptx::tc_fence_after();
-            if (ptx::elect_one_sync()) issue_kv(i, 0);
+            if (ptx::elect_one_sync()) {
+                issue_kv(i, 0);
+                if (more && q_ready) issue_st(i + 1, 0);
+            }
             __syncwarp();
-            if (more) {
+            if (more && !q_ready) {
                 ok = wait_all(&qg_full[st ^ 1], (uint32_t)(((i + 1) >> 1) & 1));
                 if (!ok) break;
                 ptx::tc_fence_after();
