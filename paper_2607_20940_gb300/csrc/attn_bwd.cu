@@ -274,56 +274,81 @@ __global__ void __launch_bounds__(128) bwd_dkdv_kernel(const BwdCommon c, const 
     }
 }
 
-// dk_win, dv_win: one warp per (stream, token, head) row; a lane holds D/32
-// consecutive elements (one vector load per entry). Entries of the token's
-// state come in a fixed order. Issuing every entry's loads before the first
-// add (fewer warps resident) measured slower than this loop.
+// dk_win, dv_win: one block per (stream, token); the token's rows of every
+// head are contiguous (H * D values), so each thread owns 8 consecutive
+// values of it and every entry's rows are whole coalesced spans, and the
+// entries of the token's state are decoded per block, not per head. Entries
+// are summed in their fixed order, two at a time with both entries' loads
+// issued before the adds, and the sum is rounded once.
 template <typename T, int D>
 __global__ void __launch_bounds__(256) bwd_gather_kernel(const BwdCommon c, const GatherArgs g,
                                                          T* __restrict__ dk, T* __restrict__ dv) {
     ptx::grid_dep_wait();
     ptx::grid_dep_launch();
-    constexpr int E = D / 32;
-    const long long w = (long long)blockIdx.x * 8 + threadIdx.x / 32;
-    const int lane = threadIdx.x % 32;
-    if (w >= (long long)c.B * c.N * c.H) return;
-    const int h = (int)(w % c.H);
-    const int t = (int)((w / c.H) % c.N);
-    const int b = (int)(w / ((long long)c.H * c.N));
+    const int t = (int)(blockIdx.x % (unsigned)c.N);
+    const int b = (int)(blockIdx.x / (unsigned)c.N);
     int l = 0;
     while (l + 1 < g.T && t >= g.st_off[l + 1]) ++l;
-    float ak[E], av[E];
-#pragma unroll
-    for (int e = 0; e < E; ++e) ak[e] = av[e] = 0.f;
-    for (int k = 0; k < g.n_ent[l]; ++k) {
+    const int ne = g.n_ent[l];
+    // context-gradient row and weight of entry k (row -1: a STRIDED entry
+    // whose pooled row does not start at this token)
+    auto decode = [&](int k, int& row, float& wgt) {
+        row = -1;
+        wgt = 0.f;
+        if (k >= ne) return;
         const GatherEntry& en = g.e[l][k];
-        int row;
-        float wgt = 1.f;
         if (en.sigma == 1) {
             row = en.crow0 + (t - en.dst0);
-        } else {
-            const int s = en.sigma, loc = t - en.dst0;
-            const int i = loc / en.src_gw, j = loc - (loc / en.src_gw) * en.src_gw;
-            if (g.mode == MSF_RESAMPLE_STRIDED) {
-                if (i % s || j % s) continue;
-            } else {
-                wgt = 1.0f / (float)(s * s);
-            }
-            row = en.crow0 + (i / s) * en.out_gw + j / s;
+            wgt = 1.f;
+            return;
         }
-        const size_t o = (((size_t)b * c.R + row) * c.H + h) * D + E * lane;
-        float xk[E], xv[E];
-        ldE<E>(c.dk_ctx + o, xk);
-        ldE<E>(c.dv_ctx + o, xv);
+        const int s = en.sigma, loc = t - en.dst0;
+        const int i = loc / en.src_gw, j = loc - i * en.src_gw;
+        if (g.mode == MSF_RESAMPLE_STRIDED && (i % s || j % s)) return;
+        row = en.crow0 + (i / s) * en.out_gw + j / s;
+        wgt = g.mode == MSF_RESAMPLE_STRIDED ? 1.f : 1.0f / (float)(s * s);
+    };
+    const int HD = c.H * D;
+    const size_t base = (size_t)b * c.R * HD;
+    for (int x = 8 * (int)threadIdx.x; x < HD; x += 8 * (int)blockDim.x) {
+        float ak[8], av[8];
 #pragma unroll
-        for (int e = 0; e < E; ++e) {
-            ak[e] = fmaf(wgt, xk[e], ak[e]);
-            av[e] = fmaf(wgt, xv[e], av[e]);
+        for (int e = 0; e < 8; ++e) ak[e] = av[e] = 0.f;
+        for (int k = 0; k < ne; k += 2) {
+            int r0, r1;
+            float w0, w1;
+            decode(k, r0, w0);
+            decode(k + 1, r1, w1);
+            float k0[8], v0[8], k1[8], v1[8];
+            if (r0 >= 0) {
+                ld8(c.dk_ctx + base + (size_t)r0 * HD + x, k0);
+                ld8(c.dv_ctx + base + (size_t)r0 * HD + x, v0);
+            }
+            if (r1 >= 0) {
+                ld8(c.dk_ctx + base + (size_t)r1 * HD + x, k1);
+                ld8(c.dv_ctx + base + (size_t)r1 * HD + x, v1);
+            }
+            if (r0 >= 0) {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    ak[e] = fmaf(w0, k0[e], ak[e]);
+                    av[e] = fmaf(w0, v0[e], av[e]);
+                }
+            }
+            if (r1 >= 0) {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    ak[e] = fmaf(w1, k1[e], ak[e]);
+                    av[e] = fmaf(w1, v1[e], av[e]);
+                }
+            }
         }
+        const size_t o = ((size_t)b * c.N + t) * HD + x;
+        stE<4>(dk + o, ak);
+        stE<4>(dk + o + 4, ak + 4);
+        stE<4>(dv + o, av);
+        stE<4>(dv + o + 4, av + 4);
     }
-    const size_t o = (((size_t)b * c.N + t) * c.H + h) * D + E * lane;
-    stE<E>(dk + o, ak);
-    stE<E>(dv + o, av);
 }
 
 }  // namespace
@@ -368,16 +393,20 @@ cudaError_t launch_bwd_dkdv_simt(const BwdCommon& c, const BwdGroup& g, bool bf1
 
 cudaError_t launch_bwd_gather(const BwdCommon& c, const GatherArgs& g, void* dk, void* dv,
                               bool bf16, cudaStream_t st) {
-    const long long rows = (long long)c.B * c.N * c.H;
-    dim3 grid((unsigned)((rows + 7) / 8));
+    const long long tokens = (long long)c.B * c.N;
+    if (tokens == 0) return cudaSuccess;
+    // one thread per 8 values of a token's H * D, in whole warps, at most 256
+    int threads = (c.H * c.D / 8 + 31) / 32 * 32;
+    if (threads > 256) threads = 256;
+    dim3 grid((unsigned)tokens);
     if (c.D == 128)
-        return bf16 ? launch_pdl(bwd_gather_kernel<__nv_bfloat16, 128>, grid, dim3(256), 0, st, c, g,
+        return bf16 ? launch_pdl(bwd_gather_kernel<__nv_bfloat16, 128>, grid, dim3(threads), 0, st, c, g,
                                  (__nv_bfloat16*)dk, (__nv_bfloat16*)dv)
-                    : launch_pdl(bwd_gather_kernel<float, 128>, grid, dim3(256), 0, st, c, g, (float*)dk,
+                    : launch_pdl(bwd_gather_kernel<float, 128>, grid, dim3(threads), 0, st, c, g, (float*)dk,
                                  (float*)dv);
-    return bf16 ? launch_pdl(bwd_gather_kernel<__nv_bfloat16, 64>, grid, dim3(256), 0, st, c, g,
+    return bf16 ? launch_pdl(bwd_gather_kernel<__nv_bfloat16, 64>, grid, dim3(threads), 0, st, c, g,
                              (__nv_bfloat16*)dk, (__nv_bfloat16*)dv)
-                : launch_pdl(bwd_gather_kernel<float, 64>, grid, dim3(256), 0, st, c, g, (float*)dk,
+                : launch_pdl(bwd_gather_kernel<float, 64>, grid, dim3(threads), 0, st, c, g, (float*)dk,
                              (float*)dv);
 }
 
