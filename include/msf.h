@@ -313,6 +313,20 @@ msf_status msf_kv_resample(msf_plan_t plan, const void* k_win, const void* v_win
 msf_status msf_mssa_forward(msf_plan_t plan, const void* q, const void* k_win, const void* v_win,
                             void* out, void* stream);
 
+/* msf_kv_resample(k_win, v_win, flags) and msf_mssa_forward in one launch
+ * (Eq. 4: the pyramid is built in the attention kernel's prologue): every CTA
+ * first pools its share of the pyramid (and, with fused_append, of the staged
+ * head), and a CTA's first tile of what that pooling writes (a pyramid
+ * segment; with fused_append also the history ring, which holds the staged
+ * head) waits (bounded) until every CTA's share is written; the pyramid, the
+ * staged head and out are
+ * exactly those of the two calls. fp32 plans run the two calls. flags:
+ * MSF_RESAMPLE_FULL or MSF_RESAMPLE_WINDOW_ONLY. Errors: INVALID_ARG,
+ * UNSUPPORTED (more pooling jobs than one launch takes), STATE (not bound),
+ * CUDA; a wait that gives up raises TIMEOUT in the device status. */
+msf_status msf_mssa_forward_resample(msf_plan_t plan, const void* q, const void* k_win,
+                                     const void* v_win, void* out, int32_t flags, void* stream);
+
 /* msf_mssa_forward that also writes, for every query row, the natural-log
  * log-sum-exp of its scaled scores over its context,
  *   lse[b, h, t] = ln sum_j exp(scale * q[b,t,h,:] . K_g[j]),

@@ -406,6 +406,31 @@ extern "C" msf_status msf_mssa_forward(msf_plan_t plan, const void* q, const voi
     return cuda_status(msf::launch_attn_simt(a, false, (cudaStream_t)stream));
 }
 
+extern "C" msf_status msf_mssa_forward_resample(msf_plan_t plan, const void* q, const void* k_win,
+                                                const void* v_win, void* out, int32_t flags, void* stream) {
+    if (!plan) return MSF_ERR_INVALID_ARG;
+    Plan& p = *plan;
+    msf_status st = check_attn_args(p, q, k_win, v_win, out);
+    if (st != MSF_OK) return st;
+    if (flags != MSF_RESAMPLE_FULL && flags != MSF_RESAMPLE_WINDOW_ONLY) return MSF_ERR_INVALID_ARG;
+    const bool with_hist = flags == MSF_RESAMPLE_FULL;
+    if (count_window_jobs(p, with_hist) > msf::kMaxPoolJobs) return MSF_ERR_UNSUPPORTED;
+    msf::PoolBatch jb;
+    memset(&jb, 0, sizeof(jb));
+    jb.row_vecs = (int)(row_bytes(p) / 16);
+    jb.mode = p.d.resample;
+    add_window_jobs(p, k_win, v_win, with_hist, jb);
+    msf::AttnArgs a;
+    build_attn_args(p, q, k_win, v_win, out, a);
+    cudaStream_t s = (cudaStream_t)stream;
+    if (p.elem == 2) return msf::launch_attn_tc(plan, a, s, &jb);
+    if (jb.n > 0) {
+        st = cuda_status(msf::launch_pool(jb, p.B, false, s));
+        if (st != MSF_OK) return st;
+    }
+    return cuda_status(msf::launch_attn_simt(a, false, s));
+}
+
 // Gradient rows of group gi: the context rows that come from the window,
 // each run with the window token its rows map back to (Eq. 4's Subsample
 // undone by the adjoint). Mirrors the context layout of build_attn_args.

@@ -43,6 +43,7 @@
 #include <string.h>
 
 #include "attn_tc.h"
+#include "pool.cuh"
 #include "ptx.cuh"
 
 namespace msf {
@@ -111,6 +112,15 @@ struct TcParams {
     long long t_sk;          // first sequence position of the stream-K part
     float* lse;              // optional [B, H, N] row log-sum-exp (natural log)
     int N;                   // query rows per stream
+    // The launch's own K/V pyramid (0 tasks: none): vector-pair tasks of the
+    // pool batch, pool_per_stream = jobs * pool_tasks per stream. pyr_sync[0]
+    // counts the CTAs whose share is written, pyr_sync[1] the CTAs that have
+    // finished; the last CTA to finish zeroes both.
+    long long pool_total;
+    int pool_per_stream;
+    int pool_tasks;
+    int pool_ring;  // the batch also writes the history ring (the staged head)
+    unsigned int* pyr_sync;
 };
 struct TcMaps {
     CUtensorMap q;
@@ -133,6 +143,12 @@ __device__ __forceinline__ float ex2(float x) {
     float y;
     asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
     return y;
+}
+
+__device__ __forceinline__ unsigned int ld_acquire(const unsigned int* p) {
+    unsigned int v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
 }
 
 // One piece of work: tiles [u0, u1) of one item.
@@ -204,9 +220,10 @@ __device__ __forceinline__ int slot_of(long long c, long long c1, long long item
     return 2 * (int)c + ((c == c1 && cta_begin(c, T, n) < item_start) ? 1 : 0);
 }
 
-template <int D>
-__global__ void __launch_bounds__(kThreads, 1)
-    mssa_tc_kernel(const __grid_constant__ TcMaps maps, const __grid_constant__ TcParams p) {
+// The kernel body; kPool: the launch also builds its K/V pyramid (`pool`),
+// compiled as its own kernel so that the plain attention carries none of it.
+template <int D, bool kPool>
+__device__ __forceinline__ void mssa_tc_body(const TcMaps& maps, const TcParams& p, const PoolBatch* pool) {
     using C = Cfg<D>;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -293,6 +310,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             long long js = 0;  // global K/V step
             int piece = 0;
             bool q_in_flight = false;
+            bool pyr_ready = !kPool || p.pool_total == 0;
             // K(j) and V(j) wait for one release: the commit that follows S1 of
             // tile j-2. It covers the last reader of K(j)'s slot (S of tile
             // j-2) and of V(j)'s slot in the 3-deep V ring (PV1 of tile j-3).
@@ -318,6 +336,24 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int u = pc.u0; u < pc.u1; ++u, ++js) {
                     int seg, row, valid;
                     tile_info(G, u, seg, row, valid);
+                    if (kPool && !pyr_ready &&
+                        (G.seg[seg].map >= kMapPyr0 || (p.pool_ring && G.seg[seg].map == kMapHist))) {
+                        // The first tile of this CTA that the launch's pooling
+                        // writes (a pyramid segment, or the history ring that
+                        // holds the staged head): every CTA's share is written
+                        // (their rows are read here through TMA, the async proxy).
+                        const long long w0 = clock64();
+                        while (ld_acquire(p.pyr_sync) < (unsigned int)ncta) {
+                            if (*abort_p || clock64() - w0 > p.wait_limit) {
+                                *abort_p = 1;
+                                ok = false;
+                                break;
+                            }
+                        }
+                        if (!ok) break;
+                        asm volatile("fence.proxy.async.global;" ::: "memory");
+                        pyr_ready = true;
+                    }
                     const CUtensorMap* mk = &maps.k[G.seg[seg].map];
                     const int st = (int)(js % kStages);
                     const uint32_t ph = (uint32_t)((js / kStages) & 1);
@@ -612,6 +648,27 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else {
         ptx::setmaxnreg_inc<kSoftmaxRegs>();
+        if (kPool && p.pool_total > 0) {
+            // =================== the launch's K/V pyramid ===================
+            // Eq. 4's Subsample of the window states (and the history, and the
+            // staged head) before the first softmax: the 256 softmax threads of
+            // every CTA take a strided share of the vector-pair tasks while the
+            // producer and the MMA issuer start on the first tiles. Only tiles
+            // of a pyramid segment wait for the count.
+            const int ti = (int)threadIdx.x - 128;
+            for (long long tk = (long long)blockIdx.x * 256 + ti; tk < p.pool_total;
+                 tk += (long long)gridDim.x * 256) {
+                const int b = (int)(tk / p.pool_per_stream);
+                const int rr = (int)(tk - (long long)b * p.pool_per_stream);
+                pool_task<__nv_bfloat16>(*pool, rr / p.pool_tasks, b, rr % p.pool_tasks);
+            }
+            // generic-proxy writes, read by other CTAs' TMA loads: proxy fence
+            // and GPU-scope fence by every writer, then one count per CTA
+            asm volatile("fence.proxy.async.global;" ::: "memory");
+            __threadfence();
+            ptx::named_bar_sync(1, 256);
+            if (threadIdx.x == 128) atomicAdd(p.pyr_sync, 1u);
+        }
         // ============================== softmax =============================
         const int t = (warp - 4) / 4;
         const int wq = warp % 4;
@@ -1024,6 +1081,28 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::tc_fence_after();
         ptx::tmem_dealloc(tbase, 512);
     }
+    if (kPool && p.pool_total > 0 && threadIdx.x == 0) {
+        // The last CTA to finish resets the pyramid counts for the next
+        // launch: no CTA of this one waits on them any more.
+        __threadfence();
+        if (atomicAdd(p.pyr_sync + 1, 1u) == (unsigned int)ncta - 1) {
+            atomicExch(p.pyr_sync, 0u);
+            atomicExch(p.pyr_sync + 1, 0u);
+        }
+    }
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    mssa_tc_kernel(const __grid_constant__ TcMaps maps, const __grid_constant__ TcParams p) {
+    mssa_tc_body<D, false>(maps, p, nullptr);
+}
+
+// The same attention with the launch's own pyramid (bf16 D = 128 plans).
+__global__ void __launch_bounds__(kThreads, 1)
+    mssa_tc_pool_kernel(const __grid_constant__ TcMaps maps, const __grid_constant__ TcParams p,
+                        const __grid_constant__ PoolBatch pool) {
+    mssa_tc_body<128, true>(maps, p, &pool);
 }
 
 // ---------------------------------------------------------------- host side
@@ -1073,7 +1152,7 @@ struct TcCache {
     const void* key_ptr[2 * kNumMaps + 1];
     int key_rows[2 * kNumMaps + 1];
     bool valid[2 * kNumMaps + 1];
-    bool attr_set[2];  // register count of the compiled kernel checked
+    bool attr_set[3];  // register count of the compiled kernel checked (D 64, D 128, D 128 + pool)
     int num_sms;
 };
 
@@ -1094,7 +1173,7 @@ void tc_cache_invalidate(msf_plan_t plan) {
     }
 }
 
-msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st) {
+msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st, const PoolBatch* pool) {
     Plan& P = *plan;
     if (!P.tc_cache) {
         P.tc_cache = calloc(1, sizeof(TcCache));
@@ -1221,8 +1300,46 @@ msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st) {
     if (tp.n_groups > 0) tp.dp_rounds = (int)(tp.g[0].n_items / ncta);
     tp.dp_stride = tp.g[0].n_virt;
     tp.t_sk = (long long)tp.dp_rounds * ncta * tp.dp_stride;
+    // The launch's own pyramid (D = 128): vector-pair tasks of every job and
+    // stream. Other head sizes run the pool kernel first.
+    const bool own_pool = pool && pool->n > 0 && P.D == 128;
+    if (pool && pool->n > 0 && !own_pool) {
+        e = launch_pool(*pool, P.B, true, st);
+        if (e != cudaSuccess) {
+            set_cuda_error((int)e);
+            return MSF_ERR_CUDA;
+        }
+    }
+    if (own_pool) {
+        int max_n = 0;
+        for (int k = 0; k < pool->n; ++k) max_n = pool->j[k].out_n > max_n ? pool->j[k].out_n : max_n;
+        tp.pool_tasks = max_n * (pool->row_vecs / 2);
+        tp.pool_per_stream = pool->n * tp.pool_tasks;
+        tp.pool_total = (long long)P.B * tp.pool_per_stream;
+        tp.pyr_sync = attn_pyr_sync(P);
+        for (int k = 0; k < pool->n; ++k)
+            if (pool->j[k].copy_k || pool->j[k].dst_k == P.k_hist) tp.pool_ring = 1;
+    }
 
-    if (P.D == 128) {
+    if (own_pool) {
+        if (!cache.attr_set[2]) {
+            cudaFuncAttributes fa;
+            e = cudaFuncGetAttributes(&fa, mssa_tc_pool_kernel);
+            if (e != cudaSuccess) {
+                set_cuda_error((int)e);
+                return MSF_ERR_CUDA;
+            }
+            if (fa.numRegs != kLaunchRegs) return MSF_ERR_UNSUPPORTED;
+            cache.attr_set[2] = true;
+        }
+        e = set_smem_attr((const void*)mssa_tc_pool_kernel, Cfg<128>::kSmem);
+        if (e != cudaSuccess) {
+            set_cuda_error((int)e);
+            return MSF_ERR_CUDA;
+        }
+        e = launch_pdl(mssa_tc_pool_kernel, dim3((unsigned)ncta), dim3(kThreads), Cfg<128>::kSmem, st,
+                       cache.maps, tp, *pool);
+    } else if (P.D == 128) {
         if (!cache.attr_set[1]) {
             // The warpgroup register split assumes exactly kLaunchRegs per thread.
             cudaFuncAttributes fa;

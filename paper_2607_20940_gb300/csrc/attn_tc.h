@@ -16,7 +16,11 @@ enum : int { kMapSink = 0, kMapHist = 1, kMapWin = 2, kMapPyr0 = 3 };
 constexpr int kMapPyr = -1;
 constexpr int kNumMaps = kMapPyr0 + MSF_MAX_GROUPS;
 
-msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st);
+// With `pool` (bf16 jobs), the launch also builds that K/V pyramid: every CTA
+// pools a share of it first, and tiles of pyramid segments wait until all
+// shares are written.
+msf_status launch_attn_tc(msf_plan_t plan, const AttnArgs& a, cudaStream_t st,
+                          const PoolBatch* pool = nullptr);
 // Tensor map of a [B, rows, H, D] bf16 tensor as 4-D {D, H, rows, B}, boxes of
 // 64 x 1 x 128 x 1 with 128-byte swizzle (one K-major MMA chunk); rows past
 // `rows` load as zeros.

@@ -78,8 +78,10 @@ inline size_t msp_scratch_bytes(const Plan& p) {
 // followed by [256 rows][2] fp32 (running max, running sum).
 constexpr int kAttnMaxCtas = 160;
 constexpr int kAttnBlockRows = 256;
+// After the counters, two words of a launch that builds its own pyramid
+// (CTAs whose pooled share is written, CTAs finished; reset by its last CTA).
 inline size_t attn_counter_bytes(const Plan& p) {
-    return p.elem == 2 ? round256((size_t)p.attn_items * 4) : 0;
+    return p.elem == 2 ? round256((size_t)p.attn_items * 4 + 8) : 0;
 }
 inline size_t attn_slot_floats(const Plan& p) { return (size_t)kAttnBlockRows * (p.D + 2); }
 inline size_t attn_partial_bytes(const Plan& p) {
@@ -130,6 +132,7 @@ inline char* msp_scratch(const Plan& p) {
 inline unsigned int* attn_counters(const Plan& p) {
     return (unsigned int*)(msp_scratch(p) + msp_scratch_bytes(p));
 }
+inline unsigned int* attn_pyr_sync(const Plan& p) { return attn_counters(p) + p.attn_items; }
 inline float* attn_partials(const Plan& p) {
     return (float*)((char*)attn_counters(p) + attn_counter_bytes(p));
 }

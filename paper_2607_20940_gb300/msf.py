@@ -38,7 +38,7 @@ EXPORTS = (
     "msf_selftest_wait_timeout", "msf_history_commit", "msf_mssa_forward_lse",
     "msf_mssa_backward", "msf_mssa_backward_simt", "msf_history_get", "msf_history_set",
     "msf_noalloc_device_status", "msf_noalloc_selftest_wait_timeout", "msf_patchify_tiers",
-    "msf_unpatchify_tier", "msf_patchify_resample",
+    "msf_unpatchify_tier", "msf_patchify_resample", "msf_mssa_forward_resample",
 )
 
 
@@ -111,6 +111,7 @@ def _load():
         "msf_kv_resample": (ctypes.c_int, [P, VP, VP, I32, VP]),
         "msf_mssa_forward": (ctypes.c_int, [P, VP, VP, VP, VP, VP]),
         "msf_mssa_forward_simt": (ctypes.c_int, [P, VP, VP, VP, VP, VP]),
+        "msf_mssa_forward_resample": (ctypes.c_int, [P, VP, VP, VP, VP, I32, VP]),
         "msf_history_append": (ctypes.c_int, [P, VP, VP, VP]),
         "msf_plan_device_status": (ctypes.c_int, [P, VP]),
         "msf_kernel_launches": (ctypes.c_uint64, []),
@@ -261,6 +262,12 @@ def msf_mssa_forward_simt(plan: int, q, k_win, v_win, out, stream=None) -> None:
                                       _stream(stream)), "msf_mssa_forward_simt")
 
 
+def msf_mssa_forward_resample(plan: int, q, k_win, v_win, out, flags: int = MSF_RESAMPLE_FULL,
+                              stream=None) -> None:
+    _check(_lib.msf_mssa_forward_resample(plan, _ptr(q), _ptr(k_win), _ptr(v_win), _ptr(out),
+                                          int(flags), _stream(stream)), "msf_mssa_forward_resample")
+
+
 def msf_history_append(plan: int, k_win, v_win, stream=None) -> None:
     _check(_lib.msf_history_append(plan, _ptr(k_win), _ptr(v_win), _stream(stream)),
            "msf_history_append")
@@ -404,6 +411,9 @@ class Plan:
 
     def mssa_forward(self, q, k_win, v_win, out, stream=None):
         msf_mssa_forward(self.handle, q, k_win, v_win, out, stream)
+
+    def mssa_forward_resample(self, q, k_win, v_win, out, flags=MSF_RESAMPLE_FULL, stream=None):
+        msf_mssa_forward_resample(self.handle, q, k_win, v_win, out, flags, stream)
 
     def mssa_forward_lse(self, q, k_win, v_win, out, lse, stream=None):
         msf_mssa_forward_lse(self.handle, q, k_win, v_win, out, lse, stream)
