@@ -145,8 +145,14 @@ def test_calls_before_bind_and_bad_pointers_fail_without_cuda():
     assert lib.msf_mssa_forward(p.handle, 4096, 8192, 12288, 16384, None) == msf.MSF_ERR_STATE
     assert lib.msf_kv_resample(p.handle, 4096, 8192, 0, None) == msf.MSF_ERR_STATE
     assert lib.msf_history_append(p.handle, 4096, 8192, None) == msf.MSF_ERR_STATE
+    assert lib.msf_mssa_forward_resample(p.handle, 4096, 8192, 12288, 16384, 0, None) == msf.MSF_ERR_STATE
     # null / misaligned
     assert lib.msf_mssa_forward(p.handle, None, 8192, 12288, 16384, None) == msf.MSF_ERR_INVALID_ARG
+    assert lib.msf_mssa_forward_resample(p.handle, None, 8192, 12288, 16384, 0, None) == \
+        msf.MSF_ERR_INVALID_ARG
+    assert lib.msf_mssa_forward_resample(p.handle, 4096, 8192, 12288, None, 0, None) == \
+        msf.MSF_ERR_INVALID_ARG
+    assert lib.msf_mssa_forward_resample(None, 4096, 8192, 12288, 16384, 0, None) == msf.MSF_ERR_INVALID_ARG
     assert lib.msf_plan_bind(p.handle, 4096, 16, 4096, 4096, 4096, 4096) == msf.MSF_ERR_WORKSPACE
     assert lib.msf_plan_bind(p.handle, 4097, 1 << 30, 4096, 4096, 4096, 4096) == msf.MSF_ERR_INVALID_ARG
     assert lib.msf_plan_index_map(p.handle, 7, None, 0, ctypes.byref(ctypes.c_size_t())) == \
