@@ -457,6 +457,30 @@ def other_configs(msf, synth, dev, flush, peaks, rank):
     plan.close()
     del ts_, ws_s, out_s
 
+    # ---- the window pyramid built in the attention launch's prologue
+    #      (msf_mssa_forward_resample) beside the pool launch + attention, at
+    #      the 480p layer with the fused history update (the step's plan)
+    plan, t = setup(wl, fused=True)
+    WO = msf.MSF_RESAMPLE_WINDOW_ONLY
+    plan.kv_resample(t["k_win"], t["v_win"], msf.MSF_RESAMPLE_FULL)
+
+    def two_launches():
+        plan.kv_resample(t["k_win"], t["v_win"], WO)
+        plan.mssa_forward(t["q"], t["k_win"], t["v_win"], t["out"])
+
+    two_ms = _timed(two_launches, flush, reps=9)
+    one_ms = _timed(lambda: plan.mssa_forward_resample(t["q"], t["k_win"], t["v_win"], t["out"], WO), flush,
+                    reps=9)
+    alone_ms = _timed(lambda: plan.mssa_forward(t["q"], t["k_win"], t["v_win"], t["out"]), flush, reps=9)
+    if plan.device_status() != msf.MSF_OK:
+        raise RuntimeError("device status error (resample in attention)")
+    out["resample_in_attention_480p"] = {
+        "workload": wl.name, "pool_launch_plus_attention_us": two_ms * 1e3,
+        "one_launch_us": one_ms * 1e3, "attention_alone_us": alone_ms * 1e3,
+        "note": "msf_mssa_forward_resample; the step uses the embedding + pyramid launch instead"}
+    plan.close()
+    del t
+
     # ---- training direction at the 480p layer: forward with the row
     #      log-sum-exp, then the MSSA gradient (dq, dk_win, dv_win)
     wl = synth.LAYER_480P

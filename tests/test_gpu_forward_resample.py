@@ -28,6 +28,7 @@ CASES = [
     ("three_scale", synth.THREE_SCALE),
     ("chunked", synth.CHUNKED_480P),
 ]
+STRIDED_CASES = [("small3", SMALL3), ("layer_480p", synth.LAYER_480P), ("three_scale", synth.THREE_SCALE)]
 
 
 def _pyramid(plan, ws, w):
@@ -70,6 +71,27 @@ def test_one_launch_equals_resample_then_forward(name, w, flags):
     stale_k, _ = _pyramid(plan, ws, w)
     assert not torch.equal(stale_k, pk_ref)
     got = _one_launch(plan, dx, fl)
+    torch.cuda.synchronize()
+    assert plan.device_status() == m.MSF_OK
+    pk, pv = _pyramid(plan, ws, w)
+    assert torch.equal(pk, pk_ref) and torch.equal(pv, pv_ref)
+    assert torch.equal(got, ref)
+    plan.close()
+
+
+@pytest.mark.parametrize("name,w", STRIDED_CASES, ids=[c[0] for c in STRIDED_CASES])
+def test_one_launch_strided_subsample(name, w):
+    """The literal stride-2 reading of Subsample (top-left token of each
+    block) through the one launch, against the two calls."""
+    m = msf()
+    x = synth.attention_inputs(w)
+    dx = device_inputs(x, w.history_capacity)
+    plan = make_plan(w, resample=m.MSF_RESAMPLE_STRIDED)
+    ws = bind(plan, dx)
+    ref = _two_calls(plan, dx, m.MSF_RESAMPLE_FULL)
+    pk_ref, pv_ref = _pyramid(plan, ws, w)
+    plan.kv_resample(dx["v_win"], dx["k_win"], m.MSF_RESAMPLE_FULL)
+    got = _one_launch(plan, dx, m.MSF_RESAMPLE_FULL)
     torch.cuda.synchronize()
     assert plan.device_status() == m.MSF_OK
     pk, pv = _pyramid(plan, ws, w)
