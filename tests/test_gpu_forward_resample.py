@@ -27,6 +27,8 @@ CASES = [
     ("stream_b4", dataclasses.replace(synth.STREAM_480P, history_frames=3)),
     ("three_scale", synth.THREE_SCALE),
     ("chunked", synth.CHUNKED_480P),
+    ("max_states", synth.Workload("fr_max_states_t16", 16, (1, 1, 2, 2, 4, 4, 8, 8) + (16,) * 8, 32, 48, 2,
+                                  64, 40, 2, 3, 2, 45)),
 ]
 STRIDED_CASES = [("small3", SMALL3), ("layer_480p", synth.LAYER_480P), ("three_scale", synth.THREE_SCALE)]
 

@@ -27,6 +27,10 @@ RAGGED = synth.Workload("ragged_t4_12x20", 4, (1, 1, 2, 4), 12, 20, 3, 128, 200,
 RAGGED64 = dataclasses.replace(RAGGED, name="ragged_d64", head_dim=64, scales=(1, 2, 2, 4), seed=22)
 COARSE_ONLY = synth.Workload("coarse_only", 3, (2, 2, 4), 16, 24, 2, 128, 37, 1, 1, 1, 23)
 NO_SINK = synth.Workload("no_sink_no_hist", 2, (1, 2), 16, 16, 2, 64, 0, 0, 0, 1, 24)
+# The plan's limits: MSF_MAX_STATES window states, five query groups (scales 1
+# to 16, coarse grids down to 2x3 tokens), 28 pooling jobs in one launch.
+MAX_STATES = synth.Workload("max_states_t16", 16, (1, 1, 2, 2, 4, 4, 8, 8) + (16,) * 8, 32, 48, 2, 64,
+                            40, 2, 3, 2, 25)
 
 
 def _run_attention(w, dtype, mode=0, simt=False):
@@ -45,7 +49,7 @@ def _run_attention(w, dtype, mode=0, simt=False):
     return x, out, plan
 
 
-@pytest.mark.parametrize("w", [synth.TINY, RAGGED, RAGGED64, COARSE_ONLY, NO_SINK],
+@pytest.mark.parametrize("w", [synth.TINY, RAGGED, RAGGED64, COARSE_ONLY, NO_SINK, MAX_STATES],
                          ids=lambda w: w.name)
 @pytest.mark.parametrize("mode", [0, 1], ids=["avg", "strided"])
 def test_attention_bf16_tensor_core(w, mode):
@@ -84,7 +88,7 @@ def test_attention_bf16_score_jumps(which, factor):
     assert mx <= 6e-2 and mean <= BF16_MEAN, (mx, mean)
 
 
-@pytest.mark.parametrize("w", [synth.TINY, RAGGED, RAGGED64, COARSE_ONLY], ids=lambda w: w.name)
+@pytest.mark.parametrize("w", [synth.TINY, RAGGED, RAGGED64, COARSE_ONLY, MAX_STATES], ids=lambda w: w.name)
 def test_attention_fp32(w):
     x, out, _ = _run_attention(w, F32, 0)
     ref = oracle_mssa(x, w, 0)
