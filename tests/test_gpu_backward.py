@@ -25,6 +25,10 @@ pytestmark = pytest.mark.gpu
 RAGGED = synth.Workload("ragged_t4_12x20", 4, (1, 1, 2, 4), 12, 20, 3, 128, 200, 2, 3, 2, 21)
 RAGGED64 = dataclasses.replace(RAGGED, name="ragged_d64", head_dim=64, scales=(1, 2, 2, 4), seed=22)
 COARSE_ONLY = synth.Workload("coarse_only", 3, (2, 2, 4), 16, 24, 2, 128, 37, 1, 1, 1, 23)
+# 16 window states in five query groups: a fine token's gradient gathers
+# entries from up to five groups (odd and even counts in the gather)
+MAX_STATES = synth.Workload("max_states_t16", 16, (1, 1, 2, 2, 4, 4, 8, 8) + (16,) * 8, 32, 48, 2, 64,
+                            40, 2, 3, 1, 26)
 
 
 def _dout(w, dtype, shape):
@@ -83,7 +87,7 @@ def _check(x, dout, lse, g, w, dtype, mode, heads=None):
         assert e.max() <= rel_max * scale and e.mean() <= rel_mean * scale, (name, e.max(), e.mean(), scale)
 
 
-@pytest.mark.parametrize("w", [synth.TINY, RAGGED, RAGGED64, COARSE_ONLY, synth.CHUNKED_SMALL],
+@pytest.mark.parametrize("w", [synth.TINY, RAGGED, RAGGED64, COARSE_ONLY, synth.CHUNKED_SMALL, MAX_STATES],
                          ids=lambda w: w.name)
 @pytest.mark.parametrize("mode", [0, 1], ids=["avg", "strided"])
 def test_backward_bf16(w, mode):
